@@ -1,0 +1,17 @@
+"""CPU oracle of the unified AI query: plain, slow, float64, obviously correct.
+
+TEST INFRASTRUCTURE ONLY.  The tests, ``__graft_entry__.smoke()`` and the
+benchmark's CPU-baseline leg are the only callers.  The product path (the
+CUDA library and its Python binding) never imports this package, and this
+package never imports the product.  Inputs come from the ``synth`` generator.
+
+Parity status per function:
+  relational.*            pinned (brute force, invariants, hand-worked cases)
+  transformer.rmsnorm     pinned (closed form on constant rows, torch rms_norm)
+  transformer.rope        pinned (rotation closed form, relative invariance)
+  transformer.causal_attention  pinned (torch SDPA, identical-key prefix mean)
+  transformer.label_logits      pinned (zero-weight bias closed form,
+                          identity-layer closed form, causality, GQA duplication)
+  whole-model numerics at random weights: parity unpinned beyond the
+                          component pins (the paper prints no model outputs).
+"""

@@ -1,0 +1,124 @@
+"""Pins of the oracle's relational half against hand-worked cases, brute force
+and invariants (CPU only)."""
+import operator
+import os
+
+import numpy as np
+import pytest
+
+from oracle import relational as rel
+from oracle import query as oq
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _read(name):
+    rows = {}
+    for line in open(os.path.join(GOLDEN, name)):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        k, *v = line.split()
+        rows.setdefault(k, []).append([int(x) if x.lstrip("-").isdigit() else float(x) for x in v])
+    return rows
+
+
+def test_where_and_hand_worked():
+    g = _read("where_and.txt")
+    cols = {"rating": np.array(g["rating"][0], np.int32), "year": np.array(g["year"][0], np.int32)}
+    mask = rel.predicate_mask(cols, [("rating", rel.GE, 4), ("year", rel.GE, 2000)], 10)
+    assert rel.compact(mask).tolist() == g["expect"][0]
+
+
+@pytest.mark.parametrize("op,pyop", [(rel.LT, operator.lt), (rel.LE, operator.le),
+                                     (rel.GT, operator.gt), (rel.GE, operator.ge),
+                                     (rel.EQ, operator.eq), (rel.NE, operator.ne)])
+def test_compare_ops_match_python(op, pyop):
+    vals = np.array([-3, 0, 2, 2, 7], np.int64)
+    got = rel.compare(vals, op, 2)
+    assert got.tolist() == [pyop(int(v), 2) for v in vals]
+
+
+@pytest.mark.parametrize("n", [0, 1, 31, 32, 33, 1000])
+def test_compaction_brute_force(n):
+    rng = np.random.default_rng(n)
+    cols = {"a": rng.integers(0, 10, n).astype(np.int32), "b": rng.integers(-5, 5, n).astype(np.int64)}
+    preds = [("a", rel.GE, 4), ("b", rel.NE, 0)]
+    ids = rel.compact(rel.predicate_mask(cols, preds, n))
+    brute = [i for i in range(n) if cols["a"][i] >= 4 and cols["b"][i] != 0]
+    assert ids.tolist() == brute
+    mask = rel.predicate_mask(cols, preds, n)
+    assert len(ids) == int(mask.sum())                      # size == popcount
+    assert np.all(np.diff(ids) > 0)                         # order preserved
+    assert rel.compact(np.zeros(n, bool)).size == 0          # nothing survives
+    assert rel.compact(np.ones(n, bool)).tolist() == list(range(n))  # everything
+
+
+def test_no_predicate_selects_all():
+    assert rel.predicate_mask({}, [], 5).all()
+
+
+def test_join_hand_worked():
+    g = _read("join_small.txt")
+    bkeys = np.array([m[1] for m in g["movie"]], np.int64)
+    byear = np.array([m[2] for m in g["movie"]], np.int32)
+    pkeys = np.array([r[1] for r in g["review"]], np.int64)
+    bm = rel.compact(rel.predicate_mask({"year": byear}, [("year", rel.GE, 2010)], len(bkeys)))
+    pr = np.arange(len(pkeys), dtype=np.int32)
+    want = [tuple(p) for p in g["pair"]]
+    assert rel.nested_loop_join(pkeys, pr, bkeys, bm) == want
+    assert rel.dict_join(pkeys, pr, bkeys, bm) == want
+
+
+@pytest.mark.parametrize("seed", range(5))
+def test_dict_join_equals_nested_loop_with_orphans_and_duplicates(seed):
+    rng = np.random.default_rng(seed)
+    bkeys = rng.integers(0, 30, 25).astype(np.int64)   # duplicate build keys too
+    pkeys = rng.integers(0, 40, 60).astype(np.int64)   # orphans (no match) and repeats
+    br = np.flatnonzero(rng.random(25) < 0.7).astype(np.int32)
+    pr = np.flatnonzero(rng.random(60) < 0.8).astype(np.int32)
+    nl = rel.nested_loop_join(pkeys, pr, bkeys, br)
+    assert rel.dict_join(pkeys, pr, bkeys, br) == nl
+    # cardinality closed form: sum over probe rows of matching build rows
+    card = sum(int(np.sum(bkeys[br] == pkeys[r])) for r in pr)
+    assert len(nl) == card
+
+
+def test_pack_layout():
+    prefix = np.array([7, 8], np.int32)
+    offsets = np.array([0, 3, 3 + 1, 3 + 1 + 2], np.int64)
+    tokens = np.array([1, 2, 3, 4, 5, 6], np.int32)
+    packed, cu, pos, last = rel.pack(prefix, offsets, tokens, np.array([0, 2], np.int32))
+    assert packed.tolist() == [7, 8, 1, 2, 3, 7, 8, 5, 6]
+    assert cu.tolist() == [0, 5, 9]
+    assert pos.tolist() == [0, 1, 2, 3, 4, 0, 1, 2, 3]
+    assert last.tolist() == [4, 8]
+    e = rel.pack(prefix, offsets, tokens, np.zeros(0, np.int32))
+    assert e[0].size == 0 and e[1].tolist() == [0] and e[3].size == 0
+
+
+def test_decide_strict_and_ties():
+    z = np.array([[1.0, 0.5], [0.5, 0.5], [-1.0, -2.0], [0.0, 1e-30]])
+    assert rel.decide(z).tolist() == [1, 0, 1, 0]          # strict >, tie -> no
+    z5 = np.array([[0, 3, 3, 1, 2], [5, 5, 5, 5, 5], [-1, -2, -3, -4, -0.5]], float)
+    assert rel.decide(z5).tolist() == [1, 0, 4]             # first index on ties
+
+
+def test_aggregate_invariants():
+    rng = np.random.default_rng(3)
+    s = 200
+    dec = rng.integers(0, 2, s).astype(np.int32)
+    cand = np.sort(rng.choice(10_000, s, replace=False)).astype(np.int32)
+    bro = rng.integers(0, 20, s).astype(np.int32)
+    bkeys = rng.integers(-100, 100, 20).astype(np.int64)
+    a = oq.aggregate(oq.AGG_ROW_IDS, dec, cand, 2)
+    assert a["count"] == len(a["row_ids"]) == int(dec.sum())
+    assert np.all(np.diff(a["row_ids"]) > 0)
+    g = oq.aggregate(oq.AGG_GROUP_BUILD_KEY, dec, cand, 2, bro, bkeys)
+    assert int(g["group_counts"].sum()) == g["count"]       # groups sum to yes count
+    assert np.all(g["group_counts"] > 0)                   # non-empty groups only
+    assert np.all(np.diff(g["group_build_rows"]) > 0)       # ascending build row
+    assert g["group_keys"].tolist() == bkeys[g["group_build_rows"]].tolist()
+    dec5 = rng.integers(0, 5, s).astype(np.int32)
+    lc = oq.aggregate(oq.AGG_GROUP_LABEL, dec5, cand, 5)["label_counts"]
+    assert lc.sum() == s and lc.tolist() == [int(np.sum(dec5 == k)) for k in range(5)]
