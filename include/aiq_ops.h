@@ -1,0 +1,63 @@
+/* aiq_ops.h - step-level C-ABI of libaiq.so: the prefill kernels one at a time.
+ *
+ * These entry points run one step of the query's prefill on caller-owned
+ * DEVICE buffers (plain device pointers, element counts), on the context's
+ * stream, and synchronise before returning.  They exist so that each kernel
+ * can be checked on its own; the whole query uses the same kernels through
+ * aiq_run_select / aiq_run_join_select.  All return aiq_status; a kernel's
+ * own check (fp16 overflow, an expired bounded wait) gives
+ * AIQ_ERR_DEVICE_CHECK.  The caller keeps ownership of every buffer.
+ */
+#ifndef AIQ_OPS_H
+#define AIQ_OPS_H
+
+#include <stdint.h>
+
+#include "aiq.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  AIQ_EPI_F16 = 0,       /* out fp16 [M, N] = A B^T */
+  AIQ_EPI_ROPE_F16 = 1,  /* as F16, then rotary embedding on columns < rope_cols */
+  AIQ_EPI_RESID_F32 = 2, /* out fp32 [M, N] += A B^T (residual stream update) */
+  AIQ_EPI_SWIGLU_F16 = 3 /* B rows interleave gate/up blocks of bn/2: out fp16 [M, N/2] = silu(g) * u */
+} aiq_epilogue;
+
+/* A decoder linear layer on the tensor cores: A fp16 [M, K] (row pitch lda
+ * elements) times B fp16 [N, K] (row pitch ldb; nn.Linear [out, in] layout),
+ * fp32 accumulation, then the epilogue.  bn = 128 or 256 is the output tile
+ * width: N % bn == 0, K % 64 == 0, rows 16-byte aligned.
+ * ROPE: `positions` int32 [M] (device), `rope_cos`/`rope_sin` fp32
+ * [max_pos, head_dim/2] (see aiq_op_rope_table); pairs (i, i + head_dim/2) of
+ * each head starting below rope_cols are rotated (the q and k heads of a
+ * fused QKV output).  SwiGLU MLP and rotary embeddings follow the decoder
+ * reading stated in aiq_model_config. */
+aiq_status aiq_op_gemm(aiq_ctx* ctx, const void* A, int64_t lda, const void* B, int64_t ldb, int32_t M, int32_t N,
+                       int32_t K, int32_t bn, int32_t epilogue, void* out, int64_t ldo, const int32_t* positions,
+                       const float* rope_cos, const float* rope_sin, int32_t rope_cols, int32_t head_dim);
+
+/* cos/sin of pos * theta^(-2i/head_dim), i < head_dim/2, pos < max_pos, computed
+ * in fp64 and stored fp32 [max_pos, head_dim/2] (device). */
+aiq_status aiq_op_rope_table(aiq_ctx* ctx, float* rope_cos, float* rope_sin, int32_t max_pos, int32_t head_dim,
+                             float theta);
+
+/* out fp16 [T, d] = x / sqrt(mean(x^2) + eps) * g, x fp32 [T, d], g bf16 [d]. */
+aiq_status aiq_op_rmsnorm(aiq_ctx* ctx, const float* x, int64_t T, int32_t d, const uint16_t* g, float eps,
+                          void* out);
+
+/* Causal grouped-query attention over a packed variable-length batch.
+ * qkv fp16 [T, (Hq + 2 Hkv) * hd]: q heads, then k heads, then v heads, with
+ * rotary embeddings already applied.  seq_start int32 [n_seqs + 1] (device):
+ * sequence i occupies rows [seq_start[i], seq_start[i+1]); seq_start[n_seqs]
+ * = T.  Query head h reads key/value head h / (Hq / Hkv).  out fp16
+ * [T, Hq * hd].  hd in {32, 64, 128}. */
+aiq_status aiq_op_attention(aiq_ctx* ctx, const void* qkv, int64_t T, const int32_t* seq_start, int32_t n_seqs,
+                            int32_t Hq, int32_t Hkv, int32_t hd, void* out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* AIQ_OPS_H */

@@ -1,0 +1,1169 @@
+// C-ABI of the unified AI-query library: contexts, device-resident tables and
+// models, the query planner and the step-level ops.
+//
+// A query is one pipeline on one CUDA stream (the paper's single compiled
+// program, Section 3): predicate + compaction (+ hash join), token packing,
+// chunked decoder prefill, label-logit decision, masked aggregate.  The host
+// reads back only control scalars between phases (survivor count, token
+// count, the chunk table) and the final results; no intermediate array
+// crosses PCIe (Section 3.3, H2D boundary consolidation).
+#include <algorithm>
+#include <cstdlib>
+#include <cstring>
+#include <map>
+#include <string>
+#include <vector>
+
+#include "aiq.h"
+#include "aiq_ops.h"
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace aiq;
+
+namespace {
+
+thread_local std::string g_err;
+
+aiq_status fail(aiq_status st, const std::string& msg) {
+  g_err = msg;
+  return st;
+}
+
+#define CUDA_TRY(x)                                                                         \
+  do {                                                                                      \
+    cudaError_t e_ = (x);                                                                   \
+    if (e_ != cudaSuccess) {                                                                \
+      cudaGetLastError();                                                                   \
+      return fail(AIQ_ERR_CUDA, std::string(#x) + ": " + cudaGetErrorString(e_));          \
+    }                                                                                       \
+  } while (0)
+
+#define AIQ_TRY(x)                 \
+  do {                             \
+    aiq_status s_ = (x);           \
+    if (s_ != AIQ_OK) return s_;   \
+  } while (0)
+
+struct DevBuf {
+  void* p = nullptr;
+  size_t bytes = 0;
+};
+
+struct ColD {
+  std::string name;
+  int32_t type = 0;
+  void* data = nullptr;
+  int64_t* offsets = nullptr;
+  size_t bytes = 0;
+  int64_t max_len = 0;   // TOKENS: longest row
+  int64_t max_id = -1;   // TOKENS: largest token id
+};
+
+struct TableD {
+  int64_t n_rows = 0;
+  std::vector<ColD> cols;
+};
+
+struct LayerD {
+  uint16_t* attn_norm = nullptr;
+  uint16_t* mlp_norm = nullptr;
+  __half* wqkv = nullptr;  // [(Hq + 2 Hkv) hd, d]
+  __half* wo = nullptr;    // [d, Hq hd]
+  __half* wgu = nullptr;   // [2 f, d], gate/up interleaved in blocks of bn_gu / 2 rows
+  __half* wd = nullptr;    // [d, f]
+};
+
+struct ModelD {
+  aiq_model_config cfg{};
+  uint16_t* embed = nullptr;
+  uint16_t* final_norm = nullptr;
+  uint16_t* lm_head = nullptr;
+  uint16_t* lm_bias = nullptr;
+  std::vector<LayerD> layers;
+  std::vector<DevBuf> allocs;
+  int bn_qkv = 128, bn_o = 128, bn_gu = 128, bn_d = 128;
+  DevBuf rope_cos, rope_sin;
+  int rope_max_pos = 0;
+  double linear_flops_per_token = 0;
+};
+
+struct ResultH {
+  aiq_result_view v{};
+  std::vector<int32_t> row_ids, group_rows, cand_ids, cand_build, decisions;
+  std::vector<int64_t> group_keys, group_counts, label_counts;
+  std::vector<float> logits;
+};
+
+struct ProfRec {
+  const char* name;
+  cudaEvent_t a, b;
+  double flops, bytes;
+};
+
+struct StatAcc {
+  int64_t launches = 0;
+  double ms = 0, flops = 0, bytes = 0;
+};
+
+}  // namespace
+
+struct aiq_ctx {
+  int device = 0;
+  int num_sms = 0;
+  cudaStream_t stream = nullptr;
+  int* d_err = nullptr;
+  int64_t* h_pin = nullptr;  // pinned staging for control scalars
+  size_t bytes_max = SIZE_MAX;
+  size_t bytes_used = 0;
+  int64_t next_handle = 1;
+  std::map<int64_t, TableD> tables;
+  std::map<int64_t, ModelD> models;
+  std::map<int64_t, ResultH> results;
+  std::map<std::string, DevBuf> ws;
+  int64_t token_budget = 131072;
+  bool profile = false;
+  std::vector<ProfRec> prof;
+  std::vector<cudaEvent_t> ev_pool;
+  std::map<std::string, StatAcc> stats;
+  std::vector<std::string> stat_names;
+  int64_t launches = 0;  // kernels launched by the current query
+};
+
+namespace {
+
+// ------------------------------------------------------------ allocation ---
+
+aiq_status dalloc(aiq_ctx* c, void** p, size_t bytes) {
+  bytes = std::max<size_t>(bytes, 256);
+  if (c->bytes_used + bytes > c->bytes_max)
+    return fail(AIQ_ERR_OOM, "device byte cap AIQ_DEVICE_BYTES_MAX exceeded (" + std::to_string(c->bytes_used + bytes) +
+                                 " > " + std::to_string(c->bytes_max) + ")");
+  cudaError_t e = cudaMalloc(p, bytes);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    *p = nullptr;
+    return fail(AIQ_ERR_OOM, std::string("cudaMalloc(") + std::to_string(bytes) + "): " + cudaGetErrorString(e));
+  }
+  c->bytes_used += bytes;
+  return AIQ_OK;
+}
+
+void dfree(aiq_ctx* c, void* p, size_t bytes) {
+  if (!p) return;
+  cudaFree(p);
+  c->bytes_used -= std::max<size_t>(bytes, 256);
+}
+
+// Grow-only named workspace buffer.
+template <typename T>
+aiq_status ws(aiq_ctx* c, const char* name, size_t count, T** out) {
+  size_t bytes = std::max<size_t>(count * sizeof(T), 256);
+  DevBuf& b = c->ws[name];
+  if (b.bytes < bytes) {
+    if (b.p) {
+      cudaStreamSynchronize(c->stream);
+      dfree(c, b.p, b.bytes);
+      b.p = nullptr;
+      b.bytes = 0;
+    }
+    size_t want = bytes + bytes / 4;
+    void* p = nullptr;
+    if (dalloc(c, &p, want) != AIQ_OK) AIQ_TRY(dalloc(c, &p, want = bytes));
+    b.p = p;
+    b.bytes = want;
+  }
+  *out = static_cast<T*>(b.p);
+  return AIQ_OK;
+}
+
+aiq_status sync_and_check(aiq_ctx* c) {
+  CUDA_TRY(cudaGetLastError());
+  CUDA_TRY(cudaStreamSynchronize(c->stream));
+  int err = 0;
+  CUDA_TRY(cudaMemcpy(&err, c->d_err, sizeof(int), cudaMemcpyDeviceToHost));
+  if (err) {
+    CUDA_TRY(cudaMemset(c->d_err, 0, sizeof(int)));
+    if (err & (DEVERR_DUP_BUILD_KEY | DEVERR_SENTINEL_KEY))
+      return fail(AIQ_ERR_INVALID_ARG, "join build keys must be unique and differ from INT64_MIN");
+    if (err & DEVERR_HASH_FULL) return fail(AIQ_ERR_CAPACITY, "hash table probe sequence exhausted");
+    if (err & DEVERR_TIMEOUT) return fail(AIQ_ERR_DEVICE_CHECK, "a kernel's bounded wait expired");
+    if (err & DEVERR_FP16_RANGE) return fail(AIQ_ERR_DEVICE_CHECK, "an activation left the fp16 range (or was NaN)");
+    return fail(AIQ_ERR_DEVICE_CHECK, "device check failed (code " + std::to_string(err) + ")");
+  }
+  return AIQ_OK;
+}
+
+// Reads `n` int64 values from the device after synchronising the stream.
+aiq_status read_i64(aiq_ctx* c, const int64_t* dev, int64_t n, int64_t* host) {
+  CUDA_TRY(cudaMemcpyAsync(host, dev, n * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream));
+  return sync_and_check(c);
+}
+
+// ------------------------------------------------------------- profiling ---
+
+cudaEvent_t take_event(aiq_ctx* c) {
+  if (!c->ev_pool.empty()) {
+    cudaEvent_t e = c->ev_pool.back();
+    c->ev_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e;
+  cudaEventCreate(&e);
+  return e;
+}
+
+struct ProfScope {
+  aiq_ctx* c;
+  const char* name;
+  double flops, bytes;
+  cudaEvent_t a = nullptr;
+  ProfScope(aiq_ctx* c_, const char* n, double f, double b) : c(c_), name(n), flops(f), bytes(b) {
+    if (c->profile) {
+      a = take_event(c);
+      cudaEventRecord(a, c->stream);
+    }
+  }
+  ~ProfScope() {
+    if (c->profile) {
+      cudaEvent_t b2 = take_event(c);
+      cudaEventRecord(b2, c->stream);
+      c->prof.push_back({name, a, b2, flops, bytes});
+    }
+  }
+};
+
+void collect_profile(aiq_ctx* c) {
+  if (c->prof.empty()) return;
+  cudaStreamSynchronize(c->stream);
+  for (auto& r : c->prof) {
+    float ms = 0;
+    cudaEventElapsedTime(&ms, r.a, r.b);
+    StatAcc& s = c->stats[r.name];
+    s.launches += 1;
+    s.ms += ms;
+    s.flops += r.flops;
+    s.bytes += r.bytes;
+    c->ev_pool.push_back(r.a);
+    c->ev_pool.push_back(r.b);
+  }
+  c->prof.clear();
+}
+
+inline void counted(aiq_ctx* c, int n) { c->launches += n; }
+
+aiq_status gemm(aiq_ctx* c, const char* name, const __half* A, int64_t lda, const __half* B, int64_t ldb, int M, int N,
+                int K, int bn, const GemmEpilogue& ep) {
+  const double out_bytes = (ep.kind == EPI_RESID_F32 ? 8.0 : (ep.kind == EPI_SWIGLU_F16 ? 1.0 : 2.0)) * M * N;
+  ProfScope ps(c, name, 2.0 * M * N * K, 2.0 * (double(M) * K + double(N) * K) + out_bytes);
+  int e = gemm_f16_tcgen05(A, lda, B, ldb, M, N, K, bn, ep, c->num_sms, c->stream);
+  if (M > 0) counted(c, 1);
+  if (e != 0)
+    return fail(AIQ_ERR_CUDA, std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(static_cast<cudaError_t>(e)));
+  return AIQ_OK;
+}
+
+// ------------------------------------------------------------ validation ---
+
+aiq_status make_pred_set(const TableD& t, const aiq_pred* preds, int32_t n, PredSet* ps) {
+  if (n < 0 || n > kMaxPreds) return fail(AIQ_ERR_INVALID_ARG, "n_preds must be 0..8");
+  if (n > 0 && !preds) return fail(AIQ_ERR_INVALID_ARG, "preds is NULL");
+  ps->n = n;
+  for (int i = 0; i < n; ++i) {
+    const aiq_pred& p = preds[i];
+    if (p.column < 0 || p.column >= static_cast<int32_t>(t.cols.size()))
+      return fail(AIQ_ERR_INVALID_ARG, "predicate column index out of range");
+    const ColD& col = t.cols[p.column];
+    if (col.type == AIQ_TOKENS) return fail(AIQ_ERR_INVALID_ARG, "predicate on a TOKENS column");
+    if (p.op < AIQ_LT || p.op > AIQ_NE) return fail(AIQ_ERR_INVALID_ARG, "unknown comparison operator");
+    ps->p[i] = PredDev{col.data, col.type, p.op, p.ivalue, p.fvalue};
+  }
+  return AIQ_OK;
+}
+
+ResultH& new_result(aiq_ctx* c, aiq_result_h* out) {
+  const int64_t h = c->next_handle++;
+  *out = h;
+  return c->results[h];
+}
+
+// ----------------------------------------------------- relational phase ---
+
+// Predicate (+ probe) over `t`, compaction into ids (and payload).  Returns S.
+aiq_status filter_compact(aiq_ctx* c, const TableD& t, const PredSet& ps, const ProbeSpec& probe, const char* tag,
+                          int64_t* S_out, int32_t** ids_out, int32_t** payload_out) {
+  const int64_t n = t.n_rows;
+  const int64_t nb = (n + kRowsPerBlock - 1) / kRowsPerBlock;
+  std::string b = tag;
+  uint32_t* bits;
+  int32_t* bcnt;
+  int64_t* boff;
+  AIQ_TRY(ws(c, (b + ".bits").c_str(), std::max<int64_t>(nb, 1) * (kRowsPerBlock / 32), &bits));
+  AIQ_TRY(ws(c, (b + ".bcnt").c_str(), std::max<int64_t>(nb, 1), &bcnt));
+  AIQ_TRY(ws(c, (b + ".boff").c_str(), nb + 1, &boff));
+  ProbeSpec pr = probe;
+  if (pr.keys) {
+    AIQ_TRY(ws(c, (b + ".match").c_str(), std::max<int64_t>(n, 1), &pr.match_out));
+  }
+  {
+    ProfScope p(c, "predicate_mask", 0, 0);
+    launch_predicate_mask(ps, pr, n, bits, bcnt, c->d_err, c->stream);
+    launch_scan_counts(bcnt, nb, boff, c->stream);
+    counted(c, (n > 0) + 1);
+  }
+  AIQ_TRY(read_i64(c, boff + nb, 1, c->h_pin));
+  const int64_t S = c->h_pin[0];
+  int32_t* ids;
+  AIQ_TRY(ws(c, (b + ".ids").c_str(), std::max<int64_t>(S, 1), &ids));
+  int32_t* pay = nullptr;
+  if (pr.keys) AIQ_TRY(ws(c, (b + ".payload").c_str(), std::max<int64_t>(S, 1), &pay));
+  {
+    ProfScope p(c, "compact", 0, 0);
+    launch_compact(bits, boff, n, ids, pr.match_out, pay, c->stream);
+    counted(c, n > 0);
+  }
+  *S_out = S;
+  *ids_out = ids;
+  if (payload_out) *payload_out = pay;
+  return AIQ_OK;
+}
+
+// --------------------------------------------------------- prefill phase ---
+
+aiq_status ensure_rope(aiq_ctx* c, ModelD& m, int max_pos) {
+  if (m.rope_max_pos >= max_pos) return AIQ_OK;
+  const int want = std::max(max_pos, 2048);
+  const size_t bytes = static_cast<size_t>(want) * (m.cfg.head_dim / 2) * sizeof(float);
+  if (m.rope_cos.p) {
+    CUDA_TRY(cudaStreamSynchronize(c->stream));
+    dfree(c, m.rope_cos.p, m.rope_cos.bytes);
+    dfree(c, m.rope_sin.p, m.rope_sin.bytes);
+    m.rope_cos = m.rope_sin = DevBuf{};
+    m.rope_max_pos = 0;
+  }
+  AIQ_TRY(dalloc(c, &m.rope_cos.p, bytes));
+  m.rope_cos.bytes = bytes;
+  AIQ_TRY(dalloc(c, &m.rope_sin.p, bytes));
+  m.rope_sin.bytes = bytes;
+  launch_rope_table(static_cast<float*>(m.rope_cos.p), static_cast<float*>(m.rope_sin.p), want, m.cfg.head_dim,
+                    m.cfg.rope_theta, c->stream);
+  counted(c, 1);
+  m.rope_max_pos = want;
+  return AIQ_OK;
+}
+
+struct PrefillBufs {
+  int32_t *tok, *pos, *seq_start, *last_idx, *tile_seq, *tile_q0, *n_tiles;
+  float* resid;
+  __half *xn, *qkv, *att, *act;
+};
+
+aiq_status prefill_bufs(aiq_ctx* c, const ModelD& m, int64_t B, PrefillBufs* pb) {
+  const aiq_model_config& g = m.cfg;
+  const int64_t nqkv = static_cast<int64_t>(g.n_heads + 2 * g.n_kv_heads) * g.head_dim;
+  AIQ_TRY(ws(c, "pf.tok", B, &pb->tok));
+  AIQ_TRY(ws(c, "pf.pos", B, &pb->pos));
+  AIQ_TRY(ws(c, "pf.seq_start", B + 1, &pb->seq_start));
+  AIQ_TRY(ws(c, "pf.last", B, &pb->last_idx));
+  AIQ_TRY(ws(c, "pf.tile_seq", B / 64 + B + 1, &pb->tile_seq));
+  AIQ_TRY(ws(c, "pf.tile_q0", B / 64 + B + 1, &pb->tile_q0));
+  AIQ_TRY(ws(c, "pf.n_tiles", 1, &pb->n_tiles));
+  AIQ_TRY(ws(c, "pf.resid", B * g.d_model, &pb->resid));
+  AIQ_TRY(ws(c, "pf.xn", B * g.d_model, &pb->xn));
+  AIQ_TRY(ws(c, "pf.qkv", B * nqkv, &pb->qkv));
+  AIQ_TRY(ws(c, "pf.att", B * g.n_heads * g.head_dim, &pb->att));
+  AIQ_TRY(ws(c, "pf.act", B * g.d_ffn, &pb->act));
+  return AIQ_OK;
+}
+
+// Decoder forward over one packed chunk of n_seqs rows / T tokens, then the
+// label head into logits[n_seqs, K].
+aiq_status run_chunk(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, int64_t n_seqs, const int32_t* labels,
+                     int K, float* logits) {
+  const aiq_model_config& g = m.cfg;
+  const int d = g.d_model, hd = g.head_dim, Hq = g.n_heads, Hkv = g.n_kv_heads, f = g.d_ffn;
+  const int nqkv = (Hq + 2 * Hkv) * hd;
+  const int M = static_cast<int>(T);
+  {
+    ProfScope p(c, "attn_tiles+embed", 0, 0);
+    launch_attn_tiles(b.seq_start, static_cast<int32_t>(n_seqs), b.tile_seq, b.tile_q0, b.n_tiles, nullptr, c->stream);
+    launch_embed(b.tok, T, m.embed, d, b.resid, c->stream);
+    counted(c, 2);
+  }
+  const int n_tiles_max = static_cast<int>((T + 63) / 64 + n_seqs);
+  for (int l = 0; l < g.n_layers; ++l) {
+    const LayerD& L = m.layers[l];
+    {
+      ProfScope p(c, "rmsnorm", 0, 12.0 * T * d / 2 * 1);
+      launch_rmsnorm(b.resid, T, d, L.attn_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+      counted(c, 1);
+    }
+    GemmEpilogue e1;
+    e1.kind = EPI_ROPE_F16;
+    e1.out = b.qkv;
+    e1.ldo = nqkv;
+    e1.positions = b.pos;
+    e1.rope_cos = static_cast<const float*>(m.rope_cos.p);
+    e1.rope_sin = static_cast<const float*>(m.rope_sin.p);
+    e1.rope_cols = (Hq + Hkv) * hd;
+    e1.head_dim = hd;
+    e1.err = c->d_err;
+    AIQ_TRY(gemm(c, "gemm_qkv_rope", b.xn, d, L.wqkv, d, M, nqkv, d, m.bn_qkv, e1));
+    {
+      ProfScope p(c, "attention", 0, 0);
+      launch_attention(b.qkv, T, b.seq_start, b.tile_seq, b.tile_q0, n_tiles_max, b.n_tiles, Hq, Hkv, hd, b.att,
+                       c->d_err, c->stream);
+      counted(c, 1);
+    }
+    GemmEpilogue e2;
+    e2.kind = EPI_RESID_F32;
+    e2.out = b.resid;
+    e2.ldo = d;
+    e2.err = c->d_err;
+    AIQ_TRY(gemm(c, "gemm_o_resid", b.att, Hq * hd, L.wo, Hq * hd, M, d, Hq * hd, m.bn_o, e2));
+    {
+      ProfScope p(c, "rmsnorm", 0, 0);
+      launch_rmsnorm(b.resid, T, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+      counted(c, 1);
+    }
+    GemmEpilogue e3;
+    e3.kind = EPI_SWIGLU_F16;
+    e3.out = b.act;
+    e3.ldo = f;
+    e3.err = c->d_err;
+    AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, d, L.wgu, d, M, 2 * f, d, m.bn_gu, e3));
+    AIQ_TRY(gemm(c, "gemm_down_resid", b.act, f, L.wd, f, M, d, f, m.bn_d, e2));
+  }
+  {
+    ProfScope p(c, "label_head", 0, 0);
+    launch_label_head(b.resid, b.last_idx, n_seqs, d, m.final_norm, g.rms_eps, m.lm_head, m.lm_bias, labels, K, logits,
+                      c->stream);
+    counted(c, 1);
+  }
+  return AIQ_OK;
+}
+
+struct QueryState {
+  int64_t S = 0;
+  int32_t* ids = nullptr;        // candidate (probe) rows
+  int32_t* build_rows = nullptr; // joins
+  float* logits = nullptr;       // [S, K]
+  int64_t T = 0, n_chunks = 0, pairs = 0;
+};
+
+aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_select* q, QueryState* st) {
+  const ColD& col = t.cols[q->text_column];
+  const int K = q->n_labels;
+  const int64_t S = st->S;
+  const int32_t P = q->prefix_len;
+  float* logits;
+  AIQ_TRY(ws(c, "q.logits", std::max<int64_t>(S * K, 1), &logits));
+  st->logits = logits;
+  if (S == 0) return AIQ_OK;
+  int32_t *lens, *prefix_d, *labels_d;
+  int64_t *cu, *scan_scratch;
+  unsigned long long* pairs_d;
+  AIQ_TRY(ws(c, "q.lens", S, &lens));
+  AIQ_TRY(ws(c, "q.cu", S + 1, &cu));
+  AIQ_TRY(ws(c, "q.scan", 2 * (S / kRowsPerBlock + 2), &scan_scratch));
+  AIQ_TRY(ws(c, "q.pairs", 1, &pairs_d));
+  AIQ_TRY(ws(c, "q.prefix", std::max<int32_t>(P, 1), &prefix_d));
+  AIQ_TRY(ws(c, "q.labels", K, &labels_d));
+  if (P > 0) CUDA_TRY(cudaMemcpyAsync(prefix_d, q->prefix, P * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
+  CUDA_TRY(cudaMemcpyAsync(labels_d, q->label_ids, K * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
+  CUDA_TRY(cudaMemsetAsync(pairs_d, 0, sizeof(unsigned long long), c->stream));
+  {
+    ProfScope p(c, "pack_plan", 0, 0);
+    launch_row_lengths(col.offsets, st->ids, S, P, lens, pairs_d, c->stream);
+    launch_scan_lengths(lens, S, cu, scan_scratch, c->stream);
+    counted(c, 4);
+  }
+  CUDA_TRY(cudaMemcpyAsync(c->h_pin + 1, pairs_d, sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream));
+  AIQ_TRY(read_i64(c, cu + S, 1, c->h_pin));
+  const int64_t T = c->h_pin[0];
+  st->T = T;
+  st->pairs = c->h_pin[1];
+  const int64_t max_len = P + col.max_len;
+  int64_t B = std::max<int64_t>(c->token_budget, max_len);
+  const int64_t step = B - max_len + 1;
+  const int64_t n_chunks = (T + step - 1) / step;
+  st->n_chunks = n_chunks;
+  int64_t* chunk_d;
+  AIQ_TRY(ws(c, "q.chunks", 2 * (n_chunks + 1), &chunk_d));
+  launch_chunk_bounds(cu, S, step, n_chunks, chunk_d, c->stream);
+  counted(c, 1);
+  std::vector<int64_t> chunks(2 * (n_chunks + 1));
+  CUDA_TRY(cudaMemcpyAsync(chunks.data(), chunk_d, chunks.size() * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream));
+  AIQ_TRY(sync_and_check(c));
+  int64_t Bmax = 0;
+  for (int64_t i = 0; i < n_chunks; ++i) Bmax = std::max(Bmax, chunks[2 * (i + 1) + 1] - chunks[2 * i + 1]);
+  AIQ_TRY(ensure_rope(c, m, static_cast<int>(max_len)));
+  PrefillBufs pb;
+  AIQ_TRY(prefill_bufs(c, m, std::max<int64_t>(Bmax, 64), &pb));
+  for (int64_t i = 0; i < n_chunks; ++i) {
+    const int64_t r0 = chunks[2 * i], r1 = chunks[2 * (i + 1)];
+    const int64_t Tc = chunks[2 * (i + 1) + 1] - chunks[2 * i + 1];
+    if (r1 <= r0) continue;
+    {
+      ProfScope p(c, "pack_chunk", 0, 0);
+      launch_pack_chunk(cu, st->ids, col.offsets, static_cast<const int32_t*>(col.data), prefix_d, P, r0, r1, pb.tok,
+                        pb.pos, pb.seq_start, pb.last_idx, c->stream);
+      counted(c, 1);
+    }
+    AIQ_TRY(run_chunk(c, m, pb, Tc, r1 - r0, labels_d, K, logits + r0 * K));
+  }
+  return AIQ_OK;
+}
+
+// ------------------------------------------------------- aggregate phase ---
+
+aiq_status aggregate_phase(aiq_ctx* c, const aiq_select* q, QueryState* st, const TableD* build, int32_t build_key,
+                           ResultH& R) {
+  const int K = q->n_labels;
+  const int64_t S = st->S;
+  const int64_t nb = (S + kRowsPerBlock - 1) / kRowsPerBlock;
+  int32_t *dec, *bcnt;
+  uint32_t* ybits;
+  int64_t* boff;
+  unsigned long long* lcnt;
+  AIQ_TRY(ws(c, "a.dec", std::max<int64_t>(S, 1), &dec));
+  AIQ_TRY(ws(c, "a.bits", std::max<int64_t>(nb, 1) * (kRowsPerBlock / 32), &ybits));
+  AIQ_TRY(ws(c, "a.bcnt", std::max<int64_t>(nb, 1), &bcnt));
+  AIQ_TRY(ws(c, "a.boff", nb + 1, &boff));
+  AIQ_TRY(ws(c, "a.lcnt", 16, &lcnt));
+  CUDA_TRY(cudaMemsetAsync(lcnt, 0, 16 * sizeof(unsigned long long), c->stream));
+  {
+    ProfScope p(c, "decide", 0, 0);
+    launch_decide(st->logits, S, K, dec, ybits, bcnt, lcnt, c->stream);
+    counted(c, S > 0);
+  }
+  R.label_counts.resize(K);
+  CUDA_TRY(cudaMemcpyAsync(R.label_counts.data(), lcnt, K * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream));
+  if (q->agg == AIQ_AGG_ROW_IDS && K == 2 && S > 0) {
+    launch_scan_counts(bcnt, nb, boff, c->stream);
+    AIQ_TRY(read_i64(c, boff + nb, 1, c->h_pin));
+    const int64_t Y = c->h_pin[0];
+    int32_t *pos, *rows;
+    AIQ_TRY(ws(c, "a.pos", std::max<int64_t>(Y, 1), &pos));
+    AIQ_TRY(ws(c, "a.rows", std::max<int64_t>(Y, 1), &rows));
+    launch_compact(ybits, boff, S, pos, st->ids, rows, c->stream);
+    counted(c, 2);
+    R.row_ids.resize(Y);
+    if (Y) CUDA_TRY(cudaMemcpyAsync(R.row_ids.data(), rows, Y * sizeof(int32_t), cudaMemcpyDeviceToHost, c->stream));
+  }
+  if (q->agg == AIQ_AGG_GROUP_BUILD_KEY) {
+    const int64_t nbr = build->n_rows;
+    const int64_t gb = (nbr + kRowsPerBlock - 1) / kRowsPerBlock;
+    unsigned long long* gcnt;
+    uint32_t* gbits;
+    int32_t* gbc;
+    int64_t* goff;
+    AIQ_TRY(ws(c, "g.cnt", std::max<int64_t>(nbr, 1), &gcnt));
+    AIQ_TRY(ws(c, "g.bits", std::max<int64_t>(gb, 1) * (kRowsPerBlock / 32), &gbits));
+    AIQ_TRY(ws(c, "g.bcnt", std::max<int64_t>(gb, 1), &gbc));
+    AIQ_TRY(ws(c, "g.boff", gb + 1, &goff));
+    CUDA_TRY(cudaMemsetAsync(gcnt, 0, std::max<int64_t>(nbr, 1) * sizeof(unsigned long long), c->stream));
+    {
+      ProfScope p(c, "group_by", 0, 0);
+      launch_group_build(dec, st->build_rows, S, gcnt, c->stream);
+      launch_nonzero_mask(gcnt, nbr, gbits, gbc, c->stream);
+      launch_scan_counts(gbc, gb, goff, c->stream);
+      counted(c, (S > 0) + (nbr > 0) + 1);
+    }
+    AIQ_TRY(read_i64(c, goff + gb, 1, c->h_pin));
+    const int64_t G = c->h_pin[0];
+    int32_t* grows;
+    int64_t *gkeys, *gcounts;
+    AIQ_TRY(ws(c, "g.rows", std::max<int64_t>(G, 1), &grows));
+    AIQ_TRY(ws(c, "g.keys", std::max<int64_t>(G, 1), &gkeys));
+    AIQ_TRY(ws(c, "g.counts", std::max<int64_t>(G, 1), &gcounts));
+    launch_compact(gbits, goff, nbr, grows, nullptr, nullptr, c->stream);
+    launch_gather_groups(grows, G, static_cast<const int64_t*>(build->cols[build_key].data), gcnt, gkeys, gcounts,
+                         c->stream);
+    counted(c, (nbr > 0) + (G > 0));
+    R.group_rows.resize(G);
+    R.group_keys.resize(G);
+    R.group_counts.resize(G);
+    if (G) {
+      CUDA_TRY(cudaMemcpyAsync(R.group_rows.data(), grows, G * 4, cudaMemcpyDeviceToHost, c->stream));
+      CUDA_TRY(cudaMemcpyAsync(R.group_keys.data(), gkeys, G * 8, cudaMemcpyDeviceToHost, c->stream));
+      CUDA_TRY(cudaMemcpyAsync(R.group_counts.data(), gcounts, G * 8, cudaMemcpyDeviceToHost, c->stream));
+    }
+  }
+  if (q->flags & AIQ_FLAG_LOGITS) {
+    R.logits.resize(S * K);
+    R.decisions.resize(S);
+    if (S) {
+      CUDA_TRY(cudaMemcpyAsync(R.logits.data(), st->logits, S * K * 4, cudaMemcpyDeviceToHost, c->stream));
+      CUDA_TRY(cudaMemcpyAsync(R.decisions.data(), dec, S * 4, cudaMemcpyDeviceToHost, c->stream));
+    }
+  }
+  return AIQ_OK;
+}
+
+void finish_view(ResultH& R, const QueryState& st, int64_t n_input, int K, int agg) {
+  aiq_result_view& v = R.v;
+  v.n_input_rows = n_input;
+  v.n_candidates = st.S;
+  v.n_tokens = st.T;
+  v.n_chunks = st.n_chunks;
+  v.count = (K == 2 && !R.label_counts.empty()) ? R.label_counts[0] : -1;
+  v.row_ids = R.row_ids.empty() ? nullptr : R.row_ids.data();
+  v.n_row_ids = static_cast<int64_t>(R.row_ids.size());
+  v.group_build_rows = R.group_rows.empty() ? nullptr : R.group_rows.data();
+  v.group_keys = R.group_keys.empty() ? nullptr : R.group_keys.data();
+  v.group_counts = R.group_counts.empty() ? nullptr : R.group_counts.data();
+  v.n_groups = static_cast<int64_t>(R.group_rows.size());
+  v.label_counts = R.label_counts.empty() ? nullptr : R.label_counts.data();
+  v.n_labels = static_cast<int32_t>(R.label_counts.size());
+  v.cand_row_ids = R.cand_ids.empty() ? nullptr : R.cand_ids.data();
+  v.cand_build_rows = R.cand_build.empty() ? nullptr : R.cand_build.data();
+  v.label_logits = R.logits.empty() ? nullptr : R.logits.data();
+  v.decisions = R.decisions.empty() ? nullptr : R.decisions.data();
+  (void)agg;
+}
+
+aiq_status validate_select(aiq_ctx* c, const TableD& t, const ModelD* m, const aiq_select* q) {
+  if (!q) return fail(AIQ_ERR_INVALID_ARG, "select is NULL");
+  const bool rel_only = q->flags & AIQ_FLAG_RELATIONAL_ONLY;
+  if (rel_only) return AIQ_OK;
+  if (!m) return fail(AIQ_ERR_NOT_FOUND, "unknown model handle");
+  if (q->text_column < 0 || q->text_column >= static_cast<int32_t>(t.cols.size()) ||
+      t.cols[q->text_column].type != AIQ_TOKENS)
+    return fail(AIQ_ERR_INVALID_ARG, "text_column must name a TOKENS column");
+  const int V = m->cfg.vocab;
+  if (t.cols[q->text_column].max_id >= V) return fail(AIQ_ERR_INVALID_ARG, "a row token id is >= vocab");
+  if (q->prefix_len < 0 || (q->prefix_len > 0 && !q->prefix)) return fail(AIQ_ERR_INVALID_ARG, "bad prefix");
+  for (int i = 0; i < q->prefix_len; ++i)
+    if (q->prefix[i] < 0 || q->prefix[i] >= V) return fail(AIQ_ERR_INVALID_ARG, "prefix token id out of range");
+  if (q->n_labels < 2 || q->n_labels > 16 || !q->label_ids) return fail(AIQ_ERR_INVALID_ARG, "n_labels must be 2..16");
+  for (int i = 0; i < q->n_labels; ++i)
+    if (q->label_ids[i] < 0 || q->label_ids[i] >= V) return fail(AIQ_ERR_INVALID_ARG, "label id out of range");
+  if (q->agg < AIQ_AGG_COUNT || q->agg > AIQ_AGG_GROUP_BUILD_KEY) return fail(AIQ_ERR_INVALID_ARG, "unknown agg");
+  if ((q->agg == AIQ_AGG_COUNT || q->agg == AIQ_AGG_ROW_IDS) && q->n_labels != 2)
+    return fail(AIQ_ERR_INVALID_ARG, "COUNT / ROW_IDS need exactly 2 labels (yes, no)");
+  if (q->agg == AIQ_AGG_GROUP_BUILD_KEY && q->n_labels != 2)
+    return fail(AIQ_ERR_INVALID_ARG, "GROUP_BUILD_KEY needs exactly 2 labels (yes, no)");
+  const int64_t max_len = q->prefix_len + t.cols[q->text_column].max_len;
+  if (max_len <= 0) return fail(AIQ_ERR_INVALID_ARG, "every prompt is empty");
+  if (max_len > (1 << 20)) return fail(AIQ_ERR_UNSUPPORTED, "a prompt is longer than 2^20 tokens");
+  (void)c;
+  return AIQ_OK;
+}
+
+aiq_status run_query(aiq_ctx* c, const TableD* build, int32_t build_key, const aiq_pred* build_preds, int32_t n_bp,
+                     const TableD& probe, int32_t probe_key, ModelD* m, const aiq_select* q, aiq_result_h* out) {
+  AIQ_TRY(validate_select(c, probe, m, q));
+  const bool rel_only = q->flags & AIQ_FLAG_RELATIONAL_ONLY;
+  PredSet ps{};
+  AIQ_TRY(make_pred_set(probe, q->preds, q->n_preds, &ps));
+  if (!rel_only && q->agg == AIQ_AGG_GROUP_BUILD_KEY && !build)
+    return fail(AIQ_ERR_INVALID_ARG, "GROUP_BUILD_KEY needs a join");
+
+  c->launches = 0;
+  cudaEvent_t ev[4];
+  for (auto& e : ev) e = take_event(c);
+  CUDA_TRY(cudaEventRecord(ev[0], c->stream));
+  QueryState st;
+  ProbeSpec pr;
+  if (build) {
+    PredSet bps{};
+    AIQ_TRY(make_pred_set(*build, build_preds, n_bp, &bps));
+    int64_t Sb = 0;
+    int32_t* bids;
+    AIQ_TRY(filter_compact(c, *build, bps, ProbeSpec{}, "jb", &Sb, &bids, nullptr));
+    int64_t cap = 64;
+    while (cap < 2 * Sb) cap <<= 1;
+    unsigned long long* tk;
+    int32_t* tv;
+    AIQ_TRY(ws(c, "j.keys", cap, &tk));
+    AIQ_TRY(ws(c, "j.vals", cap, &tv));
+    {
+      ProfScope p(c, "hash_build", 0, 0);
+      launch_fill_u64(tk, cap, 0x8000000000000000ull, c->stream);
+      launch_hash_build(static_cast<const int64_t*>(build->cols[build_key].data), bids, Sb, tk, tv, cap, c->d_err,
+                        c->stream);
+      counted(c, 1 + (Sb > 0));
+    }
+    pr.keys = static_cast<const int64_t*>(probe.cols[probe_key].data);
+    pr.table_keys = tk;
+    pr.table_vals = tv;
+    pr.capacity = cap;
+  }
+  AIQ_TRY(filter_compact(c, probe, ps, pr, "sel", &st.S, &st.ids, build ? &st.build_rows : nullptr));
+  CUDA_TRY(cudaEventRecord(ev[1], c->stream));
+
+  ResultH R;
+  if (rel_only || (q->flags & AIQ_FLAG_LOGITS)) {
+    R.cand_ids.resize(st.S);
+    if (st.S) CUDA_TRY(cudaMemcpyAsync(R.cand_ids.data(), st.ids, st.S * 4, cudaMemcpyDeviceToHost, c->stream));
+    if (build) {
+      R.cand_build.resize(st.S);
+      if (st.S)
+        CUDA_TRY(cudaMemcpyAsync(R.cand_build.data(), st.build_rows, st.S * 4, cudaMemcpyDeviceToHost, c->stream));
+    }
+  }
+  if (!rel_only) {
+    AIQ_TRY(prefill_phase(c, probe, *m, q, &st));
+    CUDA_TRY(cudaEventRecord(ev[2], c->stream));
+    AIQ_TRY(aggregate_phase(c, q, &st, build, build_key, R));
+  } else {
+    CUDA_TRY(cudaEventRecord(ev[2], c->stream));
+  }
+  CUDA_TRY(cudaEventRecord(ev[3], c->stream));
+  AIQ_TRY(sync_and_check(c));
+  float t01 = 0, t12 = 0, t23 = 0, t03 = 0;
+  cudaEventElapsedTime(&t01, ev[0], ev[1]);
+  cudaEventElapsedTime(&t12, ev[1], ev[2]);
+  cudaEventElapsedTime(&t23, ev[2], ev[3]);
+  cudaEventElapsedTime(&t03, ev[0], ev[3]);
+  for (auto& e : ev) c->ev_pool.push_back(e);
+  collect_profile(c);
+  const int K = rel_only ? 0 : q->n_labels;
+  finish_view(R, st, probe.n_rows, K, q->agg);
+  R.v.ms_relational = t01;
+  R.v.ms_prefill = t12;
+  R.v.ms_aggregate = t23;
+  R.v.ms_total = t03;
+  if (!rel_only && m) {
+    const aiq_model_config& g = m->cfg;
+    R.v.prefill_flops = m->linear_flops_per_token * static_cast<double>(st.T) +
+                        4.0 * g.n_heads * g.head_dim * g.n_layers * static_cast<double>(st.pairs) +
+                        2.0 * g.d_model * K * static_cast<double>(st.S);
+  }
+  ResultH& dst = new_result(c, out);
+  dst = std::move(R);
+  finish_view(dst, st, probe.n_rows, K, q->agg);
+  dst.v.ms_relational = t01;
+  dst.v.ms_prefill = t12;
+  dst.v.ms_aggregate = t23;
+  dst.v.ms_total = t03;
+  if (!rel_only && m) dst.v.prefill_flops = R.v.prefill_flops;
+  dst.v.n_launches = c->launches;
+  return AIQ_OK;
+}
+
+void free_model(aiq_ctx* c, ModelD& m) {
+  for (auto& b : m.allocs) dfree(c, b.p, b.bytes);
+  m.allocs.clear();
+  dfree(c, m.rope_cos.p, m.rope_cos.bytes);
+  dfree(c, m.rope_sin.p, m.rope_sin.bytes);
+}
+
+void free_table(aiq_ctx* c, TableD& t) {
+  for (auto& col : t.cols) {
+    dfree(c, col.data, col.bytes);
+    if (col.offsets) dfree(c, col.offsets, (t.n_rows + 1) * sizeof(int64_t));
+  }
+  t.cols.clear();
+}
+
+template <typename T>
+aiq_status model_alloc(aiq_ctx* c, ModelD& m, size_t count, T** out) {
+  void* p = nullptr;
+  AIQ_TRY(dalloc(c, &p, count * sizeof(T)));
+  m.allocs.push_back(DevBuf{p, std::max<size_t>(count * sizeof(T), 256)});
+  *out = static_cast<T*>(p);
+  return AIQ_OK;
+}
+
+int pick_bn(int n) { return n % 256 == 0 ? 256 : 128; }
+
+}  // namespace
+
+// =================================================================== C-ABI
+
+extern "C" {
+
+aiq_status aiq_init(int device, aiq_ctx** out) {
+  if (!out) return fail(AIQ_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  int n = 0;
+  CUDA_TRY(cudaGetDeviceCount(&n));
+  if (device < 0 || device >= n) return fail(AIQ_ERR_INVALID_ARG, "no such CUDA device");
+  CUDA_TRY(cudaSetDevice(device));
+  cudaDeviceProp prop;
+  CUDA_TRY(cudaGetDeviceProperties(&prop, device));
+  if (prop.major != 10 || prop.minor != 3)
+    return fail(AIQ_ERR_UNSUPPORTED, "this library is built for sm_103 (GB300) only");
+  aiq_ctx* c = new aiq_ctx();
+  c->device = device;
+  c->num_sms = prop.multiProcessorCount;
+  if (const char* cap = std::getenv("AIQ_DEVICE_BYTES_MAX")) c->bytes_max = std::strtoull(cap, nullptr, 10);
+  cudaError_t e = cudaStreamCreateWithFlags(&c->stream, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaMalloc(&c->d_err, sizeof(int));
+  if (e == cudaSuccess) e = cudaMemset(c->d_err, 0, sizeof(int));
+  if (e == cudaSuccess) e = cudaMallocHost(&c->h_pin, 64 * sizeof(int64_t));
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    delete c;
+    return fail(AIQ_ERR_CUDA, std::string("context setup: ") + cudaGetErrorString(e));
+  }
+  *out = c;
+  g_err.clear();
+  return AIQ_OK;
+}
+
+void aiq_shutdown(aiq_ctx* c) {
+  if (!c) return;
+  cudaSetDevice(c->device);
+  cudaStreamSynchronize(c->stream);
+  for (auto& kv : c->tables) free_table(c, kv.second);
+  for (auto& kv : c->models) free_model(c, kv.second);
+  for (auto& kv : c->ws) dfree(c, kv.second.p, kv.second.bytes);
+  for (auto& r : c->prof) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  for (auto e : c->ev_pool) cudaEventDestroy(e);
+  cudaFree(c->d_err);
+  cudaFreeHost(c->h_pin);
+  cudaStreamDestroy(c->stream);
+  delete c;
+}
+
+aiq_status aiq_load_table(aiq_ctx* c, const aiq_column* cols, int32_t n_cols, int64_t n_rows, aiq_table* out) {
+  if (!c || !out) return fail(AIQ_ERR_INVALID_ARG, "ctx/out is NULL");
+  if (n_cols <= 0 || !cols) return fail(AIQ_ERR_INVALID_ARG, "no columns");
+  if (n_rows < 0 || n_rows >= (int64_t(1) << 31)) return fail(AIQ_ERR_INVALID_ARG, "n_rows must be in [0, 2^31)");
+  CUDA_TRY(cudaSetDevice(c->device));
+  TableD t;
+  t.n_rows = n_rows;
+  for (int i = 0; i < n_cols; ++i) {
+    const aiq_column& a = cols[i];
+    ColD col;
+    col.name = a.name ? a.name : "";
+    col.type = a.type;
+    if (a.type < AIQ_INT32 || a.type > AIQ_TOKENS) {
+      free_table(c, t);
+      return fail(AIQ_ERR_INVALID_ARG, "unknown column type");
+    }
+    if (!a.data && n_rows > 0) {
+      free_table(c, t);
+      return fail(AIQ_ERR_INVALID_ARG, "column data is NULL");
+    }
+    size_t bytes = 0;
+    if (a.type == AIQ_TOKENS) {
+      if (!a.offsets) {
+        free_table(c, t);
+        return fail(AIQ_ERR_INVALID_ARG, "TOKENS column without offsets");
+      }
+      if (a.offsets[0] != 0) {
+        free_table(c, t);
+        return fail(AIQ_ERR_INVALID_ARG, "token offsets must start at 0");
+      }
+      for (int64_t r = 0; r < n_rows; ++r) {
+        const int64_t len = a.offsets[r + 1] - a.offsets[r];
+        if (len < 0) {
+          free_table(c, t);
+          return fail(AIQ_ERR_INVALID_ARG, "token offsets must be non-decreasing");
+        }
+        col.max_len = std::max(col.max_len, len);
+      }
+      const int64_t ntok = a.offsets[n_rows];
+      if (ntok >= (int64_t(1) << 31)) {
+        free_table(c, t);
+        return fail(AIQ_ERR_UNSUPPORTED, "more than 2^31 tokens in one column");
+      }
+      const int32_t* ids = static_cast<const int32_t*>(a.data);
+      for (int64_t k = 0; k < ntok; ++k) {
+        if (ids[k] < 0) {
+          free_table(c, t);
+          return fail(AIQ_ERR_INVALID_ARG, "negative token id");
+        }
+        col.max_id = std::max<int64_t>(col.max_id, ids[k]);
+      }
+      bytes = static_cast<size_t>(ntok) * sizeof(int32_t);
+      aiq_status st = dalloc(c, reinterpret_cast<void**>(&col.offsets), (n_rows + 1) * sizeof(int64_t));
+      if (st != AIQ_OK) {
+        free_table(c, t);
+        return st;
+      }
+      cudaMemcpy(col.offsets, a.offsets, (n_rows + 1) * sizeof(int64_t), cudaMemcpyHostToDevice);
+    } else {
+      bytes = static_cast<size_t>(n_rows) * (a.type == AIQ_INT64 ? 8 : 4);
+    }
+    col.bytes = bytes;
+    aiq_status st = dalloc(c, &col.data, bytes);
+    if (st != AIQ_OK) {
+      if (col.offsets) dfree(c, col.offsets, (n_rows + 1) * sizeof(int64_t));
+      free_table(c, t);
+      return st;
+    }
+    if (bytes) cudaMemcpy(col.data, a.data, bytes, cudaMemcpyHostToDevice);
+    t.cols.push_back(col);
+  }
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    free_table(c, t);
+    return fail(AIQ_ERR_CUDA, std::string("table upload: ") + cudaGetErrorString(e));
+  }
+  const int64_t h = c->next_handle++;
+  c->tables[h] = std::move(t);
+  *out = h;
+  return AIQ_OK;
+}
+
+aiq_status aiq_free_table(aiq_ctx* c, aiq_table h) {
+  if (!c) return fail(AIQ_ERR_INVALID_ARG, "ctx is NULL");
+  auto it = c->tables.find(h);
+  if (it == c->tables.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown table handle");
+  cudaStreamSynchronize(c->stream);
+  free_table(c, it->second);
+  c->tables.erase(it);
+  return AIQ_OK;
+}
+
+aiq_status aiq_load_model(aiq_ctx* c, const aiq_model_config* cfg, const void* const* tensors, int32_t n_tensors,
+                          aiq_model* out) {
+  if (!c || !cfg || !tensors || !out) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
+  const aiq_model_config g = *cfg;
+  if (g.n_layers < 1 || g.d_model <= 0 || g.n_heads <= 0 || g.n_kv_heads <= 0 || g.d_ffn <= 0 || g.vocab <= 0)
+    return fail(AIQ_ERR_INVALID_ARG, "model dimensions must be positive");
+  if (g.n_heads % g.n_kv_heads) return fail(AIQ_ERR_INVALID_ARG, "n_heads must be a multiple of n_kv_heads");
+  if (!(g.head_dim == 32 || g.head_dim == 64 || g.head_dim == 128))
+    return fail(AIQ_ERR_UNSUPPORTED, "head_dim must be 32, 64 or 128");
+  const int qd = g.n_heads * g.head_dim, kd = g.n_kv_heads * g.head_dim;
+  if (g.d_model % 128 || g.d_ffn % 128 || qd % 128 || (qd + 2 * kd) % 128)
+    return fail(AIQ_ERR_UNSUPPORTED, "d_model, d_ffn, Hq*hd and (Hq+2Hkv)*hd must be multiples of 128");
+  if (n_tensors != 1 + 9 * g.n_layers + 3) return fail(AIQ_ERR_INVALID_ARG, "n_tensors must be 1 + 9 L + 3");
+  for (int i = 0; i < n_tensors; ++i)
+    if (!tensors[i]) return fail(AIQ_ERR_INVALID_ARG, "a tensor pointer is NULL");
+  CUDA_TRY(cudaSetDevice(c->device));
+  const int64_t d = g.d_model, f = g.d_ffn, V = g.vocab;
+  ModelD m;
+  m.cfg = g;
+  m.bn_qkv = pick_bn(qd + 2 * kd);
+  m.bn_o = pick_bn(g.d_model);
+  m.bn_gu = pick_bn(2 * g.d_ffn);
+  m.bn_d = pick_bn(g.d_model);
+  if (m.bn_qkv % g.head_dim) m.bn_qkv = 128;
+  m.linear_flops_per_token = 2.0 * g.n_layers * (double(d) * (qd + 2 * kd) + double(qd) * d + 3.0 * d * f);
+  auto up_bf16 = [&](const void* src, size_t count, uint16_t** dst) -> aiq_status {
+    AIQ_TRY(model_alloc(c, m, count, dst));
+    CUDA_TRY(cudaMemcpyAsync(*dst, src, count * 2, cudaMemcpyHostToDevice, c->stream));
+    return AIQ_OK;
+  };
+  uint16_t* stage = nullptr;
+  const size_t stage_elems = std::max<size_t>(2 * f * d, (size_t)(qd + 2 * kd) * d);
+  void* sp = nullptr;
+  aiq_status st = dalloc(c, &sp, stage_elems * 2);
+  if (st != AIQ_OK) return st;
+  stage = static_cast<uint16_t*>(sp);
+  auto fail_model = [&](aiq_status s2) {
+    cudaStreamSynchronize(c->stream);
+    dfree(c, sp, stage_elems * 2);
+    free_model(c, m);
+    return s2;
+  };
+#define M_TRY(x)                           \
+  do {                                     \
+    aiq_status s_ = (x);                   \
+    if (s_ != AIQ_OK) return fail_model(s_); \
+  } while (0)
+  int ti = 0;
+  M_TRY(up_bf16(tensors[ti++], V * d, &m.embed));
+  m.layers.resize(g.n_layers);
+  for (int l = 0; l < g.n_layers; ++l) {
+    LayerD& L = m.layers[l];
+    M_TRY(up_bf16(tensors[ti++], d, &L.attn_norm));
+    // q, k, v stacked then converted: [(Hq + 2 Hkv) hd, d]
+    cudaStreamSynchronize(c->stream);
+    cudaMemcpy(stage, tensors[ti++], size_t(qd) * d * 2, cudaMemcpyHostToDevice);
+    cudaMemcpy(stage + size_t(qd) * d, tensors[ti++], size_t(kd) * d * 2, cudaMemcpyHostToDevice);
+    cudaMemcpy(stage + size_t(qd + kd) * d, tensors[ti++], size_t(kd) * d * 2, cudaMemcpyHostToDevice);
+    M_TRY(model_alloc(c, m, size_t(qd + 2 * kd) * d, &L.wqkv));
+    launch_bf16_to_f16(stage, L.wqkv, qd + 2 * kd, d, 0, 0, c->d_err, c->stream);
+    cudaStreamSynchronize(c->stream);
+    cudaMemcpy(stage, tensors[ti++], size_t(d) * qd * 2, cudaMemcpyHostToDevice);
+    M_TRY(model_alloc(c, m, size_t(d) * qd, &L.wo));
+    launch_bf16_to_f16(stage, L.wo, d, qd, 0, 0, c->d_err, c->stream);
+    M_TRY(up_bf16(tensors[ti++], d, &L.mlp_norm));
+    cudaStreamSynchronize(c->stream);
+    cudaMemcpy(stage, tensors[ti++], size_t(f) * d * 2, cudaMemcpyHostToDevice);
+    cudaMemcpy(stage + size_t(f) * d, tensors[ti++], size_t(f) * d * 2, cudaMemcpyHostToDevice);
+    M_TRY(model_alloc(c, m, size_t(2 * f) * d, &L.wgu));
+    launch_bf16_to_f16(stage, L.wgu, 2 * f, d, m.bn_gu / 2, f, c->d_err, c->stream);
+    cudaStreamSynchronize(c->stream);
+    cudaMemcpy(stage, tensors[ti++], size_t(d) * f * 2, cudaMemcpyHostToDevice);
+    M_TRY(model_alloc(c, m, size_t(d) * f, &L.wd));
+    launch_bf16_to_f16(stage, L.wd, d, f, 0, 0, c->d_err, c->stream);
+  }
+  M_TRY(up_bf16(tensors[ti++], d, &m.final_norm));
+  M_TRY(up_bf16(tensors[ti++], V * d, &m.lm_head));
+  M_TRY(up_bf16(tensors[ti++], V, &m.lm_bias));
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  if (e != cudaSuccess) return fail_model(fail(AIQ_ERR_CUDA, std::string("model upload: ") + cudaGetErrorString(e)));
+  int err = 0;
+  cudaMemcpy(&err, c->d_err, sizeof(int), cudaMemcpyDeviceToHost);
+  if (err) {
+    cudaMemset(c->d_err, 0, sizeof(int));
+    return fail_model(fail(AIQ_ERR_UNSUPPORTED, "a linear weight is outside the fp16 range"));
+  }
+#undef M_TRY
+  dfree(c, sp, stage_elems * 2);
+  const int64_t h = c->next_handle++;
+  c->models[h] = std::move(m);
+  *out = h;
+  return AIQ_OK;
+}
+
+aiq_status aiq_free_model(aiq_ctx* c, aiq_model h) {
+  if (!c) return fail(AIQ_ERR_INVALID_ARG, "ctx is NULL");
+  auto it = c->models.find(h);
+  if (it == c->models.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown model handle");
+  cudaStreamSynchronize(c->stream);
+  free_model(c, it->second);
+  c->models.erase(it);
+  return AIQ_OK;
+}
+
+aiq_status aiq_run_select(aiq_ctx* c, aiq_table table, aiq_model model, const aiq_select* q, aiq_result_h* out) {
+  if (!c || !q || !out) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
+  auto t = c->tables.find(table);
+  if (t == c->tables.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown table handle");
+  ModelD* m = nullptr;
+  auto mi = c->models.find(model);
+  if (mi != c->models.end()) m = &mi->second;
+  if (q->agg == AIQ_AGG_GROUP_BUILD_KEY && !(q->flags & AIQ_FLAG_RELATIONAL_ONLY))
+    return fail(AIQ_ERR_INVALID_ARG, "GROUP_BUILD_KEY needs aiq_run_join_select");
+  CUDA_TRY(cudaSetDevice(c->device));
+  return run_query(c, nullptr, -1, nullptr, 0, t->second, -1, m, q, out);
+}
+
+aiq_status aiq_run_join_select(aiq_ctx* c, aiq_table build, int32_t build_key, const aiq_pred* build_preds,
+                               int32_t n_build_preds, aiq_table probe, int32_t probe_key, aiq_model model,
+                               const aiq_select* q, aiq_result_h* out) {
+  if (!c || !q || !out) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
+  auto b = c->tables.find(build);
+  auto p = c->tables.find(probe);
+  if (b == c->tables.end() || p == c->tables.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown table handle");
+  if (build_key < 0 || build_key >= static_cast<int32_t>(b->second.cols.size()) ||
+      b->second.cols[build_key].type != AIQ_INT64)
+    return fail(AIQ_ERR_INVALID_ARG, "build key must be an INT64 column");
+  if (probe_key < 0 || probe_key >= static_cast<int32_t>(p->second.cols.size()) ||
+      p->second.cols[probe_key].type != AIQ_INT64)
+    return fail(AIQ_ERR_INVALID_ARG, "probe key must be an INT64 column");
+  ModelD* m = nullptr;
+  auto mi = c->models.find(model);
+  if (mi != c->models.end()) m = &mi->second;
+  CUDA_TRY(cudaSetDevice(c->device));
+  return run_query(c, &b->second, build_key, build_preds, n_build_preds, p->second, probe_key, m, q, out);
+}
+
+aiq_status aiq_result(aiq_ctx* c, aiq_result_h h, aiq_result_view* out) {
+  if (!c || !out) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
+  auto it = c->results.find(h);
+  if (it == c->results.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown result handle");
+  *out = it->second.v;
+  return AIQ_OK;
+}
+
+aiq_status aiq_result_free(aiq_ctx* c, aiq_result_h h) {
+  if (!c) return fail(AIQ_ERR_INVALID_ARG, "ctx is NULL");
+  auto it = c->results.find(h);
+  if (it == c->results.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown result handle");
+  c->results.erase(it);
+  return AIQ_OK;
+}
+
+const char* aiq_last_error(void) { return g_err.c_str(); }
+
+aiq_status aiq_set_option(aiq_ctx* c, const char* name, int64_t value) {
+  if (!c || !name) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
+  if (!std::strcmp(name, "token_budget")) {
+    if (value < 64 || value > (int64_t(1) << 30)) return fail(AIQ_ERR_INVALID_ARG, "token_budget must be 64..2^30");
+    c->token_budget = value;
+    return AIQ_OK;
+  }
+  if (!std::strcmp(name, "profile")) {
+    c->profile = value != 0;
+    return AIQ_OK;
+  }
+  return fail(AIQ_ERR_INVALID_ARG, std::string("unknown option ") + name);
+}
+
+void* aiq_stream(aiq_ctx* c) { return c ? static_cast<void*>(c->stream) : nullptr; }
+
+aiq_status aiq_kernel_stats(aiq_ctx* c, aiq_kernel_stat* out, int32_t max, int32_t* n_out) {
+  if (!c || !n_out || (max > 0 && !out)) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
+  collect_profile(c);
+  c->stat_names.clear();
+  for (auto& kv : c->stats) c->stat_names.push_back(kv.first);
+  int32_t n = 0;
+  for (size_t i = 0; i < c->stat_names.size() && n < max; ++i) {
+    const StatAcc& s = c->stats[c->stat_names[i]];
+    out[n++] = aiq_kernel_stat{c->stat_names[i].c_str(), s.launches, s.ms, s.flops, s.bytes};
+  }
+  *n_out = n;
+  return AIQ_OK;
+}
+
+aiq_status aiq_reset_kernel_stats(aiq_ctx* c) {
+  if (!c) return fail(AIQ_ERR_INVALID_ARG, "ctx is NULL");
+  collect_profile(c);
+  c->stats.clear();
+  return AIQ_OK;
+}
+
+// ------------------------------------------------------------ step ops ---
+
+aiq_status aiq_op_gemm(aiq_ctx* c, const void* A, int64_t lda, const void* B, int64_t ldb, int32_t M, int32_t N,
+                       int32_t K, int32_t bn, int32_t epilogue, void* out, int64_t ldo, const int32_t* positions,
+                       const float* rope_cos, const float* rope_sin, int32_t rope_cols, int32_t head_dim) {
+  if (!c || !A || !B || !out) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
+  if (epilogue < AIQ_EPI_F16 || epilogue > AIQ_EPI_SWIGLU_F16) return fail(AIQ_ERR_INVALID_ARG, "unknown epilogue");
+  if (M < 0 || N <= 0 || K <= 0 || K % 64 || !(bn == 128 || bn == 256) || N % bn)
+    return fail(AIQ_ERR_INVALID_ARG, "need M >= 0, K % 64 == 0, bn in {128, 256}, N % bn == 0");
+  if (lda < K || ldb < K) return fail(AIQ_ERR_INVALID_ARG, "lda/ldb smaller than K");
+  CUDA_TRY(cudaSetDevice(c->device));
+  GemmEpilogue ep;
+  ep.kind = epilogue;
+  ep.out = out;
+  ep.ldo = ldo;
+  ep.positions = positions;
+  ep.rope_cos = rope_cos;
+  ep.rope_sin = rope_sin;
+  ep.rope_cols = rope_cols;
+  ep.head_dim = head_dim;
+  ep.err = c->d_err;
+  AIQ_TRY(gemm(c, "op_gemm", static_cast<const __half*>(A), lda, static_cast<const __half*>(B), ldb, M, N, K, bn, ep));
+  aiq_status s = sync_and_check(c);
+  collect_profile(c);
+  return s;
+}
+
+aiq_status aiq_op_rope_table(aiq_ctx* c, float* cs, float* sn, int32_t max_pos, int32_t head_dim, float theta) {
+  if (!c || !cs || !sn || max_pos <= 0 || head_dim <= 0 || head_dim % 2) return fail(AIQ_ERR_INVALID_ARG, "bad args");
+  CUDA_TRY(cudaSetDevice(c->device));
+  launch_rope_table(cs, sn, max_pos, head_dim, theta, c->stream);
+  return sync_and_check(c);
+}
+
+aiq_status aiq_op_rmsnorm(aiq_ctx* c, const float* x, int64_t T, int32_t d, const uint16_t* g, float eps, void* out) {
+  if (!c || !x || !g || !out || T < 0 || d <= 0 || d % 4) return fail(AIQ_ERR_INVALID_ARG, "bad args");
+  CUDA_TRY(cudaSetDevice(c->device));
+  launch_rmsnorm(x, T, d, g, eps, static_cast<__half*>(out), c->d_err, c->stream);
+  return sync_and_check(c);
+}
+
+aiq_status aiq_op_attention(aiq_ctx* c, const void* qkv, int64_t T, const int32_t* seq_start, int32_t n_seqs,
+                            int32_t Hq, int32_t Hkv, int32_t hd, void* out) {
+  if (!c || !qkv || !seq_start || !out || T < 0 || n_seqs < 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv)
+    return fail(AIQ_ERR_INVALID_ARG, "bad args");
+  if (!(hd == 32 || hd == 64 || hd == 128)) return fail(AIQ_ERR_UNSUPPORTED, "hd must be 32, 64 or 128");
+  if (n_seqs == 0 || T == 0) return AIQ_OK;
+  CUDA_TRY(cudaSetDevice(c->device));
+  int32_t *tile_seq, *tile_q0, *n_tiles;
+  const int64_t cap = T / 64 + n_seqs + 1;
+  AIQ_TRY(ws(c, "op.tile_seq", cap, &tile_seq));
+  AIQ_TRY(ws(c, "op.tile_q0", cap, &tile_q0));
+  AIQ_TRY(ws(c, "op.n_tiles", 1, &n_tiles));
+  launch_attn_tiles(seq_start, n_seqs, tile_seq, tile_q0, n_tiles, nullptr, c->stream);
+  launch_attention(static_cast<const __half*>(qkv), T, seq_start, tile_seq, tile_q0, static_cast<int>(cap - 1),
+                   n_tiles, Hq, Hkv, hd, static_cast<__half*>(out), c->d_err, c->stream);
+  return sync_and_check(c);
+}
+
+}  // extern "C"

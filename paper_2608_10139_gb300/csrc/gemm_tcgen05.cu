@@ -1,0 +1,377 @@
+// Prefill GEMM on the 5th-generation tensor cores (tcgen05 + TMEM + TMA).
+//
+// C = A[M,K] * B[N,K]^T: A is the packed activation (tokens x features, fp16),
+// B a linear layer's weight in [out, in] layout (fp16 copy of the bf16 model),
+// accumulation in fp32 TMEM.  These are the decoder's dense contractions
+// (QKV, O, gate/up and down projections of each layer) run over every token
+// of the packed variable-length batch.
+//
+// Structure (one CTA per SM, persistent over 128 x BN output tiles, tile
+// index n-fastest so concurrently running CTAs share the weight panel in L2):
+//   warp 0  : TMA producer, STAGES-deep ring of (A 128x64, B BNx64) tiles,
+//             128-byte swizzle, one mbarrier per stage (full / empty).
+//   warp 1  : allocates 2*BN TMEM columns (two accumulators) and issues
+//             tcgen05.mma 128xBNx16 from one thread; tcgen05.commit frees a
+//             smem stage and, per tile, signals the epilogue.
+//   warps 2-5: epilogue; each thread owns one accumulator row (TMEM lane),
+//             reads 32-column slices with tcgen05.ld and applies the fused
+//             epilogue (RoPE, SwiGLU, fp32 residual add) while the MMA warp
+//             already fills the other accumulator.
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace aiq {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;      // 64 fp16 = 128 bytes = one swizzle row
+constexpr int UMMA_K = 16;  // K of one kind::f16 MMA
+constexpr int kThreads = 192;
+
+template <int BN>
+struct Cfg {
+  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * BN;  // double-buffered fp32 accumulator
+  static constexpr int BAR_BYTES = 256;
+  static constexpr int SMEM = 1024 /*align slack*/ + STAGES * STAGE_BYTES + BAR_BYTES;
+};
+
+struct KArgs {
+  int M, N, K;
+  GemmEpilogue ep;
+};
+
+__device__ __forceinline__ float u2f(uint32_t u) { return __uint_as_float(u); }
+
+__device__ __forceinline__ void store_f16x32(__half* dst, const float* v, bool& bad) {
+  uint4 pk[4];
+  uint32_t* w = reinterpret_cast<uint32_t*>(pk);
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const float a = v[2 * j], b = v[2 * j + 1];
+    bad |= !(fabsf(a) <= 65504.f) || !(fabsf(b) <= 65504.f);
+    __half2 h = __floats2half2_rn(a, b);
+    w[j] = *reinterpret_cast<uint32_t*>(&h);
+  }
+  uint4* d = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) d[j] = pk[j];
+}
+
+__device__ __forceinline__ void load32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  tmem_ld_32x32b_x32(taddr, r);
+  tmem_ld_wait();
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = u2f(r[j]);
+}
+
+template <int BN, int EPI>
+__device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int row, int n0) {
+  const GemmEpilogue& ep = a.ep;
+  const bool live = row < a.M;
+  bool bad = false;
+  if constexpr (EPI == EPI_RESID_F32) {
+    float* o = static_cast<float*>(ep.out) + static_cast<int64_t>(row) * ep.ldo + n0;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      float v[32];
+      load32(trow + c, v);
+      if (live) {
+        float4* p = reinterpret_cast<float4*>(o + c);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float4 x = p[j];
+          x.x += v[4 * j];
+          x.y += v[4 * j + 1];
+          x.z += v[4 * j + 2];
+          x.w += v[4 * j + 3];
+          p[j] = x;
+        }
+      }
+    }
+  } else if constexpr (EPI == EPI_SWIGLU_F16) {
+    __half* o = static_cast<__half*>(ep.out) + static_cast<int64_t>(row) * ep.ldo + n0 / 2;
+#pragma unroll 1
+    for (int c = 0; c < BN / 2; c += 32) {
+      float g[32], u[32];
+      load32(trow + c, g);
+      load32(trow + BN / 2 + c, u);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) g[j] = g[j] / (1.0f + expf(-g[j])) * u[j];
+      if (live) store_f16x32(o + c, g, bad);
+    }
+  } else {
+    __half* o = static_cast<__half*>(ep.out) + static_cast<int64_t>(row) * ep.ldo + n0;
+    const int hd = ep.head_dim;
+    const int half = hd >> 1;
+    const int pos = (EPI == EPI_ROPE_F16 && live) ? ep.positions[row] : 0;
+#pragma unroll 1
+    for (int c = 0; c < BN;) {
+      if (EPI == EPI_ROPE_F16 && n0 + c < ep.rope_cols) {
+        // one head [c, c + hd): rotate pairs (i, i + hd/2) by pos * inv_freq_i
+        const float* cs = ep.rope_cos + static_cast<int64_t>(pos) * half;
+        const float* sn = ep.rope_sin + static_cast<int64_t>(pos) * half;
+        if (half >= 32) {
+#pragma unroll 1
+          for (int i0 = 0; i0 < half; i0 += 32) {
+            float x1[32], x2[32];
+            load32(trow + c + i0, x1);
+            load32(trow + c + half + i0, x2);
+            if (live) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j) {
+                const float cj = cs[i0 + j], sj = sn[i0 + j];
+                const float a1 = x1[j], a2 = x2[j];
+                x1[j] = a1 * cj - a2 * sj;
+                x2[j] = a2 * cj + a1 * sj;
+              }
+              store_f16x32(o + c + i0, x1, bad);
+              store_f16x32(o + c + half + i0, x2, bad);
+            }
+          }
+        } else {  // head_dim 32: both halves in one slice
+          float x[32];
+          load32(trow + c, x);
+          if (live) {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const float cj = cs[j], sj = sn[j];
+              const float a1 = x[j], a2 = x[j + 16];
+              x[j] = a1 * cj - a2 * sj;
+              x[j + 16] = a2 * cj + a1 * sj;
+            }
+            store_f16x32(o + c, x, bad);
+          }
+        }
+        c += hd;
+      } else {
+        float v[32];
+        load32(trow + c, v);
+        if (live) store_f16x32(o + c, v, bad);
+        c += 32;
+      }
+    }
+  }
+  if (bad) set_dev_error(ep.err, DEVERR_FP16_RANGE);
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_gemm_tcgen05(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b, KArgs args) {
+  using C = Cfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + C::STAGES;
+  uint64_t* tfull = bars + 2 * C::STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* mma_done = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  int* err = args.ep.err;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], 4);  // one arrival per epilogue warp
+    }
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tma_a);
+    tma_prefetch_desc(&tma_b);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+    tc_fence_before();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int num_n = args.N / BN;
+  const int num_m = (args.M + BM - 1) / BM;
+  const int num_tiles = num_m * num_n;
+  const int kblocks = args.K / BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------- TMA producer
+      uint32_t issued = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+        const int m0 = (tile / num_n) * BM;
+        const int n0 = (tile % num_n) * BN;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          const int s = issued % C::STAGES;
+          const uint32_t ph = (issued / C::STAGES) & 1;
+          if (!mbar_wait_bounded(&empty[s], ph ^ 1, abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
+          tma_load_2d(sA + s * C::A_BYTES, &tma_a, &full[s], kb * BK, m0);
+          tma_load_2d(sB + s * C::B_BYTES, &tma_b, &full[s], kb * BK, n0);
+          ++issued;
+        }
+      }
+      if (!ok) {
+        // drain this thread's copies still in flight before the CTA can exit
+        const uint32_t first = issued > (uint32_t)C::STAGES ? issued - C::STAGES : 0;
+        volatile int never = 0;
+        for (uint32_t i = first; i < issued; ++i)
+          mbar_wait_bounded(&full[i % C::STAGES], (i / C::STAGES) & 1, &never, nullptr, 200000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------ MMA issuer
+      constexpr uint32_t idesc = idesc_f16_f32(BM, BN);
+      uint32_t consumed = 0;
+      int acc = 0;
+      uint32_t acc_ph = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+        if (!mbar_wait_bounded(&tempty[acc], acc_ph ^ 1, abort_flag, err)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          const int s = consumed % C::STAGES;
+          const uint32_t ph = (consumed / C::STAGES) & 1;
+          if (!mbar_wait_bounded(&full[s], ph, abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
+          const uint32_t b0 = smem_u32(sB + s * C::B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / UMMA_K; ++k) {
+            // advancing K inside the 128-byte swizzle row = +32 bytes on the start address
+            umma_f16_ss(d_tmem, smem_desc_k_sw128(a0 + k * UMMA_K * 2), smem_desc_k_sw128(b0 + k * UMMA_K * 2),
+                        idesc, (kb | k) != 0);
+          }
+          umma_commit(&empty[s]);
+          ++consumed;
+        }
+        if (!ok) break;
+        umma_commit(&tfull[acc]);
+        acc ^= 1;
+        if (acc == 0) acc_ph ^= 1;
+      }
+      // every MMA issued above has completed once this arrives
+      umma_commit(mma_done);
+      volatile int never = 0;
+      mbar_wait_bounded(mma_done, 0, &never, err);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int quarter = warp & 3;  // TMEM lanes this warp may access
+    int acc = 0;
+    uint32_t acc_ph = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+      const int m0 = (tile / num_n) * BM;
+      const int n0 = (tile % num_n) * BN;
+      if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
+      tc_fence_after();
+      const uint32_t trow = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
+      epilogue_tile<BN, EPI>(args, trow, m0 + quarter * 32 + lane, n0);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      acc ^= 1;
+      if (acc == 0) acc_ph ^= 1;
+    }
+  }
+
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D fp16 tensor [rows, cols] (cols contiguous, row pitch ld elements), box 64 x box_rows, 128B swizzle.
+bool make_map(CUtensorMap* m, const __half* base, int64_t rows, int64_t cols, int64_t ld, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld * 2)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+template <int BN, int EPI>
+int launch(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, int num_sms, cudaStream_t stream) {
+  using C = Cfg<BN>;
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tcgen05<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  const int tiles = ((a.M + BM - 1) / BM) * (a.N / BN);
+  const int grid = tiles < num_sms ? tiles : num_sms;
+  k_gemm_tcgen05<BN, EPI><<<grid, kThreads, C::SMEM, stream>>>(ma, mb, a);
+  return cudaGetLastError();
+}
+
+template <int BN>
+int dispatch_epi(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, int num_sms, cudaStream_t s) {
+  switch (a.ep.kind) {
+    case EPI_F16: return launch<BN, EPI_F16>(ma, mb, a, num_sms, s);
+    case EPI_ROPE_F16: return launch<BN, EPI_ROPE_F16>(ma, mb, a, num_sms, s);
+    case EPI_RESID_F32: return launch<BN, EPI_RESID_F32>(ma, mb, a, num_sms, s);
+    case EPI_SWIGLU_F16: return launch<BN, EPI_SWIGLU_F16>(ma, mb, a, num_sms, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+int gemm_f16_tcgen05(const __half* A, int64_t lda, const __half* B, int64_t ldb, int M, int N, int K, int bn,
+                     const GemmEpilogue& ep, int num_sms, cudaStream_t stream) {
+  if (M == 0) return 0;
+  if (M < 0 || N <= 0 || K <= 0 || K % BK != 0 || (bn != 128 && bn != 256) || N % bn != 0) return cudaErrorInvalidValue;
+  if ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B)) & 15) return cudaErrorMisalignedAddress;
+  if ((lda * 2) % 16 != 0 || (ldb * 2) % 16 != 0) return cudaErrorInvalidValue;
+  if (ep.kind == EPI_ROPE_F16) {
+    const int hd = ep.head_dim;
+    if (!(hd == 32 || hd == 64 || hd == 128) || bn % hd != 0 || !ep.positions || !ep.rope_cos) return cudaErrorInvalidValue;
+  }
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, B, N, K, ldb, bn)) return cudaErrorInvalidValue;
+  KArgs a{M, N, K, ep};
+  return bn == 256 ? dispatch_epi<256>(ma, mb, a, num_sms, stream) : dispatch_epi<128>(ma, mb, a, num_sms, stream);
+}
+
+}  // namespace aiq

@@ -1,0 +1,123 @@
+// Internal host-side launchers of the library's CUDA kernels.  The C-ABI
+// layer (aiq_api.cu) is the only caller; none of this is exported.
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace aiq {
+
+// ------------------------------------------------------------------ GEMM ---
+enum GemmEpi : int {
+  EPI_F16 = 0,        // out fp16 [M, N] = acc
+  EPI_ROPE_F16 = 1,   // as EPI_F16, rotary embedding applied to columns < rope_cols
+  EPI_RESID_F32 = 2,  // out fp32 [M, N] += acc  (residual stream update)
+  EPI_SWIGLU_F16 = 3, // B interleaves gate/up blocks of BN/2 rows: out fp16 [M, N/2] = silu(g) * u
+};
+
+struct GemmEpilogue {
+  int kind = EPI_F16;
+  void* out = nullptr;
+  int64_t ldo = 0;                     // elements
+  const int32_t* positions = nullptr;  // ROPE: per-row position
+  const float* rope_cos = nullptr;     // ROPE: [max_pos, head_dim/2]
+  const float* rope_sin = nullptr;
+  int rope_cols = 0;
+  int head_dim = 0;
+  int* err = nullptr;
+};
+
+// C = A[M,K] * B[N,K]^T with fp16 operands and fp32 accumulation on tcgen05.
+// Requires K % 64 == 0, N % bn == 0, bn in {128, 256}, 16-byte aligned rows.
+// Returns 0 or a cudaError_t value.
+int gemm_f16_tcgen05(const __half* A, int64_t lda, const __half* B, int64_t ldb, int M, int N, int K, int bn,
+                     const GemmEpilogue& ep, int num_sms, cudaStream_t stream);
+
+// ------------------------------------------------------------ relational ---
+struct PredDev {
+  const void* col;
+  int32_t type;   // 0 int32, 1 int64, 2 float32
+  int32_t op;     // aiq_cmp
+  int64_t ivalue;
+  double fvalue;
+};
+constexpr int kMaxPreds = 8;
+struct PredSet {
+  PredDev p[kMaxPreds];
+  int n;
+};
+
+constexpr int kRowsPerBlock = 2048;  // rows per predicate / compaction block (64 bitmask words)
+
+// Hash-join probe evaluated together with the probe-side predicate.
+struct ProbeSpec {
+  const int64_t* keys = nullptr;  // probe key column (nullptr: no join)
+  const unsigned long long* table_keys = nullptr;
+  const int32_t* table_vals = nullptr;
+  int64_t capacity = 0;           // power of two
+  int32_t* match_out = nullptr;   // build row per probe row (valid where the bit is set)
+};
+
+// mask bits + per-block survivor counts.
+void launch_predicate_mask(const PredSet& ps, const ProbeSpec& probe, int64_t n_rows, uint32_t* bits,
+                           int32_t* block_counts, int* err, cudaStream_t s);
+// Exclusive scan of n int32 counts into int64 offsets[n+1] (one block).
+void launch_scan_counts(const int32_t* counts, int64_t n, int64_t* offsets, cudaStream_t s);
+// Order-preserving compaction of set bits: ids_out[k] = row of the k-th set bit;
+// optionally gathers `payload[row]` into payload_out[k].
+void launch_compact(const uint32_t* bits, const int64_t* block_offsets, int64_t n_rows, int32_t* ids_out,
+                    const int32_t* payload, int32_t* payload_out, cudaStream_t s);
+
+void launch_hash_build(const int64_t* keys, const int32_t* rows, int64_t n, unsigned long long* table_keys,
+                       int32_t* table_vals, int64_t capacity, int* err, cudaStream_t s);
+void launch_fill_u64(unsigned long long* p, int64_t n, unsigned long long v, cudaStream_t s);
+
+// ------------------------------------------------------------------ pack ---
+// lens[i] = prefix_len + text length of row ids[i]; *pairs += causal (q, k) pairs.
+void launch_row_lengths(const int64_t* offsets, const int32_t* ids, int64_t S, int32_t prefix_len, int32_t* lens,
+                        unsigned long long* pairs, cudaStream_t s);
+// Exclusive scan of int32 lengths into int64 cu[S+1] (multi-block).
+void launch_scan_lengths(const int32_t* lens, int64_t S, int64_t* cu, int64_t* scratch_blocks, cudaStream_t s);
+// chunk_rows[c] = first row whose start offset >= c * budget_step, c = 0..n_chunks.
+void launch_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64_t n_chunks, int64_t* chunk_rows,
+                         cudaStream_t s);
+// Pack rows [r0, r1) of a chunk: tokens, positions, chunk-local cu_seqlens and last-token index,
+// and the attention q-tile list.
+void launch_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,
+                       const int32_t* prefix, int32_t prefix_len, int64_t r0, int64_t r1, int32_t* tok,
+                       int32_t* pos, int32_t* seq_start, int32_t* last_idx, cudaStream_t s);
+// Attention work list of a chunk: one entry per (sequence, 64-row q block).
+void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t* tile_seq, int32_t* tile_q0,
+                       int32_t* n_tiles_dev, int32_t* scratch, cudaStream_t s);
+
+// --------------------------------------------------------------- prefill ---
+void launch_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int interleave_block,
+                        int64_t half_rows, int* err, cudaStream_t s);
+void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, float theta, cudaStream_t s);
+void launch_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, cudaStream_t s);
+void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int* err,
+                    cudaStream_t s);
+void launch_attention(const __half* qkv, int64_t T, const int32_t* seq_start, const int32_t* tile_seq,
+                      const int32_t* tile_q0, int n_tiles_max, const int32_t* n_tiles_dev, int Hq, int Hkv,
+                      int hd, __half* out, int* err, cudaStream_t s);
+void launch_label_head(const float* resid, const int32_t* last_idx, int64_t n_rows, int d, const uint16_t* g,
+                       float eps, const uint16_t* lm_head, const uint16_t* lm_bias, const int32_t* labels,
+                       int n_labels, float* logits_out, cudaStream_t s);
+
+// ------------------------------------------------------------- aggregate ---
+// decision per row from logits [S, K] (K == 2: strict yes > no; K > 2: first argmax),
+// yes-bitmask (K == 2), per-block yes counts, label counts [K] (int64, atomics).
+void launch_decide(const float* logits, int64_t S, int K, int32_t* decision, uint32_t* yes_bits,
+                   int32_t* block_counts, unsigned long long* label_counts, cudaStream_t s);
+// group counts[build_row] += 1 for yes rows.
+void launch_group_build(const int32_t* decision, const int32_t* cand_build_rows, int64_t S,
+                        unsigned long long* group_counts, cudaStream_t s);
+// bits of non-zero group counts + per-block counts.
+void launch_nonzero_mask(const unsigned long long* counts, int64_t n, uint32_t* bits, int32_t* block_counts,
+                         cudaStream_t s);
+void launch_gather_groups(const int32_t* rows, int64_t g, const int64_t* build_keys,
+                          const unsigned long long* counts, int64_t* keys_out, int64_t* counts_out,
+                          cudaStream_t s);
+
+}  // namespace aiq

@@ -1,0 +1,130 @@
+// Token packing of the candidate rows into a variable-length batch.
+//
+// Every candidate row's prompt is the shared prefix followed by the row's
+// tokens (Table 1, AI_IF row: the text column feeds the causal LM; the prompt
+// prefix is the instruction shared by all rows).  Rows are concatenated with
+// no padding; cu (int64 [S+1]) holds each row's start.  The prefill runs
+// over token-budget chunks of consecutive rows, the GPU counterpart of the
+// paper's scan over micro-batches (Section 3.2): row i belongs to chunk
+// floor(cu[i] / step), so a chunk never holds more than step + max_len tokens.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace aiq {
+namespace {
+
+// lens[i] = P + text length of row ids[i]; pairs += sum of len * (len + 1) / 2
+// (causal query-key pairs, for the executed-FLOP count).
+__global__ void k_row_lengths(const int64_t* offsets, const int32_t* ids, int64_t S, int32_t P, int32_t* lens,
+                              unsigned long long* pairs) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  unsigned long long pr = 0;
+  if (i < S) {
+    const int32_t r = ids[i];
+    const int64_t len = P + (offsets[r + 1] - offsets[r]);
+    lens[i] = static_cast<int32_t>(len);
+    pr = static_cast<unsigned long long>(len * (len + 1) / 2);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) pr += __shfl_xor_sync(0xffffffffu, pr, o);
+  if ((threadIdx.x & 31) == 0 && pr) atomicAdd(pairs, pr);
+}
+
+// chunk_rows[2c] = first row i with cu[i] >= c * step (S if none), chunk_rows[2c+1] = cu[that row].
+__global__ void k_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64_t n_chunks, int64_t* out) {
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (c > n_chunks) return;
+  int64_t lo = 0, hi = S;  // lower bound in cu[0..S)
+  if (c == n_chunks) {
+    lo = S;
+  } else {
+    const int64_t target = c * step;
+    while (lo < hi) {
+      const int64_t mid = (lo + hi) >> 1;
+      if (cu[mid] < target) lo = mid + 1;
+      else hi = mid;
+    }
+  }
+  out[2 * c] = lo;
+  out[2 * c + 1] = cu[lo];
+}
+
+// One warp per row: prefix then the row's text tokens, positions restart at 0.
+__global__ void k_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,
+                             const int32_t* prefix, int32_t P, int64_t r0, int64_t r1, int32_t* tok, int32_t* pos,
+                             int32_t* seq_start, int32_t* last_idx) {
+  const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  const int64_t i = r0 + w;
+  if (i >= r1) return;
+  const int64_t base = cu[r0];
+  const int64_t dst = cu[i] - base;
+  const int64_t len = cu[i + 1] - cu[i];
+  const int32_t r = ids[i];
+  const int32_t* src = text + offsets[r];
+  for (int64_t j = lane; j < len; j += 32) {
+    tok[dst + j] = j < P ? prefix[j] : src[j - P];
+    pos[dst + j] = static_cast<int32_t>(j);
+  }
+  if (lane == 0) {
+    seq_start[w] = static_cast<int32_t>(dst);
+    last_idx[w] = static_cast<int32_t>(dst + len - 1);
+    if (i == r1 - 1) seq_start[w + 1] = static_cast<int32_t>(cu[r1] - base);
+  }
+}
+
+// Attention work list: one entry per (sequence, 64-row query block), one block.
+__global__ void __launch_bounds__(1024) k_attn_tiles(const int32_t* seq_start, int32_t n, int32_t* tile_seq,
+                                                     int32_t* tile_q0, int32_t* n_tiles) {
+  __shared__ int32_t sh[1024];
+  int32_t carry = 0;
+  for (int32_t b = 0; b < n; b += 1024) {
+    const int32_t i = b + threadIdx.x;
+    const int32_t cnt = i < n ? (seq_start[i + 1] - seq_start[i] + 63) / 64 : 0;
+    sh[threadIdx.x] = cnt;
+    __syncthreads();
+    for (int o = 1; o < 1024; o <<= 1) {
+      int32_t y = threadIdx.x >= o ? sh[threadIdx.x - o] : 0;
+      __syncthreads();
+      sh[threadIdx.x] += y;
+      __syncthreads();
+    }
+    int32_t at = carry + sh[threadIdx.x] - cnt;
+    for (int32_t q = 0; q < cnt; ++q) {
+      tile_seq[at + q] = i;
+      tile_q0[at + q] = q * 64;
+    }
+    carry += sh[1023];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *n_tiles = carry;
+}
+
+}  // namespace
+
+void launch_row_lengths(const int64_t* offsets, const int32_t* ids, int64_t S, int32_t prefix_len, int32_t* lens,
+                        unsigned long long* pairs, cudaStream_t s) {
+  if (S <= 0) return;
+  k_row_lengths<<<static_cast<unsigned>((S + 255) / 256), 256, 0, s>>>(offsets, ids, S, prefix_len, lens, pairs);
+}
+
+void launch_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64_t n_chunks, int64_t* chunk_rows,
+                         cudaStream_t s) {
+  k_chunk_bounds<<<static_cast<unsigned>((n_chunks + 1 + 127) / 128), 128, 0, s>>>(cu, S, step, n_chunks, chunk_rows);
+}
+
+void launch_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,
+                       const int32_t* prefix, int32_t prefix_len, int64_t r0, int64_t r1, int32_t* tok,
+                       int32_t* pos, int32_t* seq_start, int32_t* last_idx, cudaStream_t s) {
+  if (r1 <= r0) return;
+  const int64_t threads = (r1 - r0) * 32;
+  k_pack_chunk<<<static_cast<unsigned>((threads + 255) / 256), 256, 0, s>>>(cu, ids, offsets, text, prefix, prefix_len,
+                                                                            r0, r1, tok, pos, seq_start, last_idx);
+}
+
+void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t* tile_seq, int32_t* tile_q0,
+                       int32_t* n_tiles_dev, int32_t* /*scratch*/, cudaStream_t s) {
+  k_attn_tiles<<<1, 1024, 0, s>>>(seq_start, n_seqs, tile_seq, tile_q0, n_tiles_dev);
+}
+
+}  // namespace aiq

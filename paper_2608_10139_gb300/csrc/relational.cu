@@ -1,0 +1,430 @@
+// Relational operators of the unified AI query on the GPU.
+//
+//  * predicate mask (Table 1, WHERE row): a conjunction of `column op const`
+//    terms evaluated over 2048-row tiles, 8 consecutive rows per thread with
+//    16-byte vector loads; the result is a bitmask (1 bit per row) plus each
+//    tile's survivor count.  A join probe (Section 4: reviews joined with
+//    movies on movie id) runs in the same pass for rows that pass the terms.
+//  * order-preserving stream compaction: tile counts -> exclusive scan ->
+//    each tile re-reads only its 256-byte bitmask slice and writes the ids of
+//    its set bits at its offset (reduce-then-scan; no inter-block waits).
+//  * open-addressing hash table (int64 key -> build row), linear probing with
+//    a bounded probe sequence.
+//  * decision (Fig. 2: strict yes > no, or first argmax) and the masked
+//    aggregates (Table 1, SELECT row): label counts, yes bitmask for the
+//    yes-row ids, GROUP BY build row with warp-aggregated atomics.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace aiq {
+namespace {
+
+constexpr int kThreads = 256;  // 256 threads x 8 rows = kRowsPerBlock
+constexpr unsigned long long kEmptyKey = 0x8000000000000000ull;
+
+template <typename T>
+__device__ __forceinline__ bool cmp(T v, int op, T c) {
+  switch (op) {
+    case 0: return v < c;
+    case 1: return v <= c;
+    case 2: return v > c;
+    case 3: return v >= c;
+    case 4: return v == c;
+    default: return v != c;
+  }
+}
+
+// Evaluates one term on rows [r0, r0 + 8) of this thread; returns 8 bits.
+__device__ __forceinline__ uint32_t eval_term(const PredDev& p, int64_t r0, int64_t n) {
+  uint32_t bits = 0;
+  const bool full = r0 + 8 <= n;
+  if (p.type == 1) {
+    const int64_t* c = static_cast<const int64_t*>(p.col) + r0;
+    int64_t v[8];
+    if (full) {
+      const int4* q = reinterpret_cast<const int4*>(c);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        int4 x = __ldg(q + j);
+        v[2 * j] = (static_cast<int64_t>(static_cast<uint32_t>(x.y)) << 32) | static_cast<uint32_t>(x.x);
+        v[2 * j + 1] = (static_cast<int64_t>(static_cast<uint32_t>(x.w)) << 32) | static_cast<uint32_t>(x.z);
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[j] = r0 + j < n ? c[j] : 0;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<int64_t>(v[j], p.op, p.ivalue)) << j;
+  } else {
+    const int32_t* c = static_cast<const int32_t*>(p.col) + r0;
+    int32_t v[8];
+    if (full) {
+      const int4* q = reinterpret_cast<const int4*>(c);
+      int4 a = __ldg(q), b = __ldg(q + 1);
+      v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+      v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[j] = r0 + j < n ? c[j] : 0;
+    }
+    if (p.type == 0) {
+      // compare in int64 so that constants outside the int32 range behave as in SQL
+#pragma unroll
+      for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<int64_t>(v[j], p.op, p.ivalue)) << j;
+    } else {
+      const float fc = static_cast<float>(p.fvalue);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<float>(__int_as_float(v[j]), p.op, fc)) << j;
+    }
+  }
+  return bits;
+}
+
+__device__ __forceinline__ int probe_lookup(const ProbeSpec& pr, unsigned long long key) {
+  if (key == kEmptyKey) return -1;
+  const unsigned long long mask = static_cast<unsigned long long>(pr.capacity - 1);
+  unsigned long long slot = hash64(key) & mask;
+  for (int64_t i = 0; i < pr.capacity; ++i) {
+    const unsigned long long k = pr.table_keys[slot];
+    if (k == key) return pr.table_vals[slot];
+    if (k == kEmptyKey) return -1;
+    slot = (slot + 1) & mask;
+  }
+  return -1;
+}
+
+// Each thread holds one byte of row bits (rows 8*t .. 8*t+7 of the tile);
+// assemble 32-bit words (4 lanes each), write them, and return the tile's
+// popcount (valid in thread 0).
+__device__ __forceinline__ int write_words_and_count(uint32_t byte, uint32_t* bits_tile, int* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t w = byte << (8 * (lane & 3));
+  w |= __shfl_xor_sync(0xffffffffu, w, 1);
+  w |= __shfl_xor_sync(0xffffffffu, w, 2);
+  if ((lane & 3) == 0) bits_tile[threadIdx.x >> 2] = w;
+  int c = __popc(byte);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if (lane == 0) red[warp] = c;
+  __syncthreads();
+  int total = 0;
+  if (threadIdx.x == 0)
+    for (int i = 0; i < kThreads / 32; ++i) total += red[i];
+  return total;
+}
+
+__global__ void __launch_bounds__(kThreads) k_predicate_mask(PredSet ps, ProbeSpec probe, int64_t n, uint32_t* bits,
+                                                             int32_t* block_counts, int* err) {
+  __shared__ int red[kThreads / 32];
+  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock + threadIdx.x * 8;
+  uint32_t byte = 0;
+  if (r0 < n) {
+    byte = r0 + 8 <= n ? 0xFFu : ((1u << (n - r0)) - 1u);
+    for (int i = 0; i < ps.n; ++i) byte &= eval_term(ps.p[i], r0, n);
+    if (probe.keys) {
+#pragma unroll 1
+      for (int j = 0; j < 8; ++j) {
+        if (byte & (1u << j)) {
+          const int m = probe_lookup(probe, static_cast<unsigned long long>(probe.keys[r0 + j]));
+          if (m < 0) byte &= ~(1u << j);
+          else probe.match_out[r0 + j] = m;
+        }
+      }
+    }
+  }
+  const int total = write_words_and_count(byte, bits + static_cast<int64_t>(blockIdx.x) * (kRowsPerBlock / 32), red);
+  if (threadIdx.x == 0) block_counts[blockIdx.x] = total;
+}
+
+// Block-wide exclusive scan of one int per thread (kThreads threads).
+__device__ __forceinline__ int block_excl_scan(int v, int* sh, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) sh[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int s = lane < kThreads / 32 ? sh[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int y = __shfl_up_sync(0xffffffffu, s, o);
+      if (lane >= o) s += y;
+    }
+    if (lane < kThreads / 32) sh[lane] = s;
+  }
+  __syncthreads();
+  const int before = warp ? sh[warp - 1] : 0;
+  *total = sh[kThreads / 32 - 1];
+  return before + x - v;
+}
+
+__global__ void __launch_bounds__(kThreads) k_compact(const uint32_t* bits, const int64_t* block_offsets, int64_t n,
+                                                      int32_t* ids, const int32_t* payload, int32_t* payload_out) {
+  __shared__ int sh[kThreads / 32];
+  const uint32_t word = bits[static_cast<int64_t>(blockIdx.x) * (kRowsPerBlock / 32) + (threadIdx.x >> 2)];
+  const uint32_t byte = (word >> (8 * (threadIdx.x & 3))) & 0xFFu;
+  int total;
+  const int pre = block_excl_scan(__popc(byte), sh, &total);
+  int64_t out = block_offsets[blockIdx.x] + pre;
+  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock + threadIdx.x * 8;
+  uint32_t b = byte;
+  while (b) {
+    const int j = __ffs(b) - 1;
+    b &= b - 1;
+    const int64_t r = r0 + j;
+    ids[out] = static_cast<int32_t>(r);
+    if (payload_out) payload_out[out] = payload[r];
+    ++out;
+  }
+}
+
+// ---------------------------------------------------------------- scans ---
+// Tile sums (2048 ints per block) -> single-block scan of the tile sums ->
+// per-tile scan with the tile's offset.
+
+__global__ void __launch_bounds__(kThreads) k_tile_sums(const int32_t* in, int64_t n, int64_t* sums) {
+  __shared__ int64_t red[kThreads / 32];
+  const int64_t base = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock;
+  int64_t s = 0;
+  for (int i = threadIdx.x; i < kRowsPerBlock; i += kThreads)
+    if (base + i < n) s += in[base + i];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int64_t t = 0;
+    for (int i = 0; i < kThreads / 32; ++i) t += red[i];
+    sums[blockIdx.x] = t;
+  }
+}
+
+// Exclusive scan of n int64 (or int32) values into out[0..n], one block of 1024
+// threads, each scanning a contiguous run sequentially.
+template <typename T>
+__global__ void __launch_bounds__(1024) k_scan_single(const T* in, int64_t n, int64_t* out) {
+  __shared__ int64_t sh[1024];
+  const int64_t per = (n + 1023) / 1024;
+  const int64_t b = threadIdx.x * per;
+  int64_t s = 0;
+  for (int64_t i = b; i < b + per && i < n; ++i) s += in[i];
+  sh[threadIdx.x] = s;
+  __syncthreads();
+  for (int o = 1; o < 1024; o <<= 1) {
+    int64_t y = threadIdx.x >= o ? sh[threadIdx.x - o] : 0;
+    __syncthreads();
+    sh[threadIdx.x] += y;
+    __syncthreads();
+  }
+  int64_t run = sh[threadIdx.x] - s;
+  for (int64_t i = b; i < b + per && i < n; ++i) {
+    out[i] = run;
+    run += in[i];
+  }
+  if (threadIdx.x == 1023) out[n] = sh[1023];
+}
+
+__global__ void __launch_bounds__(kThreads) k_tile_scan(const int32_t* in, int64_t n, const int64_t* tile_off,
+                                                        int64_t* out) {
+  __shared__ int sh[kThreads / 32];
+  const int64_t base = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock + threadIdx.x * 8;
+  int v[8];
+  int s = 0;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    v[j] = base + j < n ? in[base + j] : 0;
+    s += v[j];
+  }
+  int total;
+  int pre = block_excl_scan(s, sh, &total);
+  int64_t run = tile_off[blockIdx.x] + pre;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    if (base + j < n) out[base + j] = run;
+    run += v[j];
+  }
+  if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) out[n] = tile_off[gridDim.x];
+}
+
+// ----------------------------------------------------------- hash build ---
+
+__global__ void k_hash_build(const int64_t* keys, const int32_t* rows, int64_t n, unsigned long long* tk,
+                             int32_t* tv, int64_t cap, int* err) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const int32_t row = rows[i];
+  const unsigned long long key = static_cast<unsigned long long>(keys[row]);
+  if (key == kEmptyKey) {
+    set_dev_error(err, DEVERR_SENTINEL_KEY);
+    return;
+  }
+  const unsigned long long mask = static_cast<unsigned long long>(cap - 1);
+  unsigned long long slot = hash64(key) & mask;
+  for (int64_t step = 0; step < cap; ++step) {
+    const unsigned long long prev = atomicCAS(tk + slot, kEmptyKey, key);
+    if (prev == kEmptyKey) {
+      tv[slot] = row;
+      return;
+    }
+    if (prev == key) {
+      set_dev_error(err, DEVERR_DUP_BUILD_KEY);
+      return;
+    }
+    slot = (slot + 1) & mask;
+  }
+  set_dev_error(err, DEVERR_HASH_FULL);
+}
+
+__global__ void k_fill_u64(unsigned long long* p, int64_t n, unsigned long long v) {
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    p[i] = v;
+}
+
+// ------------------------------------------------------ decide/aggregate ---
+
+__global__ void __launch_bounds__(kThreads) k_decide(const float* logits, int64_t S, int K, int32_t* decision,
+                                                     uint32_t* yes_bits, int32_t* block_counts,
+                                                     unsigned long long* label_counts) {
+  __shared__ int red[kThreads / 32];
+  __shared__ unsigned int hist[16];
+  if (threadIdx.x < 16) hist[threadIdx.x] = 0;
+  __syncthreads();
+  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock + threadIdx.x * 8;
+  uint32_t byte = 0;
+  for (int j = 0; j < 8; ++j) {
+    const int64_t r = r0 + j;
+    if (r >= S) break;
+    const float* z = logits + r * K;
+    int d;
+    if (K == 2) {
+      d = z[0] > z[1] ? 1 : 0;  // strict: a tie is "no"
+      byte |= static_cast<uint32_t>(d) << j;
+      atomicAdd(&hist[d ? 0 : 1], 1u);
+    } else {
+      d = 0;
+      float best = z[0];
+      for (int k = 1; k < K; ++k)
+        if (z[k] > best) {
+          best = z[k];
+          d = k;
+        }
+      atomicAdd(&hist[d], 1u);
+    }
+    decision[r] = d;
+  }
+  const int total = write_words_and_count(byte, yes_bits + static_cast<int64_t>(blockIdx.x) * (kRowsPerBlock / 32), red);
+  if (threadIdx.x == 0) block_counts[blockIdx.x] = total;
+  if (threadIdx.x < K && hist[threadIdx.x]) atomicAdd(label_counts + threadIdx.x, (unsigned long long)hist[threadIdx.x]);
+}
+
+__global__ void k_group_build(const int32_t* decision, const int32_t* build_rows, int64_t S,
+                              unsigned long long* counts) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const bool yes = i < S && decision[i] == 1;
+  const unsigned active = __ballot_sync(0xffffffffu, yes);
+  if (!yes) return;
+  const int key = build_rows[i];
+  // lanes of the warp that hit the same group add once (skewed foreign keys)
+  const unsigned same = __match_any_sync(active, key);
+  if ((threadIdx.x & 31) == __ffs(same) - 1) atomicAdd(counts + key, (unsigned long long)__popc(same));
+}
+
+__global__ void __launch_bounds__(kThreads) k_nonzero_mask(const unsigned long long* counts, int64_t n, uint32_t* bits,
+                                                           int32_t* block_counts) {
+  __shared__ int red[kThreads / 32];
+  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock + threadIdx.x * 8;
+  uint32_t byte = 0;
+  for (int j = 0; j < 8; ++j)
+    if (r0 + j < n && counts[r0 + j] != 0) byte |= 1u << j;
+  const int total = write_words_and_count(byte, bits + static_cast<int64_t>(blockIdx.x) * (kRowsPerBlock / 32), red);
+  if (threadIdx.x == 0) block_counts[blockIdx.x] = total;
+}
+
+__global__ void k_gather_groups(const int32_t* rows, int64_t g, const int64_t* keys, const unsigned long long* counts,
+                                int64_t* keys_out, int64_t* counts_out) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= g) return;
+  const int32_t r = rows[i];
+  keys_out[i] = keys[r];
+  counts_out[i] = static_cast<int64_t>(counts[r]);
+}
+
+inline unsigned blocks_for(int64_t n, int64_t per) { return static_cast<unsigned>((n + per - 1) / per); }
+
+}  // namespace
+
+void launch_predicate_mask(const PredSet& ps, const ProbeSpec& probe, int64_t n_rows, uint32_t* bits,
+                           int32_t* block_counts, int* err, cudaStream_t s) {
+  if (n_rows <= 0) return;
+  k_predicate_mask<<<blocks_for(n_rows, kRowsPerBlock), kThreads, 0, s>>>(ps, probe, n_rows, bits, block_counts, err);
+}
+
+void launch_scan_counts(const int32_t* counts, int64_t n, int64_t* offsets, cudaStream_t s) {
+  k_scan_single<int32_t><<<1, 1024, 0, s>>>(counts, n, offsets);
+}
+
+void launch_compact(const uint32_t* bits, const int64_t* block_offsets, int64_t n_rows, int32_t* ids_out,
+                    const int32_t* payload, int32_t* payload_out, cudaStream_t s) {
+  if (n_rows <= 0) return;
+  k_compact<<<blocks_for(n_rows, kRowsPerBlock), kThreads, 0, s>>>(bits, block_offsets, n_rows, ids_out, payload,
+                                                                   payload_out);
+}
+
+void launch_hash_build(const int64_t* keys, const int32_t* rows, int64_t n, unsigned long long* table_keys,
+                       int32_t* table_vals, int64_t capacity, int* err, cudaStream_t s) {
+  if (n <= 0) return;
+  k_hash_build<<<blocks_for(n, 256), 256, 0, s>>>(keys, rows, n, table_keys, table_vals, capacity, err);
+}
+
+void launch_fill_u64(unsigned long long* p, int64_t n, unsigned long long v, cudaStream_t s) {
+  if (n <= 0) return;
+  const unsigned g = blocks_for(n, 256) < 4096 ? blocks_for(n, 256) : 4096;
+  k_fill_u64<<<g, 256, 0, s>>>(p, n, v);
+}
+
+void launch_scan_lengths(const int32_t* lens, int64_t S, int64_t* cu, int64_t* scratch_blocks, cudaStream_t s) {
+  // scratch_blocks: >= 2 * (tiles + 1) int64
+  const int64_t tiles = (S + kRowsPerBlock - 1) / kRowsPerBlock;
+  if (tiles == 0) {
+    cudaMemsetAsync(cu, 0, sizeof(int64_t), s);
+    return;
+  }
+  int64_t* sums = scratch_blocks;
+  int64_t* off = scratch_blocks + tiles + 1;
+  k_tile_sums<<<static_cast<unsigned>(tiles), kThreads, 0, s>>>(lens, S, sums);
+  k_scan_single<int64_t><<<1, 1024, 0, s>>>(sums, tiles, off);
+  k_tile_scan<<<static_cast<unsigned>(tiles), kThreads, 0, s>>>(lens, S, off, cu);
+}
+
+void launch_decide(const float* logits, int64_t S, int K, int32_t* decision, uint32_t* yes_bits,
+                   int32_t* block_counts, unsigned long long* label_counts, cudaStream_t s) {
+  if (S <= 0) return;
+  k_decide<<<blocks_for(S, kRowsPerBlock), kThreads, 0, s>>>(logits, S, K, decision, yes_bits, block_counts,
+                                                             label_counts);
+}
+
+void launch_group_build(const int32_t* decision, const int32_t* cand_build_rows, int64_t S,
+                        unsigned long long* group_counts, cudaStream_t s) {
+  if (S <= 0) return;
+  k_group_build<<<blocks_for(S, 256), 256, 0, s>>>(decision, cand_build_rows, S, group_counts);
+}
+
+void launch_nonzero_mask(const unsigned long long* counts, int64_t n, uint32_t* bits, int32_t* block_counts,
+                         cudaStream_t s) {
+  if (n <= 0) return;
+  k_nonzero_mask<<<blocks_for(n, kRowsPerBlock), kThreads, 0, s>>>(counts, n, bits, block_counts);
+}
+
+void launch_gather_groups(const int32_t* rows, int64_t g, const int64_t* build_keys,
+                          const unsigned long long* counts, int64_t* keys_out, int64_t* counts_out,
+                          cudaStream_t s) {
+  if (g <= 0) return;
+  k_gather_groups<<<blocks_for(g, 256), 256, 0, s>>>(rows, g, build_keys, counts, keys_out, counts_out);
+}
+
+}  // namespace aiq

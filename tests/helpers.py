@@ -1,0 +1,68 @@
+"""Shared test helpers: GPU availability, library handles, oracle comparisons."""
+from __future__ import annotations
+
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+# Margin tolerance and decision rule of the parity bar: label-logit margins
+# within 2e-2 * max(1, |ref|); decisions must agree wherever |ref margin| > 0.1.
+MARGIN_RTOL = 2e-2
+DECISION_MARGIN = 0.1
+
+
+def header_symbols():
+    syms = set()
+    for name in os.listdir(os.path.join(ROOT, "include")):
+        if name.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", name)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            syms |= set(re.findall(r"\b(aiq_\w+)\s*\(", src))
+    return sorted(syms)
+
+
+def gpu_ctx():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_10139_gb300 import aiq
+    return aiq.Context(0)
+
+
+def weights_list(shape, W):
+    import synth
+    return [W[n] for n, _, _ in synth.weight_specs(shape)]
+
+
+def oracle_preds(preds):
+    return [(p.column, p.op, p.value) for p in preds]
+
+
+def compare_logits(gpu_logits, ref_logits, what=""):
+    """Margin parity of K-label logits (rows aligned)."""
+    from oracle import relational as rel
+    gpu = np.asarray(gpu_logits, np.float64)
+    ref = np.asarray(ref_logits, np.float64)
+    assert gpu.shape == ref.shape, (gpu.shape, ref.shape)
+    if len(ref) == 0:
+        return 0.0
+    ref_dec = rel.decide(ref)
+    mr = rel.margins(ref, ref_dec)
+    mg = rel.margins(gpu, ref_dec)
+    tol = MARGIN_RTOL * np.maximum(1.0, np.abs(mr))
+    err = np.abs(mg - mr)
+    worst = float(np.max(err / tol))
+    assert np.all(err <= tol), f"{what} margin error {err.max():.4g} > tol (worst ratio {worst:.3f})"
+    gdec = rel.decide(gpu)
+    if ref.shape[1] == 2:
+        clear = np.abs(mr) > DECISION_MARGIN
+    else:
+        # the runner-up margin decides: clear when every other label is > 0.1 below k*
+        others = np.where(np.arange(ref.shape[1])[None, :] == ref_dec[:, None], -np.inf, mr)
+        clear = others.max(axis=1) < -DECISION_MARGIN
+    assert np.array_equal(gdec[clear], ref_dec[clear]), f"{what} decision mismatch on clear rows"
+    return worst

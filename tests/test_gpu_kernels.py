@@ -1,0 +1,158 @@
+"""Step-level parity of the prefill kernels (tcgen05 GEMM with each fused
+epilogue, RoPE table, RMSNorm, varlen GQA attention) against the oracle's
+fp64 definitions, through the C-ABI (aiq_ops.h)."""
+import numpy as np
+import pytest
+
+from helpers import gpu_ctx
+from oracle import transformer as tf
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    c = gpu_ctx()
+    yield c
+    c.close()
+
+
+def _h(a):
+    t = torch.as_tensor(np.ascontiguousarray(a)).cuda()
+    torch.cuda.synchronize()
+    return t
+
+
+def _np64(t):
+    torch.cuda.synchronize()
+    return t.float().cpu().numpy().astype(np.float64)
+
+
+def _close(got, ref, rtol, atol, what):
+    err = np.abs(got - ref)
+    bound = atol + rtol * np.abs(ref)
+    bad = err > bound
+    assert not bad.any(), f"{what}: {bad.sum()} of {bad.size} outside tol, max err {err.max():.3g}"
+
+
+GEMM_CASES = [  # M, N, K, bn
+    (1, 128, 64, 128),
+    (130, 384, 128, 128),
+    (257, 512, 192, 256),
+    (1000, 256, 2048, 256),
+    (8192, 1024, 512, 256),   # more tiles than SMs: persistent loop, both accumulators
+    (3000, 768, 1024, 128),
+]
+
+
+@pytest.mark.parametrize("M,N,K,bn", GEMM_CASES)
+def test_gemm_f16_store(ctx, M, N, K, bn):
+    rng = np.random.default_rng(M + N + K)
+    A = rng.standard_normal((M, K)).astype(np.float16)
+    B = (rng.standard_normal((N, K)) * 0.05).astype(np.float16)
+    dA, dB = _h(A), _h(B)
+    out = torch.zeros((M, N), dtype=torch.float16, device="cuda")
+    ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, bn, 0, out.data_ptr(), N)
+    ref = A.astype(np.float64) @ B.astype(np.float64).T
+    _close(_np64(out), ref, 2e-3, 2e-3 * np.sqrt(K) * 0.05, f"f16 M{M} N{N} K{K}")
+
+
+@pytest.mark.parametrize("M,N,K,bn", GEMM_CASES[:4])
+def test_gemm_residual_add(ctx, M, N, K, bn):
+    rng = np.random.default_rng(7 * M + N)
+    A = rng.standard_normal((M, K)).astype(np.float16)
+    B = (rng.standard_normal((N, K)) * 0.05).astype(np.float16)
+    R = rng.standard_normal((M, N)).astype(np.float32)
+    dA, dB, dR = _h(A), _h(B), _h(R)
+    ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, bn, 2, dR.data_ptr(), N)
+    ref = R.astype(np.float64) + A.astype(np.float64) @ B.astype(np.float64).T
+    _close(_np64(dR), ref, 1e-5, 2e-6 * np.sqrt(K), f"resid M{M} N{N} K{K}")
+
+
+@pytest.mark.parametrize("M,f,K,bn", [(130, 256, 128, 256), (700, 512, 256, 128), (2049, 1024, 512, 256)])
+def test_gemm_swiglu(ctx, M, f, K, bn):
+    rng = np.random.default_rng(M + f)
+    A = rng.standard_normal((M, K)).astype(np.float16)
+    Wg = (rng.standard_normal((f, K)) * 0.05).astype(np.float16)
+    Wu = (rng.standard_normal((f, K)) * 0.05).astype(np.float16)
+    ib = bn // 2
+    inter = np.concatenate([np.concatenate([Wg[b:b + ib], Wu[b:b + ib]]) for b in range(0, f, ib)])
+    dA, dB = _h(A), _h(inter)
+    out = torch.zeros((M, f), dtype=torch.float16, device="cuda")
+    ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, 2 * f, K, bn, 3, out.data_ptr(), f)
+    a = A.astype(np.float64)
+    ref = tf.silu(a @ Wg.astype(np.float64).T) * (a @ Wu.astype(np.float64).T)
+    _close(_np64(out), ref, 3e-3, 3e-3 * K * 0.0025, f"swiglu M{M} f{f}")
+
+
+def test_rope_table(ctx):
+    max_pos, hd, theta = 1200, 64, 1.0e4
+    cs = torch.zeros((max_pos, hd // 2), dtype=torch.float32, device="cuda")
+    sn = torch.zeros_like(cs)
+    ctx.op_rope_table(cs.data_ptr(), sn.data_ptr(), max_pos, hd, theta)
+    ang = np.arange(max_pos)[:, None] * theta ** (-(2.0 * np.arange(hd // 2)) / hd)[None, :]
+    assert np.allclose(cs.cpu().numpy(), np.cos(ang), rtol=0, atol=1.2e-7)
+    assert np.allclose(sn.cpu().numpy(), np.sin(ang), rtol=0, atol=1.2e-7)
+
+
+@pytest.mark.parametrize("hd,Hq,Hkv,bn", [(32, 4, 4, 128), (64, 32, 8, 256), (128, 8, 2, 256)])
+def test_gemm_qkv_rope(ctx, hd, Hq, Hkv, bn):
+    rng = np.random.default_rng(hd)
+    M, K = 300, 256
+    N = (Hq + 2 * Hkv) * hd
+    if N % bn:
+        bn = 128
+    A = rng.standard_normal((M, K)).astype(np.float16)
+    B = (rng.standard_normal((N, K)) * 0.05).astype(np.float16)
+    pos = rng.integers(0, 1100, M).astype(np.int32)
+    max_pos = 1200
+    cs = torch.zeros((max_pos, hd // 2), dtype=torch.float32, device="cuda")
+    sn = torch.zeros_like(cs)
+    ctx.op_rope_table(cs.data_ptr(), sn.data_ptr(), max_pos, hd, 1.0e4)
+    dA, dB, dP = _h(A), _h(B), _h(pos)
+    out = torch.zeros((M, N), dtype=torch.float16, device="cuda")
+    rope_cols = (Hq + Hkv) * hd
+    ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, bn, 1, out.data_ptr(), N, dP.data_ptr(),
+                cs.data_ptr(), sn.data_ptr(), rope_cols, hd)
+    y = A.astype(np.float64) @ B.astype(np.float64).T
+    qk = y[:, :rope_cols].reshape(M, Hq + Hkv, hd)
+    ref = np.concatenate([tf.rope(qk, pos, 1.0e4).reshape(M, rope_cols), y[:, rope_cols:]], axis=1)
+    _close(_np64(out), ref, 2e-3, 2e-3 * np.sqrt(K) * 0.05, f"rope hd{hd}")
+
+
+@pytest.mark.parametrize("d", [128, 2048, 4096])
+def test_rmsnorm(ctx, d):
+    rng = np.random.default_rng(d)
+    T = 333
+    x = (rng.standard_normal((T, d)) * 3).astype(np.float32)
+    import synth
+    gb = synth.f32_to_bf16_bits((1 + 0.02 * rng.standard_normal(d)).astype(np.float32))
+    dx, dg = _h(x), _h(gb.view(np.int16))
+    out = torch.zeros((T, d), dtype=torch.float16, device="cuda")
+    ctx.op_rmsnorm(dx.data_ptr(), T, d, dg.data_ptr(), 1e-5, out.data_ptr())
+    ref = tf.rmsnorm(x.astype(np.float64), tf.bf16_to_f64(gb), 1e-5)
+    _close(_np64(out), ref, 1.5e-3, 1e-4, f"rmsnorm d{d}")
+
+
+@pytest.mark.parametrize("hd,Hq,Hkv", [(32, 4, 4), (64, 8, 2), (128, 4, 1)])
+def test_attention_varlen(ctx, hd, Hq, Hkv):
+    rng = np.random.default_rng(hd + Hq)
+    lens = [1, 5, 64, 65, 130, 300, 17]
+    T = sum(lens)
+    W = (Hq + 2 * Hkv) * hd
+    qkv = rng.standard_normal((T, W)).astype(np.float16)
+    starts = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    dq, ds = _h(qkv), _h(starts)
+    out = torch.zeros((T, Hq * hd), dtype=torch.float16, device="cuda")
+    ctx.op_attention(dq.data_ptr(), T, ds.data_ptr(), len(lens), Hq, Hkv, hd, out.data_ptr())
+    got = _np64(out)
+    q64 = qkv.astype(np.float64)
+    for i, n in enumerate(lens):
+        s = starts[i]
+        seg = q64[s:s + n]
+        q = seg[:, :Hq * hd].reshape(n, Hq, hd)
+        k = seg[:, Hq * hd:(Hq + Hkv) * hd].reshape(n, Hkv, hd)
+        v = seg[:, (Hq + Hkv) * hd:].reshape(n, Hkv, hd)
+        ref = tf.causal_attention(q, k, v).reshape(n, Hq * hd)
+        _close(got[s:s + n], ref, 4e-3, 4e-3, f"attention seq {i} len {n} hd {hd}")
