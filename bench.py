@@ -1,0 +1,330 @@
+"""Benchmark of the unified AI query on GB300.
+
+Default workload: the select AI query at scale (100,000 rows; predicate
+rating >= 4 AND year >= 2000; lognormal text of median 120 tokens behind a
+64-token shared prefix; random-init 1B-shape decoder: d=2048, 16 layers,
+32/8 heads, head_dim 64, SwiGLU 8192, vocab 32000; yes/no decision; output the
+selected row ids and their count).  One step = one whole query over the
+resident table: predicate, compaction, packing, prefill, decision, aggregate.
+
+Prints one JSON line.  `value` is input rows/s over the device-timed steps
+(table and model resident in HBM); `e2e` repeats the metric through the C-ABI
+with host buffers (table upload, query, result download per step).
+`--impl reference` times the CPU oracle instead, on a bounded sample.
+"""
+from __future__ import annotations
+
+import argparse
+import dataclasses
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+L2_BYTES = 129 * 1024 * 1024
+
+# DRAM traffic of one tcgen05 GEMM launch from an ncu capture, valid only for the
+# GEMM source it was measured on (sha256 prefix of csrc/gemm_tcgen05.cu).
+GEMM_TRAFFIC = {"source_sha": None, "bytes_per_launch": None}
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default="c2_select_1b")
+    p.add_argument("--rows", type=int, default=0, help="override the table size (testing)")
+    p.add_argument("--e2e-steps", type=int, default=2)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-sample-rows", type=int, default=12)
+    return p.parse_args()
+
+
+def workload(args):
+    w = synth.WORKLOADS[args.workload]
+    if args.rows:
+        w = synth.scaled(w, args.rows)
+    return w
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        d = json.load(open(path))
+        return d, "measured"
+    return PEAKS_FALLBACK, "fallback"
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def gemm_source_sha():
+    src = os.path.join(ROOT, "paper_2608_10139_gb300", "csrc", "gemm_tcgen05.cu")
+    return hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+
+
+# ------------------------------------------------------------ CPU oracle ---
+
+def cpu_oracle_sample(w, q, W, n_rows: int, start: int = 0):
+    """The oracle on input rows [start, start + n_rows): relational terms, then
+    the fp64 transformer on the survivors, then the aggregate.  Returns
+    (seconds, rows, candidates)."""
+    from oracle import query as oq
+    from oracle import transformer as tf
+    sub = synth.Table(n_rows, {k: v[start:start + n_rows] for k, v in q.table.cols.items()},
+                      q.table.offsets[start:start + n_rows + 1] - q.table.offsets[start],
+                      q.table.tokens[q.table.offsets[start]:q.table.offsets[start + n_rows]])
+    preds = [(p.column, p.op, p.value) for p in w.preds]
+    t0 = time.perf_counter()
+    o = oq.run_select(sub, q.prefix, preds, w.label_ids, w.agg, tf.Model(w.model, W))
+    return time.perf_counter() - t0, n_rows, len(o.cand_rows)
+
+
+def reference_arm(args):
+    """The CPU oracle as it stands, timed on this host's cores, on a bounded
+    sample of the workload per step (rank 0 only)."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    w = workload(args)
+    q = synth.make_inputs(w)
+    W = synth.make_weights(w.model, w.weight_seed)
+    n = args.cpu_sample_rows
+    for i in range(args.warmup):
+        cpu_oracle_sample(w, q, W, n, start=(i * n) % (w.n_rows - n))
+    times, cands = [], 0
+    for k in range(args.steps):
+        s, _, c = cpu_oracle_sample(w, q, W, n, start=((args.warmup + k) * n) % (w.n_rows - n))
+        times.append(s)
+        cands += c
+    total = sum(times)
+    value = n * args.steps / total
+    line = {"impl": "reference", "metric": "AI-query input rows/s", "value": value, "unit": "rows/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000 * total / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "rows": w.n_rows, "model": "1B-shape decoder, random init",
+                       "sample_rows_per_step": n},
+            "cpu_baseline": {"value": value, "unit": "rows/s", "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": f"{n} consecutive input rows per step ({cands} LM candidates over "
+                                       f"{args.steps} steps), fp64 numpy"},
+            "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------- GPU arm ---
+
+def ours(args):
+    import torch
+    from paper_2608_10139_gb300 import aiq
+    from paper_2608_10139_gb300 import build as _build
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    _build.build()
+    w = workload(args)
+    if world > 1:   # weak scaling: every rank owns its own shard of the job's table
+        w = dataclasses.replace(w, data_seed=w.data_seed + 1000 * rank)
+    q = synth.make_inputs(w)
+    W = synth.make_weights(w.model, w.weight_seed)
+    tensors = [W[n] for n, _, _ in synth.weight_specs(w.model)]
+    preds = [(p.column, p.op, p.value) for p in w.preds]
+    ctx = aiq.Context(local)
+    model = ctx.load_model(w.model, tensors)
+    table = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+    stream = torch.cuda.ExternalStream(ctx.stream())
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    def step():
+        return ctx.run_select(table, model, preds, q.prefix, w.label_ids, agg=w.agg)
+
+    for _ in range(args.warmup):
+        step()
+    clocks = ClockSampler(local)
+    ctx.reset_kernel_stats()
+    ctx.set_option("profile", 1)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    ms, launches, res = [], 0, None
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    t_wall = time.perf_counter()
+    for k in range(args.steps):
+        flush.add_(1.0)                    # write 2x L2 between steps
+        torch.cuda.synchronize()
+        ev[k][0].record(stream)
+        res = step()
+        ev[k][1].record(stream)
+        launches += res.n_launches
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t_wall
+    barrier()
+    clk = clocks.stop()
+    ctx.set_option("profile", 0)
+    ms = [a.elapsed_time(b) for a, b in ev]
+    stats = ctx.kernel_stats()
+    total_ms = sum(ms)
+    if world > 1:
+        t = torch.tensor([total_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = world * w.n_rows / (ms_per_step / 1000.0)
+
+    # dominant kernel: the tcgen05 GEMM (all four epilogue variants, one kernel template)
+    g = [v for k, v in stats.items() if k.startswith("gemm_")]
+    gemm_ms = sum(v["total_ms"] for v in g)
+    gemm_launches = sum(v["launches"] for v in g)
+    gemm_flops = sum(v["flops"] for v in g)
+    pk, src = peaks()
+    peak = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+    achieved = gemm_flops / (gemm_ms / 1000.0) / 1e12 if gemm_ms else 0.0
+    traffic = GEMM_TRAFFIC["bytes_per_launch"] if GEMM_TRAFFIC["source_sha"] == gemm_source_sha() else None
+    step_ms = {k: round(v["total_ms"] / args.steps, 3) for k, v in sorted(stats.items())}
+
+    # end to end through the C-ABI with host buffers: upload table, query, download results
+    e2e_ms, h2d, d2h = [], q.table.nbytes(), 0
+    for _ in range(args.e2e_steps):
+        barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        t_e = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+        r = ctx.run_select(t_e, model, preds, q.prefix, w.label_ids, agg=w.agg)
+        ctx.free_table(t_e)
+        torch.cuda.synchronize()
+        e2e_ms.append(1000 * (time.perf_counter() - t0))
+        d2h = 4 * len(r.row_ids) + 8 * len(r.label_counts) + 8
+    e2e_per = statistics.median(e2e_ms) if e2e_ms else float("nan")
+    if world > 1:
+        t = torch.tensor([e2e_per], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_per = float(t.item())
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        s, n, c = cpu_oracle_sample(w, q, W, args.cpu_sample_rows)
+        cpu = {"value": n / s, "unit": "rows/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"first {n} input rows ({c} LM candidates), relational + fp64 transformer, numpy"}
+
+    if rank == 0:
+        line = {
+            "metric": "AI-query input rows/s", "value": value, "unit": "rows/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f16xf16->f32 (bf16 model values)", "data": "synthetic",
+            "config": {"workload": w.name, "rows": w.n_rows, "candidates": res.n_candidates,
+                       "tokens": res.n_tokens, "chunks": res.n_chunks,
+                       "model": "1B-shape decoder d2048 L16 32/8 heads hd64 ffn8192 V32000, random init",
+                       "l2": "2x L2 written between timed steps; weights and activations exceed L2",
+                       "parallelism": f"replicas x{world}"},
+            "p50_latency_ms": statistics.median(ms),
+            "wall_ms_per_step": 1000 * wall / args.steps,
+            "prefill_tflops": res.prefill_flops / (res.ms_prefill / 1000.0) / 1e12 if res.ms_prefill else None,
+            "prefill_tokens_per_s": res.n_tokens / (res.ms_prefill / 1000.0) if res.ms_prefill else None,
+            "phase_ms": {"relational": res.ms_relational, "prefill": res.ms_prefill,
+                         "aggregate": res.ms_aggregate},
+            "kernel_ms_per_step": step_ms,
+            "roofline": {"kernel": "gemm_tcgen05 (QKV+RoPE, O+residual, gate/up+SwiGLU, down+residual)",
+                         "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                         "frac": achieved / peak if peak else None, "traffic": traffic,
+                         "peak_source": f"{src} bf16_tflops_sustained (fp16 dense rate = bf16)",
+                         "launches": gemm_launches},
+            "cpu_baseline": cpu,
+            "e2e": {"value": world * w.n_rows / (e2e_per / 1000.0), "unit": "rows/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_per},
+            "gpu_launches": launches,
+            "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+    ctx.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        reference_arm(args)
+    else:
+        ours(args)
+
+
+if __name__ == "__main__":
+    main()

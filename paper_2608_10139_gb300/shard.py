@@ -1,0 +1,65 @@
+"""Row-range sharding of one AI query over replicas (one process per GPU).
+
+Rows are independent and the model is replicated, as in the paper's
+horizontal-scaling experiment (Table 5: the same program on every device,
+different micro-batches).  Each rank runs the whole query on a contiguous
+range of the table's rows; the only exchange is the merge of the small
+results at the end (counts summed, row ids concatenated in rank order, group
+counts summed per build row), never on the data path.
+"""
+from __future__ import annotations
+
+from typing import Dict, List, Sequence, Tuple
+
+import numpy as np
+
+
+def shard_range(n_rows: int, world: int, rank: int) -> Tuple[int, int]:
+    """Contiguous, balanced [lo, hi) of rank `rank` out of `world`."""
+    if world <= 0 or not 0 <= rank < world:
+        raise ValueError("bad rank/world")
+    base, extra = divmod(n_rows, world)
+    lo = rank * base + min(rank, extra)
+    return lo, lo + base + (1 if rank < extra else 0)
+
+
+def local_result(res, row_offset: int) -> Dict[str, np.ndarray]:
+    """The mergeable part of one rank's query result, with row ids made global."""
+    return {
+        "count": np.int64(res.count),
+        "n_candidates": np.int64(res.n_candidates),
+        "row_ids": res.row_ids.astype(np.int64) + row_offset,
+        "label_counts": res.label_counts.astype(np.int64),
+        "group_build_rows": res.group_build_rows.astype(np.int64),
+        "group_keys": res.group_keys.astype(np.int64),
+        "group_counts": res.group_counts.astype(np.int64),
+    }
+
+
+def merge(parts: Sequence[Dict[str, np.ndarray]]) -> Dict[str, np.ndarray]:
+    """Merge rank results given in rank order (rank r covers rows below rank r+1)."""
+    out = {
+        "count": np.int64(sum(int(p["count"]) for p in parts)),
+        "n_candidates": np.int64(sum(int(p["n_candidates"]) for p in parts)),
+        "row_ids": np.concatenate([p["row_ids"] for p in parts]) if parts else np.zeros(0, np.int64),
+    }
+    lcs = [p["label_counts"] for p in parts if len(p["label_counts"])]
+    out["label_counts"] = np.sum(lcs, axis=0) if lcs else np.zeros(0, np.int64)
+    groups: Dict[int, Tuple[int, int]] = {}
+    for p in parts:
+        for r, k, c in zip(p["group_build_rows"], p["group_keys"], p["group_counts"]):
+            key, prev = int(r), groups.get(int(r), (int(k), 0))
+            groups[key] = (prev[0], prev[1] + int(c))
+    rows = sorted(groups)
+    out["group_build_rows"] = np.array(rows, np.int64)
+    out["group_keys"] = np.array([groups[r][0] for r in rows], np.int64)
+    out["group_counts"] = np.array([groups[r][1] for r in rows], np.int64)
+    return out
+
+
+def gather_merge(part: Dict[str, np.ndarray], group=None) -> Dict[str, np.ndarray]:
+    """All-gather every rank's part (torch.distributed, any backend) and merge."""
+    import torch.distributed as dist
+    parts: List[Dict[str, np.ndarray]] = [None] * dist.get_world_size(group)
+    dist.all_gather_object(parts, part, group=group)
+    return merge(parts)

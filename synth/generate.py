@@ -11,8 +11,9 @@ Draw order (fixed, so that a seed names one table):
   join tables  : build ``movie_id`` (distinct 63-bit), build ``year``,
                  probe foreign-key ranks, probe text lengths, probe tokens,
                  prefix; the rank -> build row permutation comes last.
-  weights      : tensors in ``weight_specs`` order, one float32 standard
-                 normal block each.
+  weights      : tensor i of ``weight_specs`` drawn from its own PCG64
+                 stream, child i of SeedSequence(seed), as float32 standard
+                 normals (so tensors can be generated in parallel).
 """
 from __future__ import annotations
 
@@ -163,23 +164,31 @@ def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
     return (np.asarray(b, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
 
 
-def make_weights(s: ModelShape, seed: int, zero: bool = False) -> Dict[str, np.ndarray]:
+def _draw_tensor(seed_seq, shape, init) -> np.ndarray:
+    rng = np.random.Generator(np.random.PCG64(seed_seq))
+    n = int(np.prod(shape))
+    bits = np.empty(n, dtype=np.uint16)
+    step = 1 << 24
+    for i in range(0, n, step):
+        k = min(step, n - i)
+        x = rng.standard_normal(k, dtype=np.float32)
+        x *= np.float32(0.02)
+        if init == "gain":
+            x += np.float32(1.0)
+        bits[i:i + k] = f32_to_bf16_bits(x)
+    return bits.reshape(shape)
+
+
+def make_weights(s: ModelShape, seed: int, zero: bool = False, threads: int = 0) -> Dict[str, np.ndarray]:
     """Random-init bf16 weights (uint16 bit patterns), keyed by spec name."""
-    rng = np.random.Generator(np.random.PCG64(seed))
-    out = {}
-    for name, shape, init in weight_specs(s):
-        n = int(np.prod(shape))
-        if zero:
-            out[name] = np.zeros(shape, dtype=np.uint16)
-            continue
-        bits = np.empty(n, dtype=np.uint16)
-        step = 1 << 26
-        for i in range(0, n, step):
-            k = min(step, n - i)
-            x = rng.standard_normal(k, dtype=np.float32)
-            x *= np.float32(0.02)
-            if init == "gain":
-                x += np.float32(1.0)
-            bits[i:i + k] = f32_to_bf16_bits(x)
-        out[name] = bits.reshape(shape)
-    return out
+    import concurrent.futures as cf
+    import os
+    specs = weight_specs(s)
+    if zero:
+        return {name: np.zeros(shape, dtype=np.uint16) for name, shape, _ in specs}
+    children = np.random.SeedSequence(seed).spawn(len(specs))
+    threads = threads or min(16, os.cpu_count() or 1)
+    with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+        arrays = list(ex.map(lambda a: _draw_tensor(*a),
+                             [(c, shape, init) for c, (_, shape, init) in zip(children, specs)]))
+    return {name: a for (name, _, _), a in zip(specs, arrays)}

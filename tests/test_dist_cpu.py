@@ -1,0 +1,80 @@
+"""The N>1 host path on CPU: two gloo ranks each take a row range of the same
+table, compute their part of the query and all-gather the results; the merge
+equals the unsharded answer bit-exactly.  The per-rank query here is the
+oracle's relational part plus a fixed decision rule (no GPU is involved)."""
+import os
+import socket
+
+import numpy as np
+import pytest
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+import synth
+from oracle import query as oq
+from oracle import relational as rel
+from paper_2608_10139_gb300 import shard
+
+
+class _Res:
+    def __init__(self, **kw):
+        self.__dict__.update(kw)
+
+
+def _query(table, lo, hi, build_keys):
+    """Candidates of rows [lo, hi): rating >= 3; decision: token sum parity."""
+    sub = {k: v[lo:hi] for k, v in table.cols.items()}
+    cand = rel.compact(rel.predicate_mask(sub, [("rating", rel.GE, 3)], hi - lo))
+    dec = np.array([int(table.text(lo + c).sum()) % 2 for c in cand], np.int32)
+    gb = (lo + cand) % len(build_keys)
+    agg = oq.aggregate(oq.AGG_GROUP_BUILD_KEY, dec, cand, 2, gb, build_keys)
+    rows, keys, counts = agg["group_build_rows"], agg["group_keys"], agg["group_counts"]
+    return _Res(count=agg["count"], n_candidates=len(cand), row_ids=rel.yes_row_ids(dec, cand),
+                label_counts=rel.group_label_counts(dec, 2), group_build_rows=rows, group_keys=keys,
+                group_counts=counts)
+
+
+def _worker(rank, world, port, n, out_q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    q = synth.make_inputs(synth.scaled(synth.C1_TINY, n))
+    keys = np.arange(37, dtype=np.int64) * 1000 - 5
+    lo, hi = shard.shard_range(n, world, rank)
+    merged = shard.gather_merge(shard.local_result(_query(q.table, lo, hi, keys), lo))
+    if rank == 0:
+        out_q.put({k: np.asarray(v).tolist() for k, v in merged.items()})
+    dist.destroy_process_group()
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+@pytest.mark.parametrize("n", [1001, 4096])
+def test_two_rank_merge_equals_unsharded(n):
+    ctx = mp.get_context("spawn")
+    q_out = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, n, q_out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    merged = q_out.get(timeout=120)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    q = synth.make_inputs(synth.scaled(synth.C1_TINY, n))
+    keys = np.arange(37, dtype=np.int64) * 1000 - 5
+    full = shard.local_result(_query(q.table, 0, n, keys), 0)
+    for k in full:
+        assert np.array_equal(np.asarray(merged[k]), np.asarray(full[k])), k
+
+
+def test_shard_ranges_partition():
+    for n in (0, 1, 7, 100):
+        for world in (1, 2, 3, 8):
+            rs = [shard.shard_range(n, world, r) for r in range(world)]
+            assert rs[0][0] == 0 and rs[-1][1] == n
+            assert all(a[1] == b[0] for a, b in zip(rs, rs[1:]))
+            assert max(h - l for l, h in rs) - min(h - l for l, h in rs) <= 1

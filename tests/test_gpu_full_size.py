@@ -1,0 +1,114 @@
+"""Parity at the workloads' full sizes, in the launch configuration the
+benchmark times (default token budget): relational results and aggregates in
+full, bit-exact; label logits of a seeded sample of candidates against the
+fp64 oracle, each candidate row run alone."""
+from dataclasses import replace
+
+import numpy as np
+import pytest
+
+import synth
+from helpers import compare_logits, gpu_ctx, oracle_preds, weights_list
+from oracle import query as oq
+from oracle import relational as rel
+from oracle import transformer as tf
+from paper_2608_10139_gb300 import aiq
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    c = gpu_ctx()
+    yield c
+    c.close()
+
+
+def _sample(n_cand, k, seed, lens=None):
+    """k seeded candidate positions; always include the shortest and longest prompt."""
+    rng = np.random.default_rng(seed)
+    pick = set(rng.choice(n_cand, size=min(k, n_cand), replace=False).tolist())
+    if lens is not None and n_cand:
+        pick |= {int(np.argmin(lens)), int(np.argmax(lens))}
+    return np.array(sorted(pick), dtype=np.int64)
+
+
+def _run_select_full(ctx, w, k_sample):
+    q = synth.make_inputs(w)
+    W = synth.make_weights(w.model, w.weight_seed)
+    m = ctx.load_model(w.model, weights_list(w.model, W))
+    t = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+    preds = oracle_preds(w.preds)
+    r = ctx.run_select(t, m, preds, q.prefix, w.label_ids, agg=w.agg, flags=aiq.FLAG_LOGITS)
+    ctx.free_table(t)
+    ctx.free_model(m)
+    cand = rel.compact(rel.predicate_mask(q.table.cols, preds, q.table.n_rows))
+    assert np.array_equal(r.cand_row_ids, cand)
+    lens = np.diff(q.table.offsets)[cand]
+    assert r.n_tokens == int(lens.sum()) + len(q.prefix) * len(cand)
+    sample = _sample(len(cand), k_sample, w.data_seed, lens)
+    o = oq.run_select(q.table, q.prefix, preds, w.label_ids, w.agg, tf.Model(w.model, W), sample=sample)
+    compare_logits(r.label_logits[sample], o.logits, w.name)
+    agg = oq.aggregate(w.agg, r.decisions, cand, len(w.label_ids))
+    return r, agg
+
+
+def test_c2_select_1b_full_size(ctx):
+    r, agg = _run_select_full(ctx, synth.C2_SELECT, 10)
+    assert r.count == agg["count"] == len(r.row_ids)
+    assert np.array_equal(r.row_ids, agg["row_ids"])
+    # rating uniform 1..5 and year uniform 1950..2024: P = 2/5 * 25/75 = 13.3 %
+    assert abs(r.n_candidates / 100_000 - 0.4 * 25 / 75) < 0.005
+
+
+def test_c3_join_1b_full_size(ctx):
+    w = synth.C3_JOIN
+    q = synth.make_inputs(w)
+    W = synth.make_weights(w.model, w.weight_seed)
+    m = ctx.load_model(w.model, weights_list(w.model, W))
+    tb = ctx.load_table(q.build.cols, n_rows=q.build.n_rows)
+    tp = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+    bp = oracle_preds(w.join_build_preds)
+    r = ctx.run_join_select(tb, "movie_id", bp, tp, "movie_id", m, [], q.prefix, w.label_ids,
+                            agg=w.agg, flags=aiq.FLAG_LOGITS)
+    for h in (tb, tp):
+        ctx.free_table(h)
+    ctx.free_model(m)
+    cand, cand_b = oq.join_candidates(q.table, q.build, "movie_id", "movie_id", [], bp)
+    assert np.array_equal(r.cand_row_ids, cand)
+    assert np.array_equal(r.cand_build_rows, cand_b)
+    sample = _sample(len(cand), 8, w.data_seed)
+    o = oq.run_join_select(q.table, q.build, "movie_id", "movie_id", [], bp, q.prefix, w.label_ids, w.agg,
+                           tf.Model(w.model, W), sample=sample)
+    compare_logits(r.label_logits[sample], o.logits, w.name)
+    agg = oq.aggregate(w.agg, r.decisions, cand, 2, cand_b, q.build.cols["movie_id"])
+    assert np.array_equal(r.group_build_rows, agg["group_build_rows"])
+    assert np.array_equal(r.group_keys, agg["group_keys"])
+    assert np.array_equal(r.group_counts, agg["group_counts"])
+    assert int(r.group_counts.sum()) == r.count == agg["count"]
+
+
+@pytest.mark.slow
+def test_c4_multilabel_8b_full_size(ctx):
+    r, agg = _run_select_full(ctx, synth.C4_MULTILABEL, 3)
+    assert np.array_equal(r.label_counts, agg["label_counts"])
+    assert r.label_counts.sum() == r.n_candidates
+
+
+def test_c5_sweep_relational_all_points(ctx):
+    """Every selectivity point of the 1M-row sweep: candidates bit-exact."""
+    for point in synth.SWEEP_POINTS:
+        w = synth.sweep_workload(point, "fixed")
+        q = synth.make_inputs(w)
+        t = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+        preds = oracle_preds(w.preds)
+        r = ctx.run_select(t, 0, preds, q.prefix, w.label_ids, flags=aiq.FLAG_RELATIONAL_ONLY)
+        ctx.free_table(t)
+        want = rel.compact(rel.predicate_mask(q.table.cols, preds, q.table.n_rows))
+        assert np.array_equal(r.cand_row_ids, want), point
+
+
+def test_c5_sweep_1pct_full_query(ctx):
+    w = synth.sweep_workload("1%", "lognormal")
+    r, agg = _run_select_full(ctx, w, 6)
+    assert np.array_equal(r.row_ids, agg["row_ids"])
