@@ -57,6 +57,40 @@ aiq_status aiq_op_rmsnorm(aiq_ctx* ctx, const float* x, int64_t T, int32_t d, co
 aiq_status aiq_op_attention(aiq_ctx* ctx, const void* qkv, int64_t T, const int32_t* seq_start, int32_t n_seqs,
                             int32_t Hq, int32_t Hkv, int32_t hd, void* out);
 
+/* One relational term for aiq_filter_compact_static: `column op constant` on a
+ * caller-owned device column of n_rows values (16-byte aligned).  INT32 and
+ * INT64 columns compare with `ivalue`, FLOAT32 columns with `fvalue`. */
+typedef struct {
+  const void* column; /* device pointer */
+  int32_t type;       /* AIQ_INT32, AIQ_INT64 or AIQ_FLOAT32 */
+  int32_t op;         /* aiq_cmp */
+  int64_t ivalue;
+  double fvalue;
+} aiq_term;
+
+/* Filter and compact without allocating: the ids (ascending, int32) of the rows
+ * of caller-owned device columns that satisfy every term, written to ids_out
+ * (device, room for n_rows ids), and their number to *count_out (device int64).
+ * The paper has no counterpart: this is for callers that must not allocate
+ * device memory while they run (work recorded into a CUDA graph, a worker
+ * confined to a fixed device arena, an operator inside another library's
+ * allocation-free loop).  It runs the same kernels as aiq_run_select's
+ * relational phase, asynchronously on `stream` (a cudaStream_t; NULL = the
+ * legacy default stream), with their scratch in one static device array of
+ * about 2.1 MB that every GPU loading the library keeps until the process exits.
+ *   - At most 16,777,216 rows per call (AIQ_ERR_CAPACITY beyond), 0..8 terms.
+ *   - No cudaMalloc, cudaFree or allocating library call is made.  The first
+ *     call on a device looks up the array's device address once
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture.
+ *   - All calls share the one array: two calls whose work overlaps on the GPU
+ *     (different streams, or different host threads on one device) race and
+ *     both results are undefined.  Calls ordered on one stream are safe; each
+ *     call rewrites every scratch word it reads.
+ *   - Errors are returned as aiq_status, described by aiq_last_error(). */
+aiq_status aiq_filter_compact_static(const aiq_term* terms, int32_t n_terms, int64_t n_rows, int32_t* ids_out,
+                                     int64_t* count_out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -65,6 +65,11 @@ class _View(C.Structure):
                 ("ms_total", C.c_float), ("prefill_flops", C.c_double), ("n_launches", C.c_int64)]
 
 
+class _Term(C.Structure):
+    _fields_ = [("column", C.c_void_p), ("type", C.c_int32), ("op", C.c_int32), ("ivalue", C.c_int64),
+                ("fvalue", C.c_double)]
+
+
 class _KStat(C.Structure):
     _fields_ = [("name", C.c_char_p), ("launches", C.c_int64), ("total_ms", C.c_double),
                 ("flops", C.c_double), ("bytes", C.c_double)]
@@ -97,6 +102,7 @@ _SIGS = {
     "aiq_op_rmsnorm": [C.c_void_p, C.c_void_p, C.c_int64, C.c_int32, C.c_void_p, C.c_float, C.c_void_p],
     "aiq_op_attention": [C.c_void_p, C.c_void_p, C.c_int64, C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32,
                          C.c_void_p],
+    "aiq_filter_compact_static": [C.POINTER(_Term), C.c_int32, C.c_int64, C.c_void_p, C.c_void_p, C.c_void_p],
 }
 
 
@@ -126,6 +132,16 @@ def load_library():
 def _check(status: int):
     if status != OK:
         raise AiqError(status, _lib.aiq_last_error().decode())
+
+
+def filter_compact_static(terms, n_rows: int, ids_out: int, count_out: int, stream: int = 0):
+    """Allocation-free filter + compaction on device columns (see aiq_ops.h).
+    terms: (device pointer, dtype code, op, constant) tuples; ids_out and
+    count_out are device pointers; runs asynchronously on `stream`."""
+    lib = load_library()
+    ts = [_Term(p, t, op, int(v) if t != FLOAT32 else 0, float(v)) for p, t, op, v in terms]
+    arr = (_Term * max(len(ts), 1))(*ts)
+    _check(lib.aiq_filter_compact_static(arr, len(ts), n_rows, ids_out or None, count_out or None, stream or None))
 
 
 def _i32(a) -> np.ndarray:

@@ -108,6 +108,8 @@ struct StatAcc {
 
 }  // namespace
 
+void aiq::set_error_message(const char* msg) { g_err = msg ? msg : ""; }
+
 struct aiq_ctx {
   int device = 0;
   int num_sms = 0;

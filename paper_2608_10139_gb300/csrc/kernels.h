@@ -120,4 +120,7 @@ void launch_gather_groups(const int32_t* rows, int64_t g, const int64_t* build_k
                           const unsigned long long* counts, int64_t* keys_out, int64_t* counts_out,
                           cudaStream_t s);
 
+// Sets the thread-local message that aiq_last_error() returns.
+void set_error_message(const char* msg);
+
 }  // namespace aiq
