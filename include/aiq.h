@@ -107,7 +107,7 @@ typedef struct {
 typedef struct {
   int64_t n_input_rows; /* rows scanned (probe side for joins) */
   int64_t n_candidates; /* rows that reached the language model */
-  int64_t n_tokens;     /* packed prompt tokens prefilled */
+  int64_t n_tokens;     /* prompt tokens of all candidates (prefix + row text each) */
   int64_t n_chunks;     /* token-budget chunks the prefill ran in */
   int64_t count;        /* number of "yes" rows (2 labels), else -1 */
   const int32_t* row_ids;
@@ -127,6 +127,7 @@ typedef struct {
   float ms_relational, ms_prefill, ms_aggregate, ms_total;
   double prefill_flops; /* executed: 2*params per token + 4*Hq*hd*L per causal pair + head */
   int64_t n_launches;   /* CUDA kernels this query launched */
+  int64_t n_prefill_tokens; /* tokens run through the decoder: the shared prefix once + every row's text */
 } aiq_result_view;
 
 typedef struct aiq_ctx aiq_ctx;

@@ -52,10 +52,13 @@ aiq_status aiq_op_rmsnorm(aiq_ctx* ctx, const float* x, int64_t T, int32_t d, co
  * qkv fp16 [T, (Hq + 2 Hkv) * hd]: q heads, then k heads, then v heads, with
  * rotary embeddings already applied.  seq_start int32 [n_seqs + 1] (device):
  * sequence i occupies rows [seq_start[i], seq_start[i+1]); seq_start[n_seqs]
- * = T.  Query head h reads key/value head h / (Hq / Hkv).  out fp16
- * [T, Hq * hd].  hd in {32, 64, 128}. */
+ * = T.  Query head h reads key/value head h / (Hq / Hkv).  prefix_kv
+ * (optional, P > 0): fp16 [P, 2 Hkv hd] keys then values of a shared prompt
+ * prefix at positions before every sequence, which every query also attends
+ * (the prefix's K/V are computed once per query and reused by every row).
+ * out fp16 [T, Hq * hd].  hd in {32, 64, 128}. */
 aiq_status aiq_op_attention(aiq_ctx* ctx, const void* qkv, int64_t T, const int32_t* seq_start, int32_t n_seqs,
-                            int32_t Hq, int32_t Hkv, int32_t hd, void* out);
+                            int32_t Hq, int32_t Hkv, int32_t hd, const void* prefix_kv, int32_t P, void* out);
 
 /* One relational term for aiq_filter_compact_static: `column op constant` on a
  * caller-owned device column of n_rows values (16-byte aligned).  INT32 and

@@ -62,7 +62,8 @@ class _View(C.Structure):
                 ("cand_row_ids", C.POINTER(C.c_int32)), ("cand_build_rows", C.POINTER(C.c_int32)),
                 ("label_logits", C.POINTER(C.c_float)), ("decisions", C.POINTER(C.c_int32)),
                 ("ms_relational", C.c_float), ("ms_prefill", C.c_float), ("ms_aggregate", C.c_float),
-                ("ms_total", C.c_float), ("prefill_flops", C.c_double), ("n_launches", C.c_int64)]
+                ("ms_total", C.c_float), ("prefill_flops", C.c_double), ("n_launches", C.c_int64),
+                ("n_prefill_tokens", C.c_int64)]
 
 
 class _Term(C.Structure):
@@ -101,7 +102,7 @@ _SIGS = {
     "aiq_op_rope_table": [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_float],
     "aiq_op_rmsnorm": [C.c_void_p, C.c_void_p, C.c_int64, C.c_int32, C.c_void_p, C.c_float, C.c_void_p],
     "aiq_op_attention": [C.c_void_p, C.c_void_p, C.c_int64, C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32,
-                         C.c_void_p],
+                         C.c_void_p, C.c_int32, C.c_void_p],
     "aiq_filter_compact_static": [C.POINTER(_Term), C.c_int32, C.c_int64, C.c_void_p, C.c_void_p, C.c_void_p],
 }
 
@@ -180,6 +181,7 @@ class Result:
     ms_total: float
     prefill_flops: float
     n_launches: int
+    n_prefill_tokens: int
 
 
 def _arr(ptr, n, dtype, shape=None):
@@ -297,7 +299,8 @@ class Context:
                 _arr(v.label_logits, s * k if v.label_logits else 0, np.float32,
                      (s, k) if v.label_logits else (0, k)),
                 _arr(v.decisions, s if v.decisions else 0, np.int32),
-                v.ms_relational, v.ms_prefill, v.ms_aggregate, v.ms_total, v.prefill_flops, v.n_launches)
+                v.ms_relational, v.ms_prefill, v.ms_aggregate, v.ms_total, v.prefill_flops, v.n_launches,
+                v.n_prefill_tokens)
         finally:
             self.lib.aiq_result_free(self.h, h)
 
@@ -349,5 +352,6 @@ class Context:
     def op_rmsnorm(self, x: int, T: int, d: int, g: int, eps: float, out: int):
         _check(self.lib.aiq_op_rmsnorm(self.h, x, T, d, g, eps, out))
 
-    def op_attention(self, qkv: int, T: int, seq_start: int, n_seqs: int, Hq: int, Hkv: int, hd: int, out: int):
-        _check(self.lib.aiq_op_attention(self.h, qkv, T, seq_start, n_seqs, Hq, Hkv, hd, out))
+    def op_attention(self, qkv: int, T: int, seq_start: int, n_seqs: int, Hq: int, Hkv: int, hd: int, out: int,
+                     prefix_kv: int = 0, P: int = 0):
+        _check(self.lib.aiq_op_attention(self.h, qkv, T, seq_start, n_seqs, Hq, Hkv, hd, prefix_kv or None, P, out))

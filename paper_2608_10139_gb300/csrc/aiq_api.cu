@@ -57,6 +57,7 @@ struct ColD {
   int64_t* offsets = nullptr;
   size_t bytes = 0;
   int64_t max_len = 0;   // TOKENS: longest row
+  int64_t min_len = 0;   // TOKENS: shortest row
   int64_t max_id = -1;   // TOKENS: largest token id
 };
 
@@ -378,27 +379,30 @@ aiq_status prefill_bufs(aiq_ctx* c, const ModelD& m, int64_t B, PrefillBufs* pb)
   return AIQ_OK;
 }
 
-// Decoder forward over one packed chunk of n_seqs rows / T tokens, then the
-// label head into logits[n_seqs, K].
-aiq_status run_chunk(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, int64_t n_seqs, const int32_t* labels,
-                     int K, float* logits) {
+// Decoder forward over one packed chunk of n_seqs sequences / T tokens.
+// pkv_in (optional): per-layer keys/values [L][P][2 Hkv hd] of the shared
+// prefix that every sequence attends; pkv_out (optional): where this pass
+// stores its own keys/values per layer (the prefix pass).
+aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, int64_t n_seqs, const __half* pkv_in,
+                      int P_in, __half* pkv_out) {
   const aiq_model_config& g = m.cfg;
   const int d = g.d_model, hd = g.head_dim, Hq = g.n_heads, Hkv = g.n_kv_heads, f = g.d_ffn;
   const int nqkv = (Hq + 2 * Hkv) * hd;
+  const int64_t ldkv = 2 * static_cast<int64_t>(Hkv) * hd;
   const int M = static_cast<int>(T);
   {
     ProfScope p(c, "attn_tiles+embed", 0, 0);
     launch_attn_tiles(b.seq_start, static_cast<int32_t>(n_seqs), b.tile_seq, b.tile_q0, b.n_tiles, nullptr, c->stream);
     launch_embed(b.tok, T, m.embed, d, b.resid, c->stream);
-    counted(c, 2);
+    counted(c, 1 + (T > 0));
   }
   const int n_tiles_max = static_cast<int>((T + 63) / 64 + n_seqs);
   for (int l = 0; l < g.n_layers; ++l) {
     const LayerD& L = m.layers[l];
     {
-      ProfScope p(c, "rmsnorm", 0, 12.0 * T * d / 2 * 1);
+      ProfScope p(c, "rmsnorm", 0, 0);
       launch_rmsnorm(b.resid, T, d, L.attn_norm, g.rms_eps, b.xn, c->d_err, c->stream);
-      counted(c, 1);
+      counted(c, T > 0);
     }
     GemmEpilogue e1;
     e1.kind = EPI_ROPE_F16;
@@ -411,11 +415,14 @@ aiq_status run_chunk(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, int
     e1.head_dim = hd;
     e1.err = c->d_err;
     AIQ_TRY(gemm(c, "gemm_qkv_rope", b.xn, d, L.wqkv, d, M, nqkv, d, m.bn_qkv, e1));
+    if (pkv_out && T > 0)
+      CUDA_TRY(cudaMemcpy2DAsync(pkv_out + l * T * ldkv, ldkv * sizeof(__half), b.qkv + Hq * hd,
+                                 nqkv * sizeof(__half), ldkv * sizeof(__half), T, cudaMemcpyDeviceToDevice, c->stream));
     {
       ProfScope p(c, "attention", 0, 0);
-      launch_attention(b.qkv, T, b.seq_start, b.tile_seq, b.tile_q0, n_tiles_max, b.n_tiles, Hq, Hkv, hd, b.att,
-                       c->d_err, c->stream);
-      counted(c, 1);
+      launch_attention(b.qkv, T, b.seq_start, b.tile_seq, b.tile_q0, n_tiles_max, b.n_tiles, Hq, Hkv, hd,
+                       pkv_in ? pkv_in + l * P_in * ldkv : nullptr, P_in, b.att, c->d_err, c->stream);
+      counted(c, n_tiles_max > 0);
     }
     GemmEpilogue e2;
     e2.kind = EPI_RESID_F32;
@@ -426,7 +433,7 @@ aiq_status run_chunk(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, int
     {
       ProfScope p(c, "rmsnorm", 0, 0);
       launch_rmsnorm(b.resid, T, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
-      counted(c, 1);
+      counted(c, T > 0);
     }
     GemmEpilogue e3;
     e3.kind = EPI_SWIGLU_F16;
@@ -436,12 +443,6 @@ aiq_status run_chunk(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, int
     AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, d, L.wgu, d, M, 2 * f, d, m.bn_gu, e3));
     AIQ_TRY(gemm(c, "gemm_down_resid", b.act, f, L.wd, f, M, d, f, m.bn_d, e2));
   }
-  {
-    ProfScope p(c, "label_head", 0, 0);
-    launch_label_head(b.resid, b.last_idx, n_seqs, d, m.final_norm, g.rms_eps, m.lm_head, m.lm_bias, labels, K, logits,
-                      c->stream);
-    counted(c, 1);
-  }
   return AIQ_OK;
 }
 
@@ -450,7 +451,8 @@ struct QueryState {
   int32_t* ids = nullptr;        // candidate (probe) rows
   int32_t* build_rows = nullptr; // joins
   float* logits = nullptr;       // [S, K]
-  int64_t T = 0, n_chunks = 0, pairs = 0;
+  int64_t T = 0, n_chunks = 0, pairs = 0;  // T: row tokens (prefix excluded)
+  int64_t P = 0;                            // prefix tokens, run once
 };
 
 aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_select* q, QueryState* st) {
@@ -485,10 +487,11 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
   const int64_t T = c->h_pin[0];
   st->T = T;
   st->pairs = c->h_pin[1];
-  const int64_t max_len = P + col.max_len;
-  int64_t B = std::max<int64_t>(c->token_budget, max_len);
+  st->P = P;
+  const int64_t max_len = col.max_len;  // longest row text; the prefix runs on its own
+  const int64_t B = std::max<int64_t>(std::max<int64_t>(c->token_budget, max_len), P);
   const int64_t step = B - max_len + 1;
-  const int64_t n_chunks = (T + step - 1) / step;
+  const int64_t n_chunks = std::max<int64_t>(1, (T + step - 1) / step);
   st->n_chunks = n_chunks;
   int64_t* chunk_d;
   AIQ_TRY(ws(c, "q.chunks", 2 * (n_chunks + 1), &chunk_d));
@@ -497,22 +500,41 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
   std::vector<int64_t> chunks(2 * (n_chunks + 1));
   CUDA_TRY(cudaMemcpyAsync(chunks.data(), chunk_d, chunks.size() * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream));
   AIQ_TRY(sync_and_check(c));
-  int64_t Bmax = 0;
+  int64_t Bmax = P;
   for (int64_t i = 0; i < n_chunks; ++i) Bmax = std::max(Bmax, chunks[2 * (i + 1) + 1] - chunks[2 * i + 1]);
-  AIQ_TRY(ensure_rope(c, m, static_cast<int>(max_len)));
+  AIQ_TRY(ensure_rope(c, m, static_cast<int>(P + max_len)));
   PrefillBufs pb;
   AIQ_TRY(prefill_bufs(c, m, std::max<int64_t>(Bmax, 64), &pb));
+  const aiq_model_config& g = m.cfg;
+  __half* pkv = nullptr;
+  float* prefix_last;
+  AIQ_TRY(ws(c, "pf.prefix_last", g.d_model, &prefix_last));
+  if (P > 0) {
+    // the shared prefix once: its per-layer keys/values and its last hidden state
+    AIQ_TRY(ws(c, "pf.prefix_kv", static_cast<int64_t>(g.n_layers) * P * 2 * g.n_kv_heads * g.head_dim, &pkv));
+    launch_pack_prefix(prefix_d, P, pb.tok, pb.pos, pb.seq_start, c->stream);
+    counted(c, 1);
+    AIQ_TRY(run_layers(c, m, pb, P, 1, nullptr, 0, pkv));
+    CUDA_TRY(cudaMemcpyAsync(prefix_last, pb.resid + static_cast<int64_t>(P - 1) * g.d_model, g.d_model * sizeof(float),
+                             cudaMemcpyDeviceToDevice, c->stream));
+  }
   for (int64_t i = 0; i < n_chunks; ++i) {
     const int64_t r0 = chunks[2 * i], r1 = chunks[2 * (i + 1)];
     const int64_t Tc = chunks[2 * (i + 1) + 1] - chunks[2 * i + 1];
     if (r1 <= r0) continue;
     {
       ProfScope p(c, "pack_chunk", 0, 0);
-      launch_pack_chunk(cu, st->ids, col.offsets, static_cast<const int32_t*>(col.data), prefix_d, P, r0, r1, pb.tok,
-                        pb.pos, pb.seq_start, pb.last_idx, c->stream);
+      launch_pack_chunk(cu, st->ids, col.offsets, static_cast<const int32_t*>(col.data), P, r0, r1, pb.tok, pb.pos,
+                        pb.seq_start, pb.last_idx, c->stream);
       counted(c, 1);
     }
-    AIQ_TRY(run_chunk(c, m, pb, Tc, r1 - r0, labels_d, K, logits + r0 * K));
+    AIQ_TRY(run_layers(c, m, pb, Tc, r1 - r0, pkv, static_cast<int>(P), nullptr));
+    {
+      ProfScope p(c, "label_head", 0, 0);
+      launch_label_head(pb.resid, pb.last_idx, prefix_last, r1 - r0, g.d_model, m.final_norm, g.rms_eps, m.lm_head,
+                        m.lm_bias, labels_d, K, logits + r0 * K, c->stream);
+      counted(c, 1);
+    }
   }
   return AIQ_OK;
 }
@@ -607,7 +629,8 @@ void finish_view(ResultH& R, const QueryState& st, int64_t n_input, int K, int a
   aiq_result_view& v = R.v;
   v.n_input_rows = n_input;
   v.n_candidates = st.S;
-  v.n_tokens = st.T;
+  v.n_tokens = st.T + st.P * st.S;
+  v.n_prefill_tokens = st.S > 0 ? st.T + st.P : 0;
   v.n_chunks = st.n_chunks;
   v.count = (K == 2 && !R.label_counts.empty()) ? R.label_counts[0] : -1;
   v.row_ids = R.row_ids.empty() ? nullptr : R.row_ids.data();
@@ -647,7 +670,8 @@ aiq_status validate_select(aiq_ctx* c, const TableD& t, const ModelD* m, const a
   if (q->agg == AIQ_AGG_GROUP_BUILD_KEY && q->n_labels != 2)
     return fail(AIQ_ERR_INVALID_ARG, "GROUP_BUILD_KEY needs exactly 2 labels (yes, no)");
   const int64_t max_len = q->prefix_len + t.cols[q->text_column].max_len;
-  if (max_len <= 0) return fail(AIQ_ERR_INVALID_ARG, "every prompt is empty");
+  if (q->prefix_len == 0 && t.cols[q->text_column].min_len == 0)
+    return fail(AIQ_ERR_INVALID_ARG, "a row with empty text needs a non-empty prefix (its prompt would be empty)");
   if (max_len > (1 << 20)) return fail(AIQ_ERR_UNSUPPORTED, "a prompt is longer than 2^20 tokens");
   (void)c;
   return AIQ_OK;
@@ -729,8 +753,9 @@ aiq_status run_query(aiq_ctx* c, const TableD* build, int32_t build_key, const a
   R.v.ms_total = t03;
   if (!rel_only && m) {
     const aiq_model_config& g = m->cfg;
-    R.v.prefill_flops = m->linear_flops_per_token * static_cast<double>(st.T) +
-                        4.0 * g.n_heads * g.head_dim * g.n_layers * static_cast<double>(st.pairs) +
+    const double pre = st.S > 0 ? static_cast<double>(st.P) : 0.0;
+    R.v.prefill_flops = m->linear_flops_per_token * (static_cast<double>(st.T) + pre) +
+                        4.0 * g.n_heads * g.head_dim * g.n_layers * (static_cast<double>(st.pairs) + pre * (pre + 1) / 2) +
                         2.0 * g.d_model * K * static_cast<double>(st.S);
   }
   ResultH& dst = new_result(c, out);
@@ -854,6 +879,7 @@ aiq_status aiq_load_table(aiq_ctx* c, const aiq_column* cols, int32_t n_cols, in
         free_table(c, t);
         return fail(AIQ_ERR_INVALID_ARG, "token offsets must start at 0");
       }
+      col.min_len = n_rows > 0 ? INT64_MAX : 0;
       for (int64_t r = 0; r < n_rows; ++r) {
         const int64_t len = a.offsets[r + 1] - a.offsets[r];
         if (len < 0) {
@@ -861,6 +887,7 @@ aiq_status aiq_load_table(aiq_ctx* c, const aiq_column* cols, int32_t n_cols, in
           return fail(AIQ_ERR_INVALID_ARG, "token offsets must be non-decreasing");
         }
         col.max_len = std::max(col.max_len, len);
+        col.min_len = std::min(col.min_len, len);
       }
       const int64_t ntok = a.offsets[n_rows];
       if (ntok >= (int64_t(1) << 31)) {
@@ -1151,7 +1178,7 @@ aiq_status aiq_op_rmsnorm(aiq_ctx* c, const float* x, int64_t T, int32_t d, cons
 }
 
 aiq_status aiq_op_attention(aiq_ctx* c, const void* qkv, int64_t T, const int32_t* seq_start, int32_t n_seqs,
-                            int32_t Hq, int32_t Hkv, int32_t hd, void* out) {
+                            int32_t Hq, int32_t Hkv, int32_t hd, const void* prefix_kv, int32_t P, void* out) {
   if (!c || !qkv || !seq_start || !out || T < 0 || n_seqs < 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv)
     return fail(AIQ_ERR_INVALID_ARG, "bad args");
   if (!(hd == 32 || hd == 64 || hd == 128)) return fail(AIQ_ERR_UNSUPPORTED, "hd must be 32, 64 or 128");
@@ -1163,8 +1190,10 @@ aiq_status aiq_op_attention(aiq_ctx* c, const void* qkv, int64_t T, const int32_
   AIQ_TRY(ws(c, "op.tile_q0", cap, &tile_q0));
   AIQ_TRY(ws(c, "op.n_tiles", 1, &n_tiles));
   launch_attn_tiles(seq_start, n_seqs, tile_seq, tile_q0, n_tiles, nullptr, c->stream);
+  if (P < 0 || (P > 0 && !prefix_kv)) return fail(AIQ_ERR_INVALID_ARG, "bad prefix");
   launch_attention(static_cast<const __half*>(qkv), T, seq_start, tile_seq, tile_q0, static_cast<int>(cap - 1),
-                   n_tiles, Hq, Hkv, hd, static_cast<__half*>(out), c->d_err, c->stream);
+                   n_tiles, Hq, Hkv, hd, static_cast<const __half*>(prefix_kv), P, static_cast<__half*>(out), c->d_err,
+                   c->stream);
   return sync_and_check(c);
 }
 

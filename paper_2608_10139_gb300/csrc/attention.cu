@@ -1,8 +1,10 @@
 // Causal grouped-query attention over the packed variable-length batch.
 //
 // Each CTA computes one 64-row query block of one sequence for one query
-// head; it walks the key/value blocks of the same sequence up to the block's
-// last query (attention never crosses a row boundary of the batch), with an
+// head; it walks the key/value blocks of the shared prompt prefix (computed
+// once per query, keys/values in prefix_kv) and then those of its own
+// sequence up to the block's last query (attention never crosses a row
+// boundary of the batch; every prefix position precedes every row token), with an
 // fp32 online softmax (running max and sum per query row) so the score matrix
 // is never materialised.  K/V blocks are double-buffered in shared memory with
 // cp.async; QK^T and PV run on m16n8k16 fp16 tensor-core MMAs with fp32
@@ -64,7 +66,8 @@ __device__ __forceinline__ void load_rows(__half* dst, const __half* src, int ro
 template <int HD>
 __global__ void __launch_bounds__(kThreads) k_attention(const __half* __restrict__ qkv, const int32_t* seq_start,
                                                         const int32_t* tile_seq, const int32_t* tile_q0,
-                                                        const int32_t* n_tiles, int Hq, int Hkv, float scale_log2,
+                                                        const int32_t* n_tiles, int Hq, int Hkv,
+                                                        const __half* __restrict__ prefix_kv, int P, float scale_log2,
                                                         __half* __restrict__ out) {
   constexpr int LDS = HD + 8;
   constexpr int KS = HD / 16;  // k-steps of QK^T
@@ -87,15 +90,27 @@ __global__ void __launch_bounds__(kThreads) k_attention(const __half* __restrict
   const __half* Kg = qkv + static_cast<int64_t>(st) * ld + (Hq + kvh) * HD;
   const __half* Vg = qkv + static_cast<int64_t>(st) * ld + (Hq + Hkv + kvh) * HD;
   const int q_end = min(q0 + BQ, len);
-  const int n_kv = (q_end + BKV - 1) / BKV;
+  const int n_pre = (P + BKV - 1) / BKV;  // blocks of prefix keys (positions 0..P-1)
+  const int n_kv = n_pre + (q_end + BKV - 1) / BKV;
+  const int64_t ldp = static_cast<int64_t>(2 * Hkv) * HD;
+  const __half* Kp = prefix_kv + kvh * HD;
+  const __half* Vp = prefix_kv + (Hkv + kvh) * HD;
+  auto load_kv = [&](int j, int buf) {
+    if (j < n_pre) {
+      load_rows<HD>(sK + buf * BKV * LDS, Kp, j * BKV, P, ldp);
+      load_rows<HD>(sV + buf * BKV * LDS, Vp, j * BKV, P, ldp);
+    } else {
+      load_rows<HD>(sK + buf * BKV * LDS, Kg, (j - n_pre) * BKV, len, ld);
+      load_rows<HD>(sV + buf * BKV * LDS, Vg, (j - n_pre) * BKV, len, ld);
+    }
+  };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gq = lane >> 2, tq = lane & 3;
   const int wrow0 = q0 + warp * 16;  // first query row of this warp (sequence-local)
 
   load_rows<HD>(sQ, Qg, q0, len, ld);
-  load_rows<HD>(sK, Kg, 0, len, ld);
-  load_rows<HD>(sV, Vg, 0, len, ld);
+  load_kv(0, 0);
   cp_async_commit();
 
   uint32_t qf[KS][4];
@@ -107,8 +122,7 @@ __global__ void __launch_bounds__(kThreads) k_attention(const __half* __restrict
   for (int j = 0; j < n_kv; ++j) {
     const int buf = j & 1;
     if (j + 1 < n_kv) {
-      load_rows<HD>(sK + (buf ^ 1) * BKV * LDS, Kg, (j + 1) * BKV, len, ld);
-      load_rows<HD>(sV + (buf ^ 1) * BKV * LDS, Vg, (j + 1) * BKV, len, ld);
+      load_kv(j + 1, buf ^ 1);
       cp_async_commit();
       cp_async_wait<1>();
     } else {
@@ -143,9 +157,11 @@ __global__ void __launch_bounds__(kThreads) k_attention(const __half* __restrict
         mma16816(sc[2 * np + 1], qf[kk], b[2], b[3]);
       }
     }
-    // scale into log2 units, mask future keys and keys past the sequence end
-    const int key0 = j * BKV;
-    const bool need_mask = (key0 + BKV - 1 > wrow0) || (key0 + BKV > len);
+    // scale into log2 units; mask prefix keys past P, future keys of the
+    // sequence and keys past its end
+    const bool pre = j < n_pre;
+    const int key0 = (pre ? j : j - n_pre) * BKV;
+    const bool need_mask = pre ? (key0 + BKV > P) : ((key0 + BKV - 1 > wrow0) || (key0 + BKV > len));
 #pragma unroll
     for (int n = 0; n < 8; ++n) {
 #pragma unroll
@@ -154,7 +170,7 @@ __global__ void __launch_bounds__(kThreads) k_attention(const __half* __restrict
         if (need_mask) {
           const int key = key0 + n * 8 + 2 * tq + (e & 1);
           const int qr = wrow0 + gq + 8 * (e >> 1);
-          if (key > qr || key >= len) v = -INFINITY;
+          if (pre ? key >= P : (key > qr || key >= len)) v = -INFINITY;
         }
         sc[n][e] = v;
       }
@@ -237,25 +253,28 @@ __global__ void __launch_bounds__(kThreads) k_attention(const __half* __restrict
 
 template <int HD>
 void launch_hd(const __half* qkv, const int32_t* seq_start, const int32_t* tile_seq, const int32_t* tile_q0,
-               int n_tiles_max, const int32_t* n_tiles_dev, int Hq, int Hkv, __half* out, cudaStream_t s) {
+               int n_tiles_max, const int32_t* n_tiles_dev, int Hq, int Hkv, const __half* pkv, int P, __half* out,
+               cudaStream_t s) {
   constexpr int LDS = HD + 8;
   const int smem = (BQ + 4 * BKV) * LDS * 2;
   cudaFuncSetAttribute(k_attention<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(HD));
   dim3 grid(n_tiles_max, Hq);
-  k_attention<HD><<<grid, kThreads, smem, s>>>(qkv, seq_start, tile_seq, tile_q0, n_tiles_dev, Hq, Hkv, scale_log2, out);
+  k_attention<HD><<<grid, kThreads, smem, s>>>(qkv, seq_start, tile_seq, tile_q0, n_tiles_dev, Hq, Hkv, pkv, P,
+                                               scale_log2, out);
 }
 
 }  // namespace
 
 void launch_attention(const __half* qkv, int64_t /*T*/, const int32_t* seq_start, const int32_t* tile_seq,
                       const int32_t* tile_q0, int n_tiles_max, const int32_t* n_tiles_dev, int Hq, int Hkv, int hd,
-                      __half* out, int* /*err*/, cudaStream_t s) {
+                      const __half* prefix_kv, int P, __half* out, int* /*err*/, cudaStream_t s) {
   if (n_tiles_max <= 0) return;
+  if (!prefix_kv) P = 0;
   switch (hd) {
-    case 32: launch_hd<32>(qkv, seq_start, tile_seq, tile_q0, n_tiles_max, n_tiles_dev, Hq, Hkv, out, s); break;
-    case 64: launch_hd<64>(qkv, seq_start, tile_seq, tile_q0, n_tiles_max, n_tiles_dev, Hq, Hkv, out, s); break;
-    case 128: launch_hd<128>(qkv, seq_start, tile_seq, tile_q0, n_tiles_max, n_tiles_dev, Hq, Hkv, out, s); break;
+    case 32: launch_hd<32>(qkv, seq_start, tile_seq, tile_q0, n_tiles_max, n_tiles_dev, Hq, Hkv, prefix_kv, P, out, s); break;
+    case 64: launch_hd<64>(qkv, seq_start, tile_seq, tile_q0, n_tiles_max, n_tiles_dev, Hq, Hkv, prefix_kv, P, out, s); break;
+    case 128: launch_hd<128>(qkv, seq_start, tile_seq, tile_q0, n_tiles_max, n_tiles_dev, Hq, Hkv, prefix_kv, P, out, s); break;
   }
 }
 

@@ -74,7 +74,8 @@ void launch_hash_build(const int64_t* keys, const int32_t* rows, int64_t n, unsi
 void launch_fill_u64(unsigned long long* p, int64_t n, unsigned long long v, cudaStream_t s);
 
 // ------------------------------------------------------------------ pack ---
-// lens[i] = prefix_len + text length of row ids[i]; *pairs += causal (q, k) pairs.
+// lens[i] = text length of row ids[i]; *pairs += causal (q, k) pairs of its tokens
+// (prefix keys included).
 void launch_row_lengths(const int64_t* offsets, const int32_t* ids, int64_t S, int32_t prefix_len, int32_t* lens,
                         unsigned long long* pairs, cudaStream_t s);
 // Exclusive scan of int32 lengths into int64 cu[S+1] (multi-block).
@@ -82,11 +83,14 @@ void launch_scan_lengths(const int32_t* lens, int64_t S, int64_t* cu, int64_t* s
 // chunk_rows[c] = first row whose start offset >= c * budget_step, c = 0..n_chunks.
 void launch_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64_t n_chunks, int64_t* chunk_rows,
                          cudaStream_t s);
-// Pack rows [r0, r1) of a chunk: tokens, positions, chunk-local cu_seqlens and last-token index,
-// and the attention q-tile list.
+// Pack rows [r0, r1) of a chunk: their own tokens at positions prefix_len + j,
+// chunk-local sequence starts and last-token index (-1 for a row without tokens).
 void launch_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,
-                       const int32_t* prefix, int32_t prefix_len, int64_t r0, int64_t r1, int32_t* tok,
-                       int32_t* pos, int32_t* seq_start, int32_t* last_idx, cudaStream_t s);
+                       int32_t prefix_len, int64_t r0, int64_t r1, int32_t* tok, int32_t* pos, int32_t* seq_start,
+                       int32_t* last_idx, cudaStream_t s);
+// The shared prefix as a single sequence at positions 0..P-1.
+void launch_pack_prefix(const int32_t* prefix, int32_t P, int32_t* tok, int32_t* pos, int32_t* seq_start,
+                        cudaStream_t s);
 // Attention work list of a chunk: one entry per (sequence, 64-row q block).
 void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t* tile_seq, int32_t* tile_q0,
                        int32_t* n_tiles_dev, int32_t* scratch, cudaStream_t s);
@@ -98,12 +102,15 @@ void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, fl
 void launch_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, cudaStream_t s);
 void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int* err,
                     cudaStream_t s);
+// prefix_kv (optional): [P, 2 Hkv hd] fp16 keys then values of a shared prefix that
+// every sequence's queries also attend (prefix positions precede the sequence).
 void launch_attention(const __half* qkv, int64_t T, const int32_t* seq_start, const int32_t* tile_seq,
                       const int32_t* tile_q0, int n_tiles_max, const int32_t* n_tiles_dev, int Hq, int Hkv,
-                      int hd, __half* out, int* err, cudaStream_t s);
-void launch_label_head(const float* resid, const int32_t* last_idx, int64_t n_rows, int d, const uint16_t* g,
-                       float eps, const uint16_t* lm_head, const uint16_t* lm_bias, const int32_t* labels,
-                       int n_labels, float* logits_out, cudaStream_t s);
+                      int hd, const __half* prefix_kv, int P, __half* out, int* err, cudaStream_t s);
+// last_idx[r] < 0 reads prefix_last (fp32 [d]) instead of a row of resid.
+void launch_label_head(const float* resid, const int32_t* last_idx, const float* prefix_last, int64_t n_rows, int d,
+                       const uint16_t* g, float eps, const uint16_t* lm_head, const uint16_t* lm_bias,
+                       const int32_t* labels, int n_labels, float* logits_out, cudaStream_t s);
 
 // ------------------------------------------------------------- aggregate ---
 // decision per row from logits [S, K] (K == 2: strict yes > no; K > 2: first argmax),

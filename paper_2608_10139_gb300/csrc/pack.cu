@@ -2,28 +2,32 @@
 //
 // Every candidate row's prompt is the shared prefix followed by the row's
 // tokens (Table 1, AI_IF row: the text column feeds the causal LM; the prompt
-// prefix is the instruction shared by all rows).  Rows are concatenated with
-// no padding; cu (int64 [S+1]) holds each row's start.  The prefill runs
-// over token-budget chunks of consecutive rows, the GPU counterpart of the
-// paper's scan over micro-batches (Section 3.2): row i belongs to chunk
-// floor(cu[i] / step), so a chunk never holds more than step + max_len tokens.
+// prefix is the instruction shared by all rows).  The prefix is run through
+// the decoder once per query and its keys/values are reused by every row
+// (causal attention makes the prefix's states independent of what follows),
+// so the packed batch holds only each row's own tokens, at positions
+// P, P+1, ...  Rows are concatenated with no padding; cu (int64 [S+1]) holds
+// each row's start.  The prefill runs over token-budget chunks of
+// consecutive rows, the GPU counterpart of the paper's scan over
+// micro-batches (Section 3.2): row i belongs to chunk floor(cu[i] / step), so
+// a chunk never holds more than step + max_len tokens.
 #include "common.cuh"
 #include "kernels.h"
 
 namespace aiq {
 namespace {
 
-// lens[i] = P + text length of row ids[i]; pairs += sum of len * (len + 1) / 2
-// (causal query-key pairs, for the executed-FLOP count).
+// lens[i] = text length of row ids[i]; pairs += len * P + len * (len + 1) / 2
+// (the causal query-key pairs its tokens attend, for the executed-FLOP count).
 __global__ void k_row_lengths(const int64_t* offsets, const int32_t* ids, int64_t S, int32_t P, int32_t* lens,
                               unsigned long long* pairs) {
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   unsigned long long pr = 0;
   if (i < S) {
     const int32_t r = ids[i];
-    const int64_t len = P + (offsets[r + 1] - offsets[r]);
+    const int64_t len = offsets[r + 1] - offsets[r];
     lens[i] = static_cast<int32_t>(len);
-    pr = static_cast<unsigned long long>(len * (len + 1) / 2);
+    pr = static_cast<unsigned long long>(len * P + len * (len + 1) / 2);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) pr += __shfl_xor_sync(0xffffffffu, pr, o);
@@ -49,9 +53,10 @@ __global__ void k_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64
   out[2 * c + 1] = cu[lo];
 }
 
-// One warp per row: prefix then the row's text tokens, positions restart at 0.
+// One warp per row: the row's tokens at positions P + j; a row with no tokens
+// of its own gets last_idx = -1 (its last position is the prefix's last).
 __global__ void k_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,
-                             const int32_t* prefix, int32_t P, int64_t r0, int64_t r1, int32_t* tok, int32_t* pos,
+                             int32_t P, int64_t r0, int64_t r1, int32_t* tok, int32_t* pos,
                              int32_t* seq_start, int32_t* last_idx) {
   const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
@@ -63,12 +68,12 @@ __global__ void k_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_
   const int32_t r = ids[i];
   const int32_t* src = text + offsets[r];
   for (int64_t j = lane; j < len; j += 32) {
-    tok[dst + j] = j < P ? prefix[j] : src[j - P];
-    pos[dst + j] = static_cast<int32_t>(j);
+    tok[dst + j] = src[j];
+    pos[dst + j] = static_cast<int32_t>(P + j);
   }
   if (lane == 0) {
     seq_start[w] = static_cast<int32_t>(dst);
-    last_idx[w] = static_cast<int32_t>(dst + len - 1);
+    last_idx[w] = len > 0 ? static_cast<int32_t>(dst + len - 1) : -1;
     if (i == r1 - 1) seq_start[w + 1] = static_cast<int32_t>(cu[r1] - base);
   }
 }
@@ -100,7 +105,24 @@ __global__ void __launch_bounds__(1024) k_attn_tiles(const int32_t* seq_start, i
   if (threadIdx.x == 0) *n_tiles = carry;
 }
 
+// The prefix as one sequence: tokens, positions 0..P-1, seq_start = {0, P}.
+__global__ void k_pack_prefix(const int32_t* prefix, int32_t P, int32_t* tok, int32_t* pos, int32_t* seq_start) {
+  for (int j = threadIdx.x; j < P; j += blockDim.x) {
+    tok[j] = prefix[j];
+    pos[j] = j;
+  }
+  if (threadIdx.x == 0) {
+    seq_start[0] = 0;
+    seq_start[1] = P;
+  }
+}
+
 }  // namespace
+
+void launch_pack_prefix(const int32_t* prefix, int32_t P, int32_t* tok, int32_t* pos, int32_t* seq_start,
+                        cudaStream_t s) {
+  k_pack_prefix<<<1, 256, 0, s>>>(prefix, P, tok, pos, seq_start);
+}
 
 void launch_row_lengths(const int64_t* offsets, const int32_t* ids, int64_t S, int32_t prefix_len, int32_t* lens,
                         unsigned long long* pairs, cudaStream_t s) {
@@ -114,12 +136,12 @@ void launch_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64_t n_c
 }
 
 void launch_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,
-                       const int32_t* prefix, int32_t prefix_len, int64_t r0, int64_t r1, int32_t* tok,
-                       int32_t* pos, int32_t* seq_start, int32_t* last_idx, cudaStream_t s) {
+                       int32_t prefix_len, int64_t r0, int64_t r1, int32_t* tok, int32_t* pos, int32_t* seq_start,
+                       int32_t* last_idx, cudaStream_t s) {
   if (r1 <= r0) return;
   const int64_t threads = (r1 - r0) * 32;
-  k_pack_chunk<<<static_cast<unsigned>((threads + 255) / 256), 256, 0, s>>>(cu, ids, offsets, text, prefix, prefix_len,
-                                                                            r0, r1, tok, pos, seq_start, last_idx);
+  k_pack_chunk<<<static_cast<unsigned>((threads + 255) / 256), 256, 0, s>>>(cu, ids, offsets, text, prefix_len, r0, r1,
+                                                                            tok, pos, seq_start, last_idx);
 }
 
 void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t* tile_seq, int32_t* tile_q0,

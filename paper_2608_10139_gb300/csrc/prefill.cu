@@ -123,13 +123,14 @@ __global__ void k_rmsnorm_any(const float* x, int64_t T, int d, const uint16_t* 
 
 // One warp per candidate row: final RMSNorm of the last token's hidden state,
 // then K dot products with the label rows of the LM head plus its bias.
-__global__ void k_label_head(const float* resid, const int32_t* last_idx, int64_t n, int d, const uint16_t* g,
-                             float eps, const uint16_t* W, const uint16_t* bias, const int32_t* labels, int K,
-                             float* logits) {
+__global__ void k_label_head(const float* resid, const int32_t* last_idx, const float* prefix_last, int64_t n, int d,
+                             const uint16_t* g, float eps, const uint16_t* W, const uint16_t* bias,
+                             const int32_t* labels, int K, float* logits) {
   const int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (r >= n) return;
-  const float* x = resid + static_cast<int64_t>(last_idx[r]) * d;
+  const int32_t li = last_idx[r];
+  const float* x = li >= 0 ? resid + static_cast<int64_t>(li) * d : prefix_last;
   float ss = 0.f;
   for (int c = lane; c < d; c += 32) ss += x[c] * x[c];
   ss = warp_sum(ss);
@@ -184,12 +185,12 @@ void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float e
   }
 }
 
-void launch_label_head(const float* resid, const int32_t* last_idx, int64_t n_rows, int d, const uint16_t* g,
-                       float eps, const uint16_t* lm_head, const uint16_t* lm_bias, const int32_t* labels,
-                       int n_labels, float* logits_out, cudaStream_t s) {
+void launch_label_head(const float* resid, const int32_t* last_idx, const float* prefix_last, int64_t n_rows, int d,
+                       const uint16_t* g, float eps, const uint16_t* lm_head, const uint16_t* lm_bias,
+                       const int32_t* labels, int n_labels, float* logits_out, cudaStream_t s) {
   if (n_rows <= 0) return;
-  k_label_head<<<grid_for(n_rows * 32), 256, 0, s>>>(resid, last_idx, n_rows, d, g, eps, lm_head, lm_bias, labels,
-                                                     n_labels, logits_out);
+  k_label_head<<<grid_for(n_rows * 32), 256, 0, s>>>(resid, last_idx, prefix_last, n_rows, d, g, eps, lm_head,
+                                                     lm_bias, labels, n_labels, logits_out);
 }
 
 }  // namespace aiq

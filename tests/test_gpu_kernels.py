@@ -156,3 +156,29 @@ def test_attention_varlen(ctx, hd, Hq, Hkv):
         v = seg[:, (Hq + Hkv) * hd:].reshape(n, Hkv, hd)
         ref = tf.causal_attention(q, k, v).reshape(n, Hq * hd)
         _close(got[s:s + n], ref, 4e-3, 4e-3, f"attention seq {i} len {n} hd {hd}")
+
+
+@pytest.mark.parametrize("hd,Hq,Hkv,P", [(32, 4, 4, 16), (64, 8, 2, 64), (64, 8, 2, 70), (128, 4, 1, 130)])
+def test_attention_with_shared_prefix(ctx, hd, Hq, Hkv, P):
+    """Rows attend a shared prefix's keys/values plus their own: the output at
+    each row token equals the oracle's attention over prefix ++ row at that position."""
+    rng = np.random.default_rng(P + hd)
+    lens = [1, 5, 64, 65, 130, 17]
+    T = sum(lens)
+    W = (Hq + 2 * Hkv) * hd
+    pre = rng.standard_normal((P, W)).astype(np.float16)
+    rows = rng.standard_normal((T, W)).astype(np.float16)
+    pkv = np.ascontiguousarray(pre[:, Hq * hd:])            # [P, 2 Hkv hd]: keys then values
+    starts = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    dq, ds, dp = _h(rows), _h(starts), _h(pkv)
+    out = torch.zeros((T, Hq * hd), dtype=torch.float16, device="cuda")
+    ctx.op_attention(dq.data_ptr(), T, ds.data_ptr(), len(lens), Hq, Hkv, hd, out.data_ptr(), dp.data_ptr(), P)
+    got = _np64(out)
+    for i, n in enumerate(lens):
+        seq = np.concatenate([pre, rows[starts[i]:starts[i] + n]]).astype(np.float64)
+        m = P + n
+        q = seq[:, :Hq * hd].reshape(m, Hq, hd)
+        k = seq[:, Hq * hd:(Hq + Hkv) * hd].reshape(m, Hkv, hd)
+        v = seq[:, (Hq + Hkv) * hd:].reshape(m, Hkv, hd)
+        ref = tf.causal_attention(q, k, v).reshape(m, Hq * hd)[P:]
+        _close(got[starts[i]:starts[i] + n], ref, 4e-3, 4e-3, f"prefix attention P{P} seq {i} len {n}")

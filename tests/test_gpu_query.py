@@ -130,6 +130,8 @@ def _select_parity(ctx, w, budget=None):
         assert np.array_equal(r.label_counts, agg["label_counts"])
     n_tok = sum(len(q.prefix) + len(q.table.text(i)) for i in o.cand_rows)
     assert r.n_tokens == n_tok
+    if len(o.cand_rows):   # the shared prefix runs once; each row runs only its own tokens
+        assert r.n_prefill_tokens == n_tok - len(q.prefix) * (len(o.cand_rows) - 1)
     ctx.free_table(t)
     ctx.free_model(mh)
     return r
@@ -178,6 +180,32 @@ def test_tiny_join_group_by_build_key(ctx):
     assert np.array_equal(r.group_keys, agg["group_keys"])
     assert np.array_equal(r.group_counts, agg["group_counts"])
     assert int(r.group_counts.sum()) == r.count
+
+
+def test_rows_with_empty_text(ctx):
+    """A row whose text is empty is decided on the prefix alone; with no prefix
+    such a row's prompt would be empty, which is refused."""
+    w = synth.C1_TINY
+    q = synth.make_inputs(w)
+    lens = np.diff(q.table.offsets)
+    lens[::7] = 0                                   # every 7th row loses its text
+    offsets = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    tokens = np.concatenate([q.table.text(i)[:lens[i]] for i in range(q.table.n_rows)]).astype(np.int32)
+    table = synth.Table(q.table.n_rows, q.table.cols, offsets, tokens)
+    mh, W = _model(ctx, w.model, w.weight_seed)
+    t = _load(ctx, table)
+    preds = oracle_preds(w.preds)
+    r = ctx.run_select(t, mh, preds, q.prefix, w.label_ids, agg=w.agg, flags=aiq.FLAG_LOGITS)
+    o = oq.run_select(table, q.prefix, preds, w.label_ids, w.agg, tf.Model(w.model, W, True))
+    assert np.array_equal(r.cand_row_ids, o.cand_rows)
+    compare_logits(r.label_logits, o.logits, "empty-text rows")
+    empty = np.diff(offsets)[o.cand_rows] == 0
+    assert empty.sum() > 5 and np.all(r.label_logits[empty] == r.label_logits[empty][0])
+    with pytest.raises(aiq.AiqError) as e:
+        ctx.run_select(t, mh, preds, np.zeros(0, np.int32), w.label_ids)
+    assert e.value.status == aiq.ERR_INVALID_ARG
+    ctx.free_table(t)
+    ctx.free_model(mh)
 
 
 def test_degenerate_queries(ctx):
