@@ -140,93 +140,108 @@ __global__ void __launch_bounds__(kThreads) k_attention(const __half* __restrict
     }
     const __half* kb = sK + buf * BKV * LDS;
     const __half* vb = sV + buf * BKV * LDS;
-
-    float sc[8][4];
-#pragma unroll
-    for (int n = 0; n < 8; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < KS; ++kk) {
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        const int mat = lane >> 3;
-        const int key = np * 16 + (lane & 7) + 8 * (mat >> 1);
-        const int dim = kk * 16 + 8 * (mat & 1);
-        uint32_t b[4];
-        ldsm_x4(b, kb + key * LDS + dim);
-        mma16816(sc[2 * np], qf[kk], b[0], b[1]);
-        mma16816(sc[2 * np + 1], qf[kk], b[2], b[3]);
-      }
-    }
-    // scale into log2 units; mask prefix keys past P, future keys of the
-    // sequence and keys past its end
     const bool pre = j < n_pre;
     const int key0 = (pre ? j : j - n_pre) * BKV;
-    const bool need_mask = pre ? (key0 + BKV > P) : ((key0 + BKV - 1 > wrow0) || (key0 + BKV > len));
+    // 8-key column tiles this warp needs: all for prefix blocks, up to its last
+    // query row on the causal diagonal; none when every row of the warp lies
+    // past the sequence end (warp-uniform, so whole MMAs are skipped)
+    int n_lim = 8;
+    if (!pre) {
+      const int last_row = min(wrow0 + 15, len - 1);
+      n_lim = last_row < key0 ? 0 : min(8, (last_row - key0) / 8 + 1);
+    }
+    if (wrow0 >= len) n_lim = 0;
+
+    if (n_lim > 0) {
+      float sc[8][4];
 #pragma unroll
-    for (int n = 0; n < 8; ++n) {
+      for (int n = 0; n < 8; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        float v = sc[n][e] * scale_log2;
-        if (need_mask) {
-          const int key = key0 + n * 8 + 2 * tq + (e & 1);
-          const int qr = wrow0 + gq + 8 * (e >> 1);
-          if (pre ? key >= P : (key > qr || key >= len)) v = -INFINITY;
+      for (int kk = 0; kk < KS; ++kk) {
+#pragma unroll
+        for (int np = 0; np < 4; ++np) {
+          if (2 * np < n_lim) {
+            const int mat = lane >> 3;
+            const int key = np * 16 + (lane & 7) + 8 * (mat >> 1);
+            const int dim = kk * 16 + 8 * (mat & 1);
+            uint32_t b[4];
+            ldsm_x4(b, kb + key * LDS + dim);
+            mma16816(sc[2 * np], qf[kk], b[0], b[1]);
+            mma16816(sc[2 * np + 1], qf[kk], b[2], b[3]);
+          }
         }
-        sc[n][e] = v;
       }
-    }
-    float mx0 = -INFINITY, mx1 = -INFINITY;
+      // scale into log2 units; mask prefix keys past P, future keys of the
+      // sequence, keys past its end and the column tiles skipped above
+      const bool need_mask = pre ? (key0 + BKV > P) : ((key0 + BKV - 1 > wrow0) || (key0 + BKV > len));
 #pragma unroll
-    for (int n = 0; n < 8; ++n) {
-      mx0 = fmaxf(mx0, fmaxf(sc[n][0], sc[n][1]));
-      mx1 = fmaxf(mx1, fmaxf(sc[n][2], sc[n][3]));
-    }
+      for (int n = 0; n < 8; ++n) {
 #pragma unroll
-    for (int o2 = 1; o2 <= 2; o2 <<= 1) {
-      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o2));
-      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o2));
-    }
-    const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-    const float base0 = mn0 == -INFINITY ? 0.f : mn0;
-    const float base1 = mn1 == -INFINITY ? 0.f : mn1;
-    const float c0 = exp2f(m0 - base0), c1 = exp2f(m1 - base1);
-    m0 = mn0;
-    m1 = mn1;
-    float rs0 = 0.f, rs1 = 0.f;
+        for (int e = 0; e < 4; ++e) {
+          float v = sc[n][e] * scale_log2;
+          if (need_mask) {
+            const int key = key0 + n * 8 + 2 * tq + (e & 1);
+            const int qr = wrow0 + gq + 8 * (e >> 1);
+            if (pre ? key >= P : (key > qr || key >= len)) v = -INFINITY;
+          }
+          sc[n][e] = v;
+        }
+      }
+      float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
-    for (int n = 0; n < 8; ++n) {
-      sc[n][0] = exp2f(sc[n][0] - base0);
-      sc[n][1] = exp2f(sc[n][1] - base0);
-      sc[n][2] = exp2f(sc[n][2] - base1);
-      sc[n][3] = exp2f(sc[n][3] - base1);
-      rs0 += sc[n][0] + sc[n][1];
-      rs1 += sc[n][2] + sc[n][3];
-    }
-    l0 = l0 * c0 + rs0;
-    l1 = l1 * c1 + rs1;
+      for (int n = 0; n < 8; ++n) {
+        mx0 = fmaxf(mx0, fmaxf(sc[n][0], sc[n][1]));
+        mx1 = fmaxf(mx1, fmaxf(sc[n][2], sc[n][3]));
+      }
 #pragma unroll
-    for (int i = 0; i < DN; ++i) {
-      o[i][0] *= c0;
-      o[i][1] *= c0;
-      o[i][2] *= c1;
-      o[i][3] *= c1;
-    }
+      for (int o2 = 1; o2 <= 2; o2 <<= 1) {
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o2));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o2));
+      }
+      const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+      const float base0 = mn0 == -INFINITY ? 0.f : mn0;
+      const float base1 = mn1 == -INFINITY ? 0.f : mn1;
+      const float c0 = exp2f(m0 - base0), c1 = exp2f(m1 - base1);
+      m0 = mn0;
+      m1 = mn1;
+      float rs0 = 0.f, rs1 = 0.f;
 #pragma unroll
-    for (int k2 = 0; k2 < 4; ++k2) {
-      uint32_t pa[4];
-      pa[0] = pack_h2(sc[2 * k2][0], sc[2 * k2][1]);
-      pa[1] = pack_h2(sc[2 * k2][2], sc[2 * k2][3]);
-      pa[2] = pack_h2(sc[2 * k2 + 1][0], sc[2 * k2 + 1][1]);
-      pa[3] = pack_h2(sc[2 * k2 + 1][2], sc[2 * k2 + 1][3]);
+      for (int n = 0; n < 8; ++n) {
+        sc[n][0] = exp2f(sc[n][0] - base0);
+        sc[n][1] = exp2f(sc[n][1] - base0);
+        sc[n][2] = exp2f(sc[n][2] - base1);
+        sc[n][3] = exp2f(sc[n][3] - base1);
+        rs0 += sc[n][0] + sc[n][1];
+        rs1 += sc[n][2] + sc[n][3];
+      }
+      l0 = l0 * c0 + rs0;
+      l1 = l1 * c1 + rs1;
 #pragma unroll
-      for (int dp = 0; dp < DN / 2; ++dp) {
-        const int mat = lane >> 3;
-        const int key = k2 * 16 + (lane & 7) + 8 * (mat & 1);
-        const int dim = dp * 16 + 8 * (mat >> 1);
-        uint32_t b[4];
-        ldsm_x4_t(b, vb + key * LDS + dim);
-        mma16816(o[2 * dp], pa, b[0], b[1]);
-        mma16816(o[2 * dp + 1], pa, b[2], b[3]);
+      for (int i = 0; i < DN; ++i) {
+        o[i][0] *= c0;
+        o[i][1] *= c0;
+        o[i][2] *= c1;
+        o[i][3] *= c1;
+      }
+#pragma unroll
+      for (int k2 = 0; k2 < 4; ++k2) {
+        if (2 * k2 < n_lim) {
+          uint32_t pa[4];
+          pa[0] = pack_h2(sc[2 * k2][0], sc[2 * k2][1]);
+          pa[1] = pack_h2(sc[2 * k2][2], sc[2 * k2][3]);
+          pa[2] = pack_h2(sc[2 * k2 + 1][0], sc[2 * k2 + 1][1]);
+          pa[3] = pack_h2(sc[2 * k2 + 1][2], sc[2 * k2 + 1][3]);
+#pragma unroll
+          for (int dp = 0; dp < DN / 2; ++dp) {
+            const int mat = lane >> 3;
+            const int key = k2 * 16 + (lane & 7) + 8 * (mat & 1);
+            const int dim = dp * 16 + 8 * (mat >> 1);
+            uint32_t b[4];
+            ldsm_x4_t(b, vb + key * LDS + dim);
+            mma16816(o[2 * dp], pa, b[0], b[1]);
+            mma16816(o[2 * dp + 1], pa, b[2], b[3]);
+          }
+        }
       }
     }
     __syncthreads();

@@ -71,6 +71,68 @@ __device__ __forceinline__ void load32(uint32_t taddr, float* v) {
   for (int j = 0; j < 32; ++j) v[j] = u2f(r[j]);
 }
 
+// Two 32-column slices with one wait (both loads in flight together).
+__device__ __forceinline__ void load2x32(uint32_t ta, uint32_t tb, float* va, float* vb) {
+  uint32_t ra[32], rb[32];
+  tmem_ld_32x32b_x32(ta, ra);
+  tmem_ld_32x32b_x32(tb, rb);
+  tmem_ld_wait();
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    va[j] = u2f(ra[j]);
+    vb[j] = u2f(rb[j]);
+  }
+}
+
+__device__ __forceinline__ void load_f32x32(const float* src, float* v) {
+  const float4* p = reinterpret_cast<const float4*>(src);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const float4 x = __ldg(p + j);
+    v[4 * j] = x.x;
+    v[4 * j + 1] = x.y;
+    v[4 * j + 2] = x.z;
+    v[4 * j + 3] = x.w;
+  }
+}
+
+__device__ __forceinline__ void add_store_f32x32(float* dst, const float* v) {
+  float4* p = reinterpret_cast<float4*>(dst);
+  float4 x[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) x[j] = p[j];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    x[j].x += v[4 * j];
+    x[j].y += v[4 * j + 1];
+    x[j].z += v[4 * j + 2];
+    x[j].w += v[4 * j + 3];
+    p[j] = x[j];
+  }
+}
+
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+// Issued before the epilogue waits for its accumulator: pulls the bytes this
+// thread's row will read into L2 while the tile's MMAs still run.
+template <int BN, int EPI>
+__device__ __forceinline__ void epilogue_prefetch(const KArgs& a, int row, int n0) {
+  if (row >= a.M) return;
+  const GemmEpilogue& ep = a.ep;
+  if constexpr (EPI == EPI_RESID_F32) {
+    prefetch_l2(static_cast<const float*>(ep.out) + static_cast<int64_t>(row) * ep.ldo + n0, BN * 4);
+  } else if constexpr (EPI == EPI_ROPE_F16) {
+    if (n0 < ep.rope_cols) {
+      const int half = ep.head_dim >> 1;
+      const int64_t off = static_cast<int64_t>(ep.positions[row]) * half;
+      prefetch_l2(ep.rope_cos + off, half * 4);
+      prefetch_l2(ep.rope_sin + off, half * 4);
+    }
+  }
+}
+
 template <int BN, int EPI>
 __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int row, int n0) {
   const GemmEpilogue& ep = a.ep;
@@ -79,20 +141,12 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
   if constexpr (EPI == EPI_RESID_F32) {
     float* o = static_cast<float*>(ep.out) + static_cast<int64_t>(row) * ep.ldo + n0;
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      float v[32];
-      load32(trow + c, v);
+    for (int c = 0; c < BN; c += 64) {
+      float v0[32], v1[32];
+      load2x32(trow + c, trow + c + 32, v0, v1);
       if (live) {
-        float4* p = reinterpret_cast<float4*>(o + c);
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          float4 x = p[j];
-          x.x += v[4 * j];
-          x.y += v[4 * j + 1];
-          x.z += v[4 * j + 2];
-          x.w += v[4 * j + 3];
-          p[j] = x;
-        }
+        add_store_f32x32(o + c, v0);
+        add_store_f32x32(o + c + 32, v1);
       }
     }
   } else if constexpr (EPI == EPI_SWIGLU_F16) {
@@ -100,62 +154,84 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
 #pragma unroll 1
     for (int c = 0; c < BN / 2; c += 32) {
       float g[32], u[32];
-      load32(trow + c, g);
-      load32(trow + BN / 2 + c, u);
+      load2x32(trow + c, trow + BN / 2 + c, g, u);
 #pragma unroll
       for (int j = 0; j < 32; ++j) g[j] = g[j] / (1.0f + expf(-g[j])) * u[j];
       if (live) store_f16x32(o + c, g, bad);
     }
   } else {
     __half* o = static_cast<__half*>(ep.out) + static_cast<int64_t>(row) * ep.ldo + n0;
-    const int hd = ep.head_dim;
-    const int half = hd >> 1;
-    const int pos = (EPI == EPI_ROPE_F16 && live) ? ep.positions[row] : 0;
+    int rot_end = 0;  // columns [0, rot_end) of the tile hold rotated (q, k) heads
+    if constexpr (EPI == EPI_ROPE_F16) {
+      const int hd = ep.head_dim;
+      const int half = hd >> 1;
+      rot_end = ep.rope_cols - n0;
+      rot_end = rot_end < 0 ? 0 : (rot_end > BN ? BN : rot_end);
+      const int64_t toff = live ? static_cast<int64_t>(ep.positions[row]) * half : 0;
+      if (half >= 32) {
+        // cos/sin of this row's position, 32 frequencies at a time, reused by every head of the tile
 #pragma unroll 1
-    for (int c = 0; c < BN;) {
-      if (EPI == EPI_ROPE_F16 && n0 + c < ep.rope_cols) {
-        // one head [c, c + hd): rotate pairs (i, i + hd/2) by pos * inv_freq_i
-        const float* cs = ep.rope_cos + static_cast<int64_t>(pos) * half;
-        const float* sn = ep.rope_sin + static_cast<int64_t>(pos) * half;
-        if (half >= 32) {
+        for (int i0 = 0; i0 < half; i0 += 32) {
+          float cs[32], sn[32];
+          load_f32x32(ep.rope_cos + toff + i0, cs);
+          load_f32x32(ep.rope_sin + toff + i0, sn);
 #pragma unroll 1
-          for (int i0 = 0; i0 < half; i0 += 32) {
+          for (int h = 0; h < rot_end; h += hd) {
             float x1[32], x2[32];
-            load32(trow + c + i0, x1);
-            load32(trow + c + half + i0, x2);
+            load2x32(trow + h + i0, trow + h + half + i0, x1, x2);
             if (live) {
 #pragma unroll
               for (int j = 0; j < 32; ++j) {
-                const float cj = cs[i0 + j], sj = sn[i0 + j];
                 const float a1 = x1[j], a2 = x2[j];
-                x1[j] = a1 * cj - a2 * sj;
-                x2[j] = a2 * cj + a1 * sj;
+                x1[j] = a1 * cs[j] - a2 * sn[j];
+                x2[j] = a2 * cs[j] + a1 * sn[j];
               }
-              store_f16x32(o + c + i0, x1, bad);
-              store_f16x32(o + c + half + i0, x2, bad);
+              store_f16x32(o + h + i0, x1, bad);
+              store_f16x32(o + h + half + i0, x2, bad);
             }
           }
-        } else {  // head_dim 32: both halves in one slice
+        }
+      } else {  // head_dim 32: both halves of a head in one 32-column slice
+        float cs[16], sn[16];
+        const float4* c4 = reinterpret_cast<const float4*>(ep.rope_cos + toff);
+        const float4* s4 = reinterpret_cast<const float4*>(ep.rope_sin + toff);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float4 cv = __ldg(c4 + j), sv = __ldg(s4 + j);
+          cs[4 * j] = cv.x; cs[4 * j + 1] = cv.y; cs[4 * j + 2] = cv.z; cs[4 * j + 3] = cv.w;
+          sn[4 * j] = sv.x; sn[4 * j + 1] = sv.y; sn[4 * j + 2] = sv.z; sn[4 * j + 3] = sv.w;
+        }
+#pragma unroll 1
+        for (int h = 0; h < rot_end; h += 32) {
           float x[32];
-          load32(trow + c, x);
+          load32(trow + h, x);
           if (live) {
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
-              const float cj = cs[j], sj = sn[j];
               const float a1 = x[j], a2 = x[j + 16];
-              x[j] = a1 * cj - a2 * sj;
-              x[j + 16] = a2 * cj + a1 * sj;
+              x[j] = a1 * cs[j] - a2 * sn[j];
+              x[j + 16] = a2 * cs[j] + a1 * sn[j];
             }
-            store_f16x32(o + c, x, bad);
+            store_f16x32(o + h, x, bad);
           }
         }
-        c += hd;
-      } else {
-        float v[32];
-        load32(trow + c, v);
-        if (live) store_f16x32(o + c, v, bad);
-        c += 32;
       }
+    }
+    // plain fp16 columns (all of them for EPI_F16; the value heads for EPI_ROPE_F16)
+    int c = rot_end;
+#pragma unroll 1
+    for (; c + 64 <= BN; c += 64) {
+      float v0[32], v1[32];
+      load2x32(trow + c, trow + c + 32, v0, v1);
+      if (live) {
+        store_f16x32(o + c, v0, bad);
+        store_f16x32(o + c + 32, v1, bad);
+      }
+    }
+    if (c < BN) {
+      float v[32];
+      load32(trow + c, v);
+      if (live) store_f16x32(o + c, v, bad);
     }
   }
   if (bad) set_dev_error(ep.err, DEVERR_FP16_RANGE);
@@ -289,6 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
       const int m0 = (tile / num_n) * BM;
       const int n0 = (tile % num_n) * BN;
+      epilogue_prefetch<BN, EPI>(args, m0 + quarter * 32 + lane, n0);
       if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
       tc_fence_after();
       const uint32_t trow = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
