@@ -307,8 +307,9 @@ def ours(args):
                          "peak_source": f"{src} bf16_tflops_sustained (fp16 dense rate = bf16)",
                          "launches": gemm_launches},
             "cpu_baseline": cpu,
-            "e2e": {"value": world * w.n_rows / (e2e_per / 1000.0), "unit": "rows/s",
-                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_per},
+            "e2e": ({"value": world * w.n_rows / (e2e_per / 1000.0), "unit": "rows/s",
+                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_per}
+                    if e2e_ms else None),
             "gpu_launches": launches,
             "clocks": clk,
         }

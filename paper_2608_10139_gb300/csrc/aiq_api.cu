@@ -356,12 +356,12 @@ aiq_status ensure_rope(aiq_ctx* c, ModelD& m, int max_pos) {
 }
 
 struct PrefillBufs {
-  int32_t *tok, *pos, *seq_start, *last_idx, *tile_seq, *tile_q0, *n_tiles;
-  float* resid;
+  int32_t *tok, *pos, *seq_start, *last_idx, *tile_seq, *tile_q0, *n_tiles, *last_compact;
+  float *resid, *resid_last;
   __half *xn, *qkv, *att, *act;
 };
 
-aiq_status prefill_bufs(aiq_ctx* c, const ModelD& m, int64_t B, PrefillBufs* pb) {
+aiq_status prefill_bufs(aiq_ctx* c, const ModelD& m, int64_t B, int64_t max_rows, PrefillBufs* pb) {
   const aiq_model_config& g = m.cfg;
   const int64_t nqkv = static_cast<int64_t>(g.n_heads + 2 * g.n_kv_heads) * g.head_dim;
   AIQ_TRY(ws(c, "pf.tok", B, &pb->tok));
@@ -375,7 +375,9 @@ aiq_status prefill_bufs(aiq_ctx* c, const ModelD& m, int64_t B, PrefillBufs* pb)
   AIQ_TRY(ws(c, "pf.xn", B * g.d_model, &pb->xn));
   AIQ_TRY(ws(c, "pf.qkv", B * nqkv, &pb->qkv));
   AIQ_TRY(ws(c, "pf.att", B * g.n_heads * g.head_dim, &pb->att));
-  AIQ_TRY(ws(c, "pf.act", B * g.d_ffn, &pb->act));
+  AIQ_TRY(ws(c, "pf.act", std::max(B, max_rows) * g.d_ffn, &pb->act));
+  AIQ_TRY(ws(c, "pf.resid_last", max_rows * g.d_model, &pb->resid_last));
+  AIQ_TRY(ws(c, "pf.last_compact", max_rows, &pb->last_compact));
   return AIQ_OK;
 }
 
@@ -383,8 +385,11 @@ aiq_status prefill_bufs(aiq_ctx* c, const ModelD& m, int64_t B, PrefillBufs* pb)
 // pkv_in (optional): per-layer keys/values [L][P][2 Hkv hd] of the shared
 // prefix that every sequence attends; pkv_out (optional): where this pass
 // stores its own keys/values per layer (the prefix pass).
+// rows_only_last: the final layer's O-projection and MLP run only on each
+// sequence's last token (the only position whose output reaches the label
+// head); the result lands in b.resid_last, rows in sequence order.
 aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, int64_t n_seqs, const __half* pkv_in,
-                      int P_in, __half* pkv_out) {
+                      int P_in, __half* pkv_out, bool rows_only_last) {
   const aiq_model_config& g = m.cfg;
   const int d = g.d_model, hd = g.head_dim, Hq = g.n_heads, Hkv = g.n_kv_heads, f = g.d_ffn;
   const int nqkv = (Hq + 2 * Hkv) * hd;
@@ -424,24 +429,38 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
                        pkv_in ? pkv_in + l * P_in * ldkv : nullptr, P_in, b.att, c->d_err, c->stream);
       counted(c, n_tiles_max > 0);
     }
+    const bool prune = rows_only_last && l == g.n_layers - 1;
+    const __half* att = b.att;
+    float* resid = b.resid;
+    int Mo = M;
+    if (prune) {
+      // the attention output is dead after this gather, so its rows are packed into b.qkv
+      ProfScope p(c, "gather_last", 0, 0);
+      launch_gather_last(b.att, Hq * hd, b.resid, d, b.last_idx, n_seqs, b.qkv, b.resid_last, b.last_compact,
+                         c->stream);
+      counted(c, n_seqs > 0);
+      att = b.qkv;
+      resid = b.resid_last;
+      Mo = static_cast<int>(n_seqs);
+    }
     GemmEpilogue e2;
     e2.kind = EPI_RESID_F32;
-    e2.out = b.resid;
+    e2.out = resid;
     e2.ldo = d;
     e2.err = c->d_err;
-    AIQ_TRY(gemm(c, "gemm_o_resid", b.att, Hq * hd, L.wo, Hq * hd, M, d, Hq * hd, m.bn_o, e2));
+    AIQ_TRY(gemm(c, "gemm_o_resid", att, Hq * hd, L.wo, Hq * hd, Mo, d, Hq * hd, m.bn_o, e2));
     {
       ProfScope p(c, "rmsnorm", 0, 0);
-      launch_rmsnorm(b.resid, T, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
-      counted(c, T > 0);
+      launch_rmsnorm(resid, Mo, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+      counted(c, Mo > 0);
     }
     GemmEpilogue e3;
     e3.kind = EPI_SWIGLU_F16;
     e3.out = b.act;
     e3.ldo = f;
     e3.err = c->d_err;
-    AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, d, L.wgu, d, M, 2 * f, d, m.bn_gu, e3));
-    AIQ_TRY(gemm(c, "gemm_down_resid", b.act, f, L.wd, f, M, d, f, m.bn_d, e2));
+    AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, d, L.wgu, d, Mo, 2 * f, d, m.bn_gu, e3));
+    AIQ_TRY(gemm(c, "gemm_down_resid", b.act, f, L.wd, f, Mo, d, f, m.bn_d, e2));
   }
   return AIQ_OK;
 }
@@ -500,11 +519,14 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
   std::vector<int64_t> chunks(2 * (n_chunks + 1));
   CUDA_TRY(cudaMemcpyAsync(chunks.data(), chunk_d, chunks.size() * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream));
   AIQ_TRY(sync_and_check(c));
-  int64_t Bmax = P;
-  for (int64_t i = 0; i < n_chunks; ++i) Bmax = std::max(Bmax, chunks[2 * (i + 1) + 1] - chunks[2 * i + 1]);
+  int64_t Bmax = P, Rmax = 1;
+  for (int64_t i = 0; i < n_chunks; ++i) {
+    Bmax = std::max(Bmax, chunks[2 * (i + 1) + 1] - chunks[2 * i + 1]);
+    Rmax = std::max(Rmax, chunks[2 * (i + 1)] - chunks[2 * i]);
+  }
   AIQ_TRY(ensure_rope(c, m, static_cast<int>(P + max_len)));
   PrefillBufs pb;
-  AIQ_TRY(prefill_bufs(c, m, std::max<int64_t>(Bmax, 64), &pb));
+  AIQ_TRY(prefill_bufs(c, m, std::max<int64_t>(Bmax, 64), Rmax, &pb));
   const aiq_model_config& g = m.cfg;
   __half* pkv = nullptr;
   float* prefix_last;
@@ -514,7 +536,7 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
     AIQ_TRY(ws(c, "pf.prefix_kv", static_cast<int64_t>(g.n_layers) * P * 2 * g.n_kv_heads * g.head_dim, &pkv));
     launch_pack_prefix(prefix_d, P, pb.tok, pb.pos, pb.seq_start, c->stream);
     counted(c, 1);
-    AIQ_TRY(run_layers(c, m, pb, P, 1, nullptr, 0, pkv));
+    AIQ_TRY(run_layers(c, m, pb, P, 1, nullptr, 0, pkv, false));
     CUDA_TRY(cudaMemcpyAsync(prefix_last, pb.resid + static_cast<int64_t>(P - 1) * g.d_model, g.d_model * sizeof(float),
                              cudaMemcpyDeviceToDevice, c->stream));
   }
@@ -528,11 +550,11 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
                         pb.seq_start, pb.last_idx, c->stream);
       counted(c, 1);
     }
-    AIQ_TRY(run_layers(c, m, pb, Tc, r1 - r0, pkv, static_cast<int>(P), nullptr));
+    AIQ_TRY(run_layers(c, m, pb, Tc, r1 - r0, pkv, static_cast<int>(P), nullptr, true));
     {
       ProfScope p(c, "label_head", 0, 0);
-      launch_label_head(pb.resid, pb.last_idx, prefix_last, r1 - r0, g.d_model, m.final_norm, g.rms_eps, m.lm_head,
-                        m.lm_bias, labels_d, K, logits + r0 * K, c->stream);
+      launch_label_head(pb.resid_last, pb.last_compact, prefix_last, r1 - r0, g.d_model, m.final_norm, g.rms_eps,
+                        m.lm_head, m.lm_bias, labels_d, K, logits + r0 * K, c->stream);
       counted(c, 1);
     }
   }
@@ -754,7 +776,13 @@ aiq_status run_query(aiq_ctx* c, const TableD* build, int32_t build_key, const a
   if (!rel_only && m) {
     const aiq_model_config& g = m->cfg;
     const double pre = st.S > 0 ? static_cast<double>(st.P) : 0.0;
-    R.v.prefill_flops = m->linear_flops_per_token * (static_cast<double>(st.T) + pre) +
+    // final layer: Q/K/V for every token, O-projection and MLP for each row's last token only
+    const double d = g.d_model, qd = double(g.n_heads) * g.head_dim, kd = double(g.n_kv_heads) * g.head_dim;
+    const double per_layer = m->linear_flops_per_token / g.n_layers;
+    const double tail = 2.0 * (qd * d + 3.0 * d * g.d_ffn);
+    R.v.prefill_flops = per_layer * (g.n_layers - 1) * (static_cast<double>(st.T) + pre) +
+                        2.0 * d * (qd + 2 * kd) * static_cast<double>(st.T) + tail * static_cast<double>(st.S) +
+                        per_layer * pre +
                         4.0 * g.n_heads * g.head_dim * g.n_layers * (static_cast<double>(st.pairs) + pre * (pre + 1) / 2) +
                         2.0 * g.d_model * K * static_cast<double>(st.S);
   }

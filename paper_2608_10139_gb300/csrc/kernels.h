@@ -107,6 +107,10 @@ void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float e
 void launch_attention(const __half* qkv, int64_t T, const int32_t* seq_start, const int32_t* tile_seq,
                       const int32_t* tile_q0, int n_tiles_max, const int32_t* n_tiles_dev, int Hq, int Hkv,
                       int hd, const __half* prefix_kv, int P, __half* out, int* err, cudaStream_t s);
+// Gathers each row's last-token attention output and residual into dense [n, .]
+// buffers for the final layer's row-only O-projection and MLP.
+void launch_gather_last(const __half* att, int ld_att, const float* resid, int d, const int32_t* last_idx, int64_t n,
+                        __half* att_out, float* resid_out, int32_t* last_compact, cudaStream_t s);
 // last_idx[r] < 0 reads prefix_last (fp32 [d]) instead of a row of resid.
 void launch_label_head(const float* resid, const int32_t* last_idx, const float* prefix_last, int64_t n_rows, int d,
                        const uint16_t* g, float eps, const uint16_t* lm_head, const uint16_t* lm_bias,

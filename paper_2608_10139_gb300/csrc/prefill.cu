@@ -144,6 +144,25 @@ __global__ void k_label_head(const float* resid, const int32_t* last_idx, const 
   }
 }
 
+// Final layer, rows only: gather each row's last token (attention output and
+// residual) into dense [n, .] buffers; last_compact[r] = r, or -1 for a row
+// without tokens of its own (its logits come from the prefix's last state).
+__global__ void k_gather_last(const __half* att, int ld_att, const float* resid, int d, const int32_t* last_idx,
+                              int64_t n, __half* att_out, float* resid_out, int32_t* last_compact) {
+  const int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (r >= n) return;
+  const int32_t li = last_idx[r];
+  if (lane == 0) last_compact[r] = li >= 0 ? static_cast<int32_t>(r) : -1;
+  const int64_t src = li >= 0 ? li : 0;
+  const uint4* a = reinterpret_cast<const uint4*>(att + src * ld_att);
+  uint4* ao = reinterpret_cast<uint4*>(att_out + r * ld_att);
+  for (int c = lane; c < ld_att / 8; c += 32) ao[c] = a[c];
+  const float4* x = reinterpret_cast<const float4*>(resid + src * d);
+  float4* xo = reinterpret_cast<float4*>(resid_out + r * d);
+  for (int c = lane; c < d / 4; c += 32) xo[c] = x[c];
+}
+
 inline unsigned grid_for(int64_t threads) { return static_cast<unsigned>((threads + 255) / 256); }
 
 }  // namespace
@@ -183,6 +202,12 @@ void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float e
     case 4096: k_rmsnorm<32><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, err); break;
     default: k_rmsnorm_any<<<grid, 256, 0, s>>>(x, T, d, g, eps, out, err); break;
   }
+}
+
+void launch_gather_last(const __half* att, int ld_att, const float* resid, int d, const int32_t* last_idx, int64_t n,
+                        __half* att_out, float* resid_out, int32_t* last_compact, cudaStream_t s) {
+  if (n <= 0) return;
+  k_gather_last<<<grid_for(n * 32), 256, 0, s>>>(att, ld_att, resid, d, last_idx, n, att_out, resid_out, last_compact);
 }
 
 void launch_label_head(const float* resid, const int32_t* last_idx, const float* prefix_last, int64_t n_rows, int d,
