@@ -183,7 +183,9 @@ aiq_status aiq_result_free(aiq_ctx* ctx, aiq_result_h result);
 const char* aiq_last_error(void);
 
 /* Options: "token_budget" (max packed tokens per prefill chunk, default
- * 131072), "profile" (0/1: time every GEMM launch with CUDA events). */
+ * 131072), "profile" (0/1: time every GEMM launch with CUDA events),
+ * "gemm_pair" (0/1, default 1: 256 x 256 GEMM tiles on CTA pairs where
+ * N % 256 == 0 and M >= 512; also selects them for aiq_op_gemm with bn = 256). */
 aiq_status aiq_set_option(aiq_ctx* ctx, const char* name, int64_t value);
 
 /* The context's CUDA stream (a cudaStream_t), for callers that time the

@@ -126,6 +126,7 @@ struct aiq_ctx {
   std::map<std::string, DevBuf> ws;
   int64_t token_budget = 131072;
   bool profile = false;
+  bool gemm_pair = true;  // CTA-pair (cta_group::2) GEMM tiles where the shape allows
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
   std::map<std::string, StatAcc> stats;
@@ -259,7 +260,8 @@ aiq_status gemm(aiq_ctx* c, const char* name, const __half* A, int64_t lda, cons
                 int K, int bn, const GemmEpilogue& ep) {
   const double out_bytes = (ep.kind == EPI_RESID_F32 ? 8.0 : (ep.kind == EPI_SWIGLU_F16 ? 1.0 : 2.0)) * M * N;
   ProfScope ps(c, name, 2.0 * M * N * K, 2.0 * (double(M) * K + double(N) * K) + out_bytes);
-  int e = gemm_f16_tcgen05(A, lda, B, ldb, M, N, K, bn, ep, c->num_sms, c->stream);
+  const bool pair = c->gemm_pair && bn == 256 && M >= 512;
+  int e = gemm_f16_tcgen05(A, lda, B, ldb, M, N, K, bn, pair, ep, c->num_sms, c->stream);
   if (M > 0) counted(c, 1);
   if (e != 0)
     return fail(AIQ_ERR_CUDA, std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(static_cast<cudaError_t>(e)));
@@ -1136,6 +1138,10 @@ aiq_status aiq_set_option(aiq_ctx* c, const char* name, int64_t value) {
   }
   if (!std::strcmp(name, "profile")) {
     c->profile = value != 0;
+    return AIQ_OK;
+  }
+  if (!std::strcmp(name, "gemm_pair")) {
+    c->gemm_pair = value != 0;
     return AIQ_OK;
   }
   return fail(AIQ_ERR_INVALID_ARG, std::string("unknown option ") + name);

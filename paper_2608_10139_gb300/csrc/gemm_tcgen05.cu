@@ -385,6 +385,178 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+
+// ------------------------------------------------------------ CTA pairs ---
+// 256 x 256 output tiles on a cluster of two CTAs (tcgen05.mma.cta_group::2).
+// Each CTA stages its own 128 rows of A and 128 columns of B per k-block
+// (32 KB, 6 stages), so every SM moves half the B bytes of the single-CTA
+// 128 x 256 tile for the same MMA work; its TMA completes on the leader's
+// barrier, the leader alone issues the M = 256 MMA, and each CTA's epilogue
+// drains its own 128 accumulator rows and reports back to the leader.
+struct CfgPair {
+  static constexpr int STAGES = 6;
+  static constexpr int A_BYTES = 128 * BK * 2;
+  static constexpr int B_BYTES = 128 * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 512;
+  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + 256;
+};
+
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_gemm_tcgen05_pair(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
+                        KArgs args) {
+  using C = CfgPair;
+  constexpr int BN = 256;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* full = bars;                 // used in the leader only
+  uint64_t* empty = bars + C::STAGES;    // per CTA, multicast by the leader's commits
+  uint64_t* tfull = bars + 2 * C::STAGES;
+  uint64_t* tempty = tfull + 2;          // used in the leader only: 4 warps x 2 CTAs
+  uint64_t* mma_done = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int pair = blockIdx.x >> 1;
+  const int n_pairs = gridDim.x >> 1;
+  int* err = args.ep.err;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], 8);
+    }
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tma_a);
+    tma_prefetch_desc(&tma_b);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish_pair();
+    tc_fence_before();
+  }
+  __syncthreads();
+  cluster_sync();  // barriers of both CTAs initialised before any remote arrival
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int num_n = args.N / BN;
+  const int num_m = (args.M + 2 * BM - 1) / (2 * BM);
+  const int num_tiles = num_m * num_n;
+  const int kblocks = args.K / BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------- TMA producer
+      const uint32_t full_leader = map_to_cta(smem_u32(full), 0);
+      uint32_t issued = 0;
+      bool ok = true;
+      for (int tile = pair; tile < num_tiles && ok; tile += n_pairs) {
+        const int m0 = (tile / num_n) * 2 * BM;
+        const int n0 = (tile % num_n) * BN;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          const int s = issued % C::STAGES;
+          const uint32_t ph = (issued / C::STAGES) & 1;
+          if (!mbar_wait_bounded(&empty[s], ph ^ 1, abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          if (leader) mbar_arrive_expect_tx(&full[s], 2 * C::STAGE_BYTES);
+          tma_load_2d_pair(sA + s * C::A_BYTES, &tma_a, full_leader + s * 8, kb * BK, m0 + rank * BM);
+          tma_load_2d_pair(sB + s * C::B_BYTES, &tma_b, full_leader + s * 8, kb * BK, n0 + rank * 128);
+          ++issued;
+        }
+      }
+      if (!ok && leader) {
+        // the leader's barrier completes only once both CTAs' bytes have landed
+        const uint32_t first = issued > (uint32_t)C::STAGES ? issued - C::STAGES : 0;
+        volatile int never = 0;
+        for (uint32_t i = first; i < issued; ++i)
+          mbar_wait_bounded(&full[i % C::STAGES], (i / C::STAGES) & 1, &never, nullptr, 200000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      // ------------------------------------------------ MMA issuer (leader)
+      constexpr uint32_t idesc = idesc_f16_f32(2 * BM, BN);
+      uint32_t consumed = 0;
+      int acc = 0;
+      uint32_t acc_ph = 0;
+      bool ok = true;
+      for (int tile = pair; tile < num_tiles && ok; tile += n_pairs) {
+        if (!mbar_wait_bounded(&tempty[acc], acc_ph ^ 1, abort_flag, err)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          const int s = consumed % C::STAGES;
+          const uint32_t ph = (consumed / C::STAGES) & 1;
+          if (!mbar_wait_bounded(&full[s], ph, abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
+          const uint32_t b0 = smem_u32(sB + s * C::B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / UMMA_K; ++k)
+            umma_f16_ss_pair(d_tmem, smem_desc_k_sw128(a0 + k * UMMA_K * 2), smem_desc_k_sw128(b0 + k * UMMA_K * 2),
+                             idesc, (kb | k) != 0);
+          umma_commit_pair_mc(&empty[s], 0x3);
+          ++consumed;
+        }
+        if (!ok) break;
+        umma_commit_pair_mc(&tfull[acc], 0x3);
+        acc ^= 1;
+        if (acc == 0) acc_ph ^= 1;
+      }
+      umma_commit_pair_mc(mma_done, 0x1);
+      volatile int never = 0;
+      mbar_wait_bounded(mma_done, 0, &never, err);
+    }
+  } else {
+    // ------------------------------------------------ epilogue (both CTAs)
+    const int quarter = warp & 3;
+    const uint32_t tempty_leader = map_to_cta(smem_u32(tempty), 0);
+    int acc = 0;
+    uint32_t acc_ph = 0;
+    for (int tile = pair; tile < num_tiles; tile += n_pairs) {
+      const int m0 = (tile / num_n) * 2 * BM + rank * BM;
+      const int n0 = (tile % num_n) * BN;
+      epilogue_prefetch<BN, EPI>(args, m0 + quarter * 32 + lane, n0);
+      if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
+      tc_fence_after();
+      const uint32_t trow = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
+      epilogue_tile<BN, EPI>(args, trow, m0 + quarter * 32 + lane, n0);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(tempty_leader + acc * 8);
+      acc ^= 1;
+      if (acc == 0) acc_ph ^= 1;
+    }
+  }
+
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while its peer may still signal it
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, C::TMEM_COLS);
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   if (!fn) {
@@ -422,6 +594,40 @@ int launch(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, int num
   return cudaGetLastError();
 }
 
+template <int EPI>
+int launch_pair(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, int num_sms, cudaStream_t stream) {
+  using C = CfgPair;
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tcgen05_pair<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  const int tiles = ((a.M + 2 * BM - 1) / (2 * BM)) * (a.N / 256);
+  const int pairs = tiles < num_sms / 2 ? tiles : num_sms / 2;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * pairs, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, k_gemm_tcgen05_pair<EPI>, ma, mb, a);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+int dispatch_pair(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, int num_sms, cudaStream_t s) {
+  switch (a.ep.kind) {
+    case EPI_F16: return launch_pair<EPI_F16>(ma, mb, a, num_sms, s);
+    case EPI_ROPE_F16: return launch_pair<EPI_ROPE_F16>(ma, mb, a, num_sms, s);
+    case EPI_RESID_F32: return launch_pair<EPI_RESID_F32>(ma, mb, a, num_sms, s);
+    case EPI_SWIGLU_F16: return launch_pair<EPI_SWIGLU_F16>(ma, mb, a, num_sms, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
 template <int BN>
 int dispatch_epi(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, int num_sms, cudaStream_t s) {
   switch (a.ep.kind) {
@@ -436,9 +642,10 @@ int dispatch_epi(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, i
 }  // namespace
 
 int gemm_f16_tcgen05(const __half* A, int64_t lda, const __half* B, int64_t ldb, int M, int N, int K, int bn,
-                     const GemmEpilogue& ep, int num_sms, cudaStream_t stream) {
+                     bool pair, const GemmEpilogue& ep, int num_sms, cudaStream_t stream) {
   if (M == 0) return 0;
   if (M < 0 || N <= 0 || K <= 0 || K % BK != 0 || (bn != 128 && bn != 256) || N % bn != 0) return cudaErrorInvalidValue;
+  if (pair && bn != 256) return cudaErrorInvalidValue;
   if ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B)) & 15) return cudaErrorMisalignedAddress;
   if ((lda * 2) % 16 != 0 || (ldb * 2) % 16 != 0) return cudaErrorInvalidValue;
   if (ep.kind == EPI_ROPE_F16) {
@@ -446,8 +653,9 @@ int gemm_f16_tcgen05(const __half* A, int64_t lda, const __half* B, int64_t ldb,
     if (!(hd == 32 || hd == 64 || hd == 128) || bn % hd != 0 || !ep.positions || !ep.rope_cos) return cudaErrorInvalidValue;
   }
   CUtensorMap ma, mb;
-  if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, B, N, K, ldb, bn)) return cudaErrorInvalidValue;
+  if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, B, N, K, ldb, pair ? 128 : bn)) return cudaErrorInvalidValue;
   KArgs a{M, N, K, ep};
+  if (pair) return dispatch_pair(ma, mb, a, num_sms, stream);
   return bn == 256 ? dispatch_epi<256>(ma, mb, a, num_sms, stream) : dispatch_epi<128>(ma, mb, a, num_sms, stream);
 }
 

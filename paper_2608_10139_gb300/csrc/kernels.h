@@ -30,9 +30,10 @@ struct GemmEpilogue {
 
 // C = A[M,K] * B[N,K]^T with fp16 operands and fp32 accumulation on tcgen05.
 // Requires K % 64 == 0, N % bn == 0, bn in {128, 256}, 16-byte aligned rows.
+// pair: 256 x 256 tiles on clusters of two CTAs (cta_group::2); needs bn == 256.
 // Returns 0 or a cudaError_t value.
 int gemm_f16_tcgen05(const __half* A, int64_t lda, const __half* B, int64_t ldb, int M, int N, int K, int bn,
-                     const GemmEpilogue& ep, int num_sms, cudaStream_t stream);
+                     bool pair, const GemmEpilogue& ep, int num_sms, cudaStream_t stream);
 
 // ------------------------------------------------------------ relational ---
 struct PredDev {

@@ -182,3 +182,59 @@ def test_attention_with_shared_prefix(ctx, hd, Hq, Hkv, P):
         v = seq[:, (Hq + Hkv) * hd:].reshape(m, Hkv, hd)
         ref = tf.causal_attention(q, k, v).reshape(m, Hq * hd)[P:]
         _close(got[starts[i]:starts[i] + n], ref, 4e-3, 4e-3, f"prefix attention P{P} seq {i} len {n}")
+
+
+@pytest.mark.parametrize("pair", [0, 1])
+@pytest.mark.parametrize("M,N,K,epi", [(512, 256, 128, 0), (1000, 512, 2048, 0), (4099, 1536, 512, 2),
+                                       (3000, 2048, 256, 3), (70000, 1024, 256, 0)])
+def test_gemm_cta_pair_vs_single(ctx, pair, M, N, K, epi):
+    """256 x 256 tiles on CTA pairs (tcgen05 cta_group::2) and 128 x 256 tiles on
+    single CTAs give the oracle's product, ragged M included."""
+    rng = np.random.default_rng(M + N + K + epi)
+    A = rng.standard_normal((M, K)).astype(np.float16)
+    B = (rng.standard_normal((N, K)) * 0.05).astype(np.float16)
+    dA, dB = _h(A), _h(B)
+    a, b = A.astype(np.float64), B.astype(np.float64)
+    ctx.set_option("gemm_pair", pair)
+    try:
+        if epi == 0:
+            out = torch.zeros((M, N), dtype=torch.float16, device="cuda")
+            ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, 256, 0, out.data_ptr(), N)
+            _close(_np64(out), a @ b.T, 2e-3, 2e-3 * np.sqrt(K) * 0.05, f"pair{pair} f16 M{M}")
+        elif epi == 2:
+            R = rng.standard_normal((M, N)).astype(np.float32)
+            dR = _h(R)
+            ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, 256, 2, dR.data_ptr(), N)
+            _close(_np64(dR), R.astype(np.float64) + a @ b.T, 1e-5, 2e-6 * np.sqrt(K), f"pair{pair} resid M{M}")
+        else:
+            f = N // 2
+            g, u = b[:f], b[f:]
+            inter = np.concatenate([np.concatenate([B[i:i + 128], B[f + i:f + i + 128]]) for i in range(0, f, 128)])
+            dI = _h(inter)
+            out = torch.zeros((M, f), dtype=torch.float16, device="cuda")
+            ctx.op_gemm(dA.data_ptr(), K, dI.data_ptr(), K, M, N, K, 256, 3, out.data_ptr(), f)
+            ref = tf.silu(a @ g.T) * (a @ u.T)
+            _close(_np64(out), ref, 3e-3, 3e-3 * K * 0.0025, f"pair{pair} swiglu M{M}")
+    finally:
+        ctx.set_option("gemm_pair", 1)
+
+
+def test_gemm_cta_pair_rope(ctx):
+    rng = np.random.default_rng(99)
+    hd, Hq, Hkv, M, K = 64, 32, 8, 1300, 512
+    N = (Hq + 2 * Hkv) * hd
+    A = rng.standard_normal((M, K)).astype(np.float16)
+    B = (rng.standard_normal((N, K)) * 0.05).astype(np.float16)
+    pos = rng.integers(0, 1100, M).astype(np.int32)
+    cs = torch.zeros((1200, hd // 2), dtype=torch.float32, device="cuda")
+    sn = torch.zeros_like(cs)
+    ctx.op_rope_table(cs.data_ptr(), sn.data_ptr(), 1200, hd, 1.0e4)
+    dA, dB, dP = _h(A), _h(B), _h(pos)
+    out = torch.zeros((M, N), dtype=torch.float16, device="cuda")
+    rope_cols = (Hq + Hkv) * hd
+    ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, 256, 1, out.data_ptr(), N, dP.data_ptr(),
+                cs.data_ptr(), sn.data_ptr(), rope_cols, hd)
+    y = A.astype(np.float64) @ B.astype(np.float64).T
+    qk = y[:, :rope_cols].reshape(M, Hq + Hkv, hd)
+    ref = np.concatenate([tf.rope(qk, pos, 1.0e4).reshape(M, rope_cols), y[:, rope_cols:]], axis=1)
+    _close(_np64(out), ref, 2e-3, 2e-3 * np.sqrt(K) * 0.05, "pair rope")
