@@ -51,14 +51,31 @@ def parse():
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-sample-rows", type=int, default=12)
+    p.add_argument("--micro", default="", choices=["", "relational"],
+                   help="relational: predicate + compaction alone on a 2^28-row table, against HBM bandwidth")
+    p.add_argument("--micro-rows", type=int, default=1 << 28)
+    p.add_argument("--sweep", default="", help="selectivity sweep: 'fixed', 'lognormal' or 'both'")
     return p.parse_args()
 
 
 def workload(args):
     w = synth.WORKLOADS[args.workload]
     if args.rows:
-        w = synth.scaled(w, args.rows)
+        w = synth.scaled(w, args.rows, join_build_rows=(max(1, args.rows // 10) if w.join_build_rows else None))
     return w
+
+
+def make_step(ctx, w, q, model, aiq):
+    """One whole query on the resident tables: the select form, or the
+    reviews-movies join form with GROUP BY movie."""
+    preds = [(p.column, p.op, p.value) for p in w.preds]
+    table = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+    if not w.join_build_rows:
+        return (lambda: ctx.run_select(table, model, preds, q.prefix, w.label_ids, agg=w.agg)), [table]
+    build = ctx.load_table(q.build.cols, n_rows=q.build.n_rows)
+    bpreds = [(p.column, p.op, p.value) for p in w.join_build_preds]
+    return (lambda: ctx.run_join_select(build, "movie_id", bpreds, table, "movie_id", model, preds, q.prefix,
+                                        w.label_ids, agg=w.agg)), [table, build]
 
 
 def peaks():
@@ -204,16 +221,13 @@ def ours(args):
     preds = [(p.column, p.op, p.value) for p in w.preds]
     ctx = aiq.Context(local)
     model = ctx.load_model(w.model, tensors)
-    table = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+    step, tables = make_step(ctx, w, q, model, aiq)
     stream = torch.cuda.ExternalStream(ctx.stream())
     flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
 
     def barrier():
         if world > 1:
             torch.distributed.barrier()
-
-    def step():
-        return ctx.run_select(table, model, preds, q.prefix, w.label_ids, agg=w.agg)
 
     for _ in range(args.warmup):
         step()
@@ -259,18 +273,21 @@ def ours(args):
     traffic = GEMM_TRAFFIC["bytes_per_launch"] if GEMM_TRAFFIC["source_sha"] == gemm_source_sha() else None
     step_ms = {k: round(v["total_ms"] / args.steps, 3) for k, v in sorted(stats.items())}
 
-    # end to end through the C-ABI with host buffers: upload table, query, download results
-    e2e_ms, h2d, d2h = [], q.table.nbytes(), 0
+    # end to end through the C-ABI with host buffers: upload table(s), query, download results
+    e2e_ms, h2d, d2h = [], q.table.nbytes() + (q.build.nbytes() if q.build else 0), 0
+    for t in tables:
+        ctx.free_table(t)
     for _ in range(args.e2e_steps):
         barrier()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
-        t_e = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
-        r = ctx.run_select(t_e, model, preds, q.prefix, w.label_ids, agg=w.agg)
-        ctx.free_table(t_e)
+        step_e, tabs = make_step(ctx, w, q, model, aiq)
+        r = step_e()
+        for t in tabs:
+            ctx.free_table(t)
         torch.cuda.synchronize()
         e2e_ms.append(1000 * (time.perf_counter() - t0))
-        d2h = 4 * len(r.row_ids) + 8 * len(r.label_counts) + 8
+        d2h = (4 * len(r.row_ids) + 8 * len(r.label_counts) + 8 + 20 * len(r.group_keys))
     e2e_per = statistics.median(e2e_ms) if e2e_ms else float("nan")
     if world > 1:
         t = torch.tensor([e2e_per], device="cuda")
@@ -278,7 +295,7 @@ def ours(args):
         e2e_per = float(t.item())
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not w.join_build_rows:
         s, n, c = cpu_oracle_sample(w, q, W, args.cpu_sample_rows)
         cpu = {"value": n / s, "unit": "rows/s", "cores": os.cpu_count(), "kind": "oracle",
                "sample": f"first {n} input rows ({c} LM candidates), relational + fp64 transformer, numpy"}
@@ -290,14 +307,16 @@ def ours(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f16xf16->f32 (bf16 model values)", "data": "synthetic",
             "config": {"workload": w.name, "rows": w.n_rows, "candidates": res.n_candidates,
-                       "tokens": res.n_tokens, "chunks": res.n_chunks,
-                       "model": "1B-shape decoder d2048 L16 32/8 heads hd64 ffn8192 V32000, random init",
+                       "tokens": res.n_tokens, "prefill_tokens": res.n_prefill_tokens, "chunks": res.n_chunks,
+                       "model": (f"decoder d{w.model.d_model} L{w.model.n_layers} {w.model.n_heads}/"
+                                 f"{w.model.n_kv_heads} heads hd{w.model.head_dim} ffn{w.model.d_ffn} "
+                                 f"V{w.model.vocab}, random init"),
                        "l2": "2x L2 written between timed steps; weights and activations exceed L2",
                        "parallelism": f"replicas x{world}"},
             "p50_latency_ms": statistics.median(ms),
             "wall_ms_per_step": 1000 * wall / args.steps,
             "prefill_tflops": res.prefill_flops / (res.ms_prefill / 1000.0) / 1e12 if res.ms_prefill else None,
-            "prefill_tokens_per_s": res.n_tokens / (res.ms_prefill / 1000.0) if res.ms_prefill else None,
+            "prompt_tokens_per_s": res.n_tokens / (res.ms_prefill / 1000.0) if res.ms_prefill else None,
             "phase_ms": {"relational": res.ms_relational, "prefill": res.ms_prefill,
                          "aggregate": res.ms_aggregate},
             "kernel_ms_per_step": step_ms,
@@ -319,10 +338,96 @@ def ours(args):
         torch.distributed.destroy_process_group()
 
 
+def micro_relational(args):
+    """Predicate (rating >= 4 AND year >= 2000) + order-preserving compaction
+    over a 2^28-row table of two int32 columns, timed per kernel with events."""
+    import torch
+    from paper_2608_10139_gb300 import aiq
+    from paper_2608_10139_gb300 import build as _build
+    _build.build()
+    n = args.micro_rows
+    rng = np.random.Generator(np.random.PCG64(7))
+    cols = {"rating": rng.integers(1, 6, n, dtype=np.int32), "year": rng.integers(1950, 2025, n, dtype=np.int32)}
+    preds = [("rating", aiq.GE, 4), ("year", aiq.GE, 2000)]
+    ctx = aiq.Context(0)
+    t = ctx.load_table(cols, n_rows=n)
+    for _ in range(args.warmup):
+        ctx.run_select(t, 0, preds, [], [0, 1], flags=aiq.FLAG_RELATIONAL_ONLY)
+    ctx.reset_kernel_stats()
+    ctx.set_option("profile", 1)
+    clocks = ClockSampler(0)
+    clocks.start()
+    totals = []
+    for _ in range(args.steps):
+        r = ctx.run_select(t, 0, preds, [], [0, 1], flags=aiq.FLAG_RELATIONAL_ONLY)
+        totals.append(r.ms_relational)
+    clk = clocks.stop()
+    st = ctx.kernel_stats()
+    S = r.n_candidates
+    pk, src = peaks()
+    mask_ms = st["predicate_mask"]["total_ms"] / args.steps
+    comp_ms = st["compact"]["total_ms"] / args.steps
+    mask_bytes = 8.0 * n + n / 8          # two int32 columns read, 1 bit/row written
+    comp_bytes = n / 8 + 4.0 * S          # bitmask read, survivor ids written
+    line = {"metric": "relational predicate + compaction HBM throughput", "rows": n, "survivors": S,
+            "steps": args.steps, "warmup": args.warmup,
+            "predicate_mask": {"ms": mask_ms, "GB/s": mask_bytes / mask_ms / 1e6,
+                               "frac": mask_bytes / mask_ms / 1e6 / pk["hbm_gbs"]},
+            "compact": {"ms": comp_ms, "GB/s": comp_bytes / comp_ms / 1e6,
+                        "frac": comp_bytes / comp_ms / 1e6 / pk["hbm_gbs"]},
+            "combined": {"ms": mask_ms + comp_ms, "GB/s": (mask_bytes + comp_bytes) / (mask_ms + comp_ms) / 1e6,
+                         "frac": (mask_bytes + comp_bytes) / (mask_ms + comp_ms) / 1e6 / pk["hbm_gbs"]},
+            "query_relational_ms_p50": statistics.median(totals),
+            "peak": {"hbm_gbs": pk["hbm_gbs"], "source": src}, "clocks": clk}
+    print(json.dumps(line), flush=True)
+    ctx.close()
+
+
+def sweep(args):
+    """Selectivity sweep on the 1M-row table: rows/s, p50 latency and the
+    relational / prefill time split at each point (one JSON line per point)."""
+    import torch
+    from paper_2608_10139_gb300 import aiq
+    from paper_2608_10139_gb300 import build as _build
+    _build.build()
+    kinds = ["fixed", "lognormal"] if args.sweep == "both" else [args.sweep]
+    base = synth.sweep_workload("1%", kinds[0])
+    W = synth.make_weights(base.model, base.weight_seed)
+    ctx = aiq.Context(0)
+    model = ctx.load_model(base.model, [W[n] for n, _, _ in synth.weight_specs(base.model)])
+    for kind in kinds:
+        q = synth.make_inputs(synth.sweep_workload("1%", kind))   # one table per text kind
+        table = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+        for point in synth.SWEEP_POINTS:
+            w = synth.sweep_workload(point, kind)
+            preds = [(p.column, p.op, p.value) for p in w.preds]
+            runs = args.steps if point in ("1%", "5%", "25%") else max(1, min(args.steps, 3))
+            ctx.run_select(table, model, preds, q.prefix, w.label_ids, agg=w.agg)   # warm-up
+            res = [ctx.run_select(table, model, preds, q.prefix, w.label_ids, agg=w.agg) for _ in range(runs)]
+            tot = [r.ms_total for r in res]
+            r = res[-1]
+            line = {"metric": "AI-query input rows/s", "workload": w.name, "point": point, "text": kind,
+                    "rows": w.n_rows, "candidates": r.n_candidates, "prefill_tokens": r.n_prefill_tokens,
+                    "runs": runs, "p50_latency_ms": statistics.median(tot),
+                    "rows_per_s": w.n_rows / (statistics.median(tot) / 1000.0),
+                    "relational_ms": statistics.median([x.ms_relational for x in res]),
+                    "prefill_ms": statistics.median([x.ms_prefill for x in res]),
+                    "aggregate_ms": statistics.median([x.ms_aggregate for x in res]),
+                    "prefill_tflops": r.prefill_flops / (r.ms_prefill / 1000.0) / 1e12 if r.ms_prefill else None,
+                    "count": r.count}
+            print(json.dumps(line), flush=True)
+        ctx.free_table(table)
+    ctx.close()
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         reference_arm(args)
+    elif args.micro == "relational":
+        micro_relational(args)
+    elif args.sweep:
+        sweep(args)
     else:
         ours(args)
 

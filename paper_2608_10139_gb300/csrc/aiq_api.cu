@@ -111,6 +111,25 @@ struct StatAcc {
 
 void aiq::set_error_message(const char* msg) { g_err = msg ? msg : ""; }
 
+namespace {
+thread_local cudaError_t g_launch_err = cudaSuccess;
+thread_local std::string g_launch_what;
+}  // namespace
+
+void aiq::set_launch_error(const char* what, cudaError_t e) {
+  if (g_launch_err == cudaSuccess) {
+    g_launch_err = e;
+    g_launch_what = what ? what : "";
+  }
+}
+
+cudaError_t aiq::take_launch_error(const char** what) {
+  const cudaError_t e = g_launch_err;
+  g_launch_err = cudaSuccess;
+  if (what) *what = g_launch_what.c_str();
+  return e;
+}
+
 struct aiq_ctx {
   int device = 0;
   int num_sms = 0;
@@ -182,6 +201,12 @@ aiq_status ws(aiq_ctx* c, const char* name, size_t count, T** out) {
 }
 
 aiq_status sync_and_check(aiq_ctx* c) {
+  const char* what = nullptr;
+  const cudaError_t le = take_launch_error(&what);
+  if (le != cudaSuccess) {
+    cudaGetLastError();
+    return fail(AIQ_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(le));
+  }
   CUDA_TRY(cudaGetLastError());
   CUDA_TRY(cudaStreamSynchronize(c->stream));
   int err = 0;
@@ -306,6 +331,8 @@ aiq_status filter_compact(aiq_ctx* c, const TableD& t, const PredSet& ps, const 
   AIQ_TRY(ws(c, (b + ".bits").c_str(), std::max<int64_t>(nb, 1) * (kRowsPerBlock / 32), &bits));
   AIQ_TRY(ws(c, (b + ".bcnt").c_str(), std::max<int64_t>(nb, 1), &bcnt));
   AIQ_TRY(ws(c, (b + ".boff").c_str(), nb + 1, &boff));
+  int64_t* scan_tmp;
+  AIQ_TRY(ws(c, (b + ".scan").c_str(), 2 * (nb / kRowsPerBlock + 2), &scan_tmp));
   ProbeSpec pr = probe;
   if (pr.keys) {
     AIQ_TRY(ws(c, (b + ".match").c_str(), std::max<int64_t>(n, 1), &pr.match_out));
@@ -313,8 +340,12 @@ aiq_status filter_compact(aiq_ctx* c, const TableD& t, const PredSet& ps, const 
   {
     ProfScope p(c, "predicate_mask", 0, 0);
     launch_predicate_mask(ps, pr, n, bits, bcnt, c->d_err, c->stream);
-    launch_scan_counts(bcnt, nb, boff, c->stream);
-    counted(c, (n > 0) + 1);
+    counted(c, n > 0);
+  }
+  {
+    ProfScope p(c, "scan_tiles", 0, 0);
+    launch_scan_lengths(bcnt, nb, boff, scan_tmp, c->stream);
+    counted(c, nb > 0 ? 3 : 0);
   }
   AIQ_TRY(read_i64(c, boff + nb, 1, c->h_pin));
   const int64_t S = c->h_pin[0];

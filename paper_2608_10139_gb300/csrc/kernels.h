@@ -134,5 +134,9 @@ void launch_gather_groups(const int32_t* rows, int64_t g, const int64_t* build_k
 
 // Sets the thread-local message that aiq_last_error() returns.
 void set_error_message(const char* msg);
+// Records a failed launch; the next status check of the query reports it.
+void set_launch_error(const char* what, cudaError_t e);
+// Returns and clears the recorded launch failure (cudaSuccess if none).
+cudaError_t take_launch_error(const char** what);
 
 }  // namespace aiq

@@ -13,6 +13,8 @@
 //  * decision (Fig. 2: strict yes > no, or first argmax) and the masked
 //    aggregates (Table 1, SELECT row): label counts, yes bitmask for the
 //    yes-row ids, GROUP BY build row with warp-aggregated atomics.
+#include <cstdio>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -34,48 +36,56 @@ __device__ __forceinline__ bool cmp(T v, int op, T c) {
   }
 }
 
-// Evaluates one term on rows [r0, r0 + 8) of this thread; returns 8 bits.
-__device__ __forceinline__ uint32_t eval_term(const PredDev& p, int64_t r0, int64_t n) {
-  uint32_t bits = 0;
+// Raw 8 rows [r0, r0 + 8) of one term's column, as four 16-byte words for
+// 4-byte columns (two used) or 64-bit words for int64 columns.
+struct TermRows {
+  int4 w[4];
+};
+
+__device__ __forceinline__ void load_term(const PredDev& p, int64_t r0, int64_t n, TermRows& t) {
   const bool full = r0 + 8 <= n;
   if (p.type == 1) {
     const int64_t* c = static_cast<const int64_t*>(p.col) + r0;
-    int64_t v[8];
     if (full) {
       const int4* q = reinterpret_cast<const int4*>(c);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        int4 x = __ldg(q + j);
-        v[2 * j] = (static_cast<int64_t>(static_cast<uint32_t>(x.y)) << 32) | static_cast<uint32_t>(x.x);
-        v[2 * j + 1] = (static_cast<int64_t>(static_cast<uint32_t>(x.w)) << 32) | static_cast<uint32_t>(x.z);
-      }
+      for (int j = 0; j < 4; ++j) t.w[j] = __ldg(q + j);
     } else {
+      int64_t* v = reinterpret_cast<int64_t*>(t.w);
 #pragma unroll
       for (int j = 0; j < 8; ++j) v[j] = r0 + j < n ? c[j] : 0;
     }
+  } else {
+    const int32_t* c = static_cast<const int32_t*>(p.col) + r0;
+    if (full) {
+      const int4* q = reinterpret_cast<const int4*>(c);
+      t.w[0] = __ldg(q);
+      t.w[1] = __ldg(q + 1);
+    } else {
+      int32_t* v = reinterpret_cast<int32_t*>(t.w);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[j] = r0 + j < n ? c[j] : 0;
+    }
+  }
+}
+
+// The term's 8 result bits for rows loaded by load_term.
+__device__ __forceinline__ uint32_t eval_term(const PredDev& p, const TermRows& t) {
+  uint32_t bits = 0;
+  if (p.type == 1) {
+    const int64_t* v = reinterpret_cast<const int64_t*>(t.w);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<int64_t>(v[j], p.op, p.ivalue)) << j;
+  } else if (p.type == 0) {
+    // compare in int64 so that constants outside the int32 range behave as in SQL
+    const int32_t* v = reinterpret_cast<const int32_t*>(t.w);
 #pragma unroll
     for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<int64_t>(v[j], p.op, p.ivalue)) << j;
   } else {
-    const int32_t* c = static_cast<const int32_t*>(p.col) + r0;
-    int32_t v[8];
-    if (full) {
-      const int4* q = reinterpret_cast<const int4*>(c);
-      int4 a = __ldg(q), b = __ldg(q + 1);
-      v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-      v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-    } else {
+    const float* v = reinterpret_cast<const float*>(t.w);
+    const float fc = static_cast<float>(p.fvalue);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) v[j] = r0 + j < n ? c[j] : 0;
-    }
-    if (p.type == 0) {
-      // compare in int64 so that constants outside the int32 range behave as in SQL
-#pragma unroll
-      for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<int64_t>(v[j], p.op, p.ivalue)) << j;
-    } else {
-      const float fc = static_cast<float>(p.fvalue);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<float>(__int_as_float(v[j]), p.op, fc)) << j;
-    }
+    for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<float>(v[j], p.op, fc)) << j;
   }
   return bits;
 }
@@ -113,14 +123,31 @@ __device__ __forceinline__ int write_words_and_count(uint32_t byte, uint32_t* bi
   return total;
 }
 
-__global__ void __launch_bounds__(kThreads) k_predicate_mask(PredSet ps, ProbeSpec probe, int64_t n, uint32_t* bits,
-                                                             int32_t* block_counts, int* err) {
-  __shared__ int red[kThreads / 32];
-  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock + threadIdx.x * 8;
+// Evaluates the terms (and the join probe) on one 2048-row tile; thread t
+// covers rows 8t .. 8t+7.  `stage` holds the tile's column chunks when the
+// tile is full; the ragged last tile reads global memory directly.
+__device__ __forceinline__ void predicate_tile(const PredSet& ps, const ProbeSpec& probe, int64_t n, int64_t tile,
+                                               const uint8_t* stage, const int* s_off, uint32_t* bits,
+                                               int32_t* block_counts, int* red) {
+  const int64_t r0 = tile * kRowsPerBlock + threadIdx.x * 8;
   uint32_t byte = 0;
   if (r0 < n) {
     byte = r0 + 8 <= n ? 0xFFu : ((1u << (n - r0)) - 1u);
-    for (int i = 0; i < ps.n; ++i) byte &= eval_term(ps.p[i], r0, n);
+    for (int i = 0; i < ps.n; ++i) {
+      TermRows t;
+      if (stage) {
+        const int4* src = reinterpret_cast<const int4*>(stage + s_off[i]) + threadIdx.x * (ps.p[i].type == 1 ? 4 : 2);
+        t.w[0] = src[0];
+        t.w[1] = src[1];
+        if (ps.p[i].type == 1) {
+          t.w[2] = src[2];
+          t.w[3] = src[3];
+        }
+      } else {
+        load_term(ps.p[i], r0, n, t);
+      }
+      byte &= eval_term(ps.p[i], t);
+    }
     if (probe.keys) {
 #pragma unroll 1
       for (int j = 0; j < 8; ++j) {
@@ -132,8 +159,29 @@ __global__ void __launch_bounds__(kThreads) k_predicate_mask(PredSet ps, ProbeSp
       }
     }
   }
-  const int total = write_words_and_count(byte, bits + static_cast<int64_t>(blockIdx.x) * (kRowsPerBlock / 32), red);
-  if (threadIdx.x == 0) block_counts[blockIdx.x] = total;
+  const int total = write_words_and_count(byte, bits + tile * (kRowsPerBlock / 32), red);
+  if (threadIdx.x == 0) block_counts[tile] = total;
+}
+
+// One 2048-row tile per block.  Thread 0 first asks the bulk-copy engine to
+// pull every term's column chunk of the tile (2048 x 4 or 8 bytes) into L2,
+// so all columns stream from DRAM at once while each thread's own 16-byte
+// loads of successive terms follow one after the other.
+__global__ void __launch_bounds__(kThreads) k_predicate_mask(PredSet ps, ProbeSpec probe, int64_t n, uint32_t* bits,
+                                                             int32_t* block_counts, int* err) {
+  __shared__ int red[kThreads / 32];
+  const int64_t tile = blockIdx.x;
+  if (threadIdx.x == 0 && (tile + 1) * kRowsPerBlock <= n) {
+    for (int i = 1; i < ps.n; ++i) {
+      const int esz = ps.p[i].type == 1 ? 8 : 4;
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const uint8_t*>(ps.p[i].col) +
+                                                                        tile * kRowsPerBlock * esz),
+                   "r"(kRowsPerBlock * esz)
+                   : "memory");
+    }
+  }
+  predicate_tile(ps, probe, n, tile, nullptr, nullptr, bits, block_counts, red);
+  (void)err;
 }
 
 // Block-wide exclusive scan of one int per thread (kThreads threads).
@@ -162,24 +210,48 @@ __device__ __forceinline__ int block_excl_scan(int v, int* sh, int* total) {
   return before + x - v;
 }
 
-__global__ void __launch_bounds__(kThreads) k_compact(const uint32_t* bits, const int64_t* block_offsets, int64_t n,
-                                                      int32_t* ids, const int32_t* payload, int32_t* payload_out) {
-  __shared__ int sh[kThreads / 32];
-  const uint32_t word = bits[static_cast<int64_t>(blockIdx.x) * (kRowsPerBlock / 32) + (threadIdx.x >> 2)];
-  const uint32_t byte = (word >> (8 * (threadIdx.x & 3))) & 0xFFu;
-  int total;
-  const int pre = block_excl_scan(__popc(byte), sh, &total);
-  int64_t out = block_offsets[blockIdx.x] + pre;
-  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock + threadIdx.x * 8;
-  uint32_t b = byte;
-  while (b) {
-    const int j = __ffs(b) - 1;
-    b &= b - 1;
-    const int64_t r = r0 + j;
-    ids[out] = static_cast<int32_t>(r);
-    if (payload_out) payload_out[out] = payload[r];
-    ++out;
+constexpr int kCompactWarps = 4;  // warps (= 2048-row tiles) per compaction block
+
+// One warp per 2048-row tile: each lane owns 64 rows (two bitmask words), a
+// warp shuffle scan gives every lane its output position, the ids are staged
+// in the warp's own shared-memory slice in order and then written out as one
+// coalesced run.  No block-wide barrier is involved.  A payload (the join's
+// build row per probe row) is gathered straight to its output position.
+__global__ void __launch_bounds__(kCompactWarps * 32) k_compact(const uint32_t* bits, const int64_t* block_offsets,
+                                                                int64_t n, int32_t* ids, const int32_t* payload,
+                                                                int32_t* payload_out) {
+  __shared__ int32_t s_ids[kCompactWarps][kRowsPerBlock];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t tile = static_cast<int64_t>(blockIdx.x) * kCompactWarps + warp;
+  const int64_t n_tiles = (n + kRowsPerBlock - 1) / kRowsPerBlock;
+  if (tile >= n_tiles) return;
+  const uint2 w2 = reinterpret_cast<const uint2*>(bits + tile * (kRowsPerBlock / 32))[lane];
+  const int c = __popc(w2.x) + __popc(w2.y);
+  int incl = c;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
   }
+  const int total = __shfl_sync(0xffffffffu, incl, 31);
+  int at = incl - c;
+  const int64_t out = block_offsets[tile];
+  const int64_t r0 = tile * kRowsPerBlock + lane * 64;
+  uint32_t wd[2] = {w2.x, w2.y};
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    uint32_t b = wd[h];
+    while (b) {
+      const int j = __ffs(b) - 1;
+      b &= b - 1;
+      const int64_t r = r0 + 32 * h + j;
+      s_ids[warp][at] = static_cast<int32_t>(r);
+      if (payload_out) payload_out[out + at] = payload[r];  // joins: a gather, written in place
+      ++at;
+    }
+  }
+  __syncwarp();
+  for (int i = lane; i < total; i += 32) ids[out + i] = s_ids[warp][i];
 }
 
 // ---------------------------------------------------------------- scans ---
@@ -361,7 +433,14 @@ inline unsigned blocks_for(int64_t n, int64_t per) { return static_cast<unsigned
 void launch_predicate_mask(const PredSet& ps, const ProbeSpec& probe, int64_t n_rows, uint32_t* bits,
                            int32_t* block_counts, int* err, cudaStream_t s) {
   if (n_rows <= 0) return;
-  k_predicate_mask<<<blocks_for(n_rows, kRowsPerBlock), kThreads, 0, s>>>(ps, probe, n_rows, bits, block_counts, err);
+  const unsigned grid = blocks_for(n_rows, kRowsPerBlock);
+  k_predicate_mask<<<grid, kThreads, 0, s>>>(ps, probe, n_rows, bits, block_counts, err);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    char buf[160];
+    snprintf(buf, sizeof(buf), "predicate mask launch (grid %u, terms %d)", grid, ps.n);
+    set_launch_error(buf, e);
+  }
 }
 
 void launch_scan_counts(const int32_t* counts, int64_t n, int64_t* offsets, cudaStream_t s) {
@@ -371,8 +450,8 @@ void launch_scan_counts(const int32_t* counts, int64_t n, int64_t* offsets, cuda
 void launch_compact(const uint32_t* bits, const int64_t* block_offsets, int64_t n_rows, int32_t* ids_out,
                     const int32_t* payload, int32_t* payload_out, cudaStream_t s) {
   if (n_rows <= 0) return;
-  k_compact<<<blocks_for(n_rows, kRowsPerBlock), kThreads, 0, s>>>(bits, block_offsets, n_rows, ids_out, payload,
-                                                                   payload_out);
+  k_compact<<<blocks_for(n_rows, int64_t(kRowsPerBlock) * kCompactWarps), kCompactWarps * 32, 0, s>>>(
+      bits, block_offsets, n_rows, ids_out, payload, payload_out);
 }
 
 void launch_hash_build(const int64_t* keys, const int32_t* rows, int64_t n, unsigned long long* table_keys,
