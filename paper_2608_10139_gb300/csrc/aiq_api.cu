@@ -146,6 +146,7 @@ struct aiq_ctx {
   int64_t token_budget = 131072;
   bool profile = false;
   bool gemm_pair = true;  // CTA-pair (cta_group::2) GEMM tiles where the shape allows
+  bool attention_tc = true;  // tcgen05 attention where the head shape allows
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
   std::map<std::string, StatAcc> stats;
@@ -293,6 +294,31 @@ aiq_status gemm(aiq_ctx* c, const char* name, const __half* A, int64_t lda, cons
   return AIQ_OK;
 }
 
+// Causal GQA attention over a packed chunk: the work list, then the tcgen05
+// kernel (head_dim 64/128) or the mma.sync kernel.
+aiq_status attention(aiq_ctx* c, const __half* qkv, int64_t T, int64_t n_seqs, const int32_t* seq_start,
+                     int32_t* tile_seq, int32_t* tile_q0, int32_t* n_tiles, int Hq, int Hkv, int hd,
+                     const __half* pkv, int P, __half* out) {
+  const bool tc = c->attention_tc && attention_tc_supported(hd, Hq, Hkv);
+  const int tq = tc ? attention_tc_tile_tokens(Hq, Hkv) : 64;
+  const int n_tiles_max = static_cast<int>((T + tq - 1) / tq + n_seqs);
+  launch_attn_tiles(seq_start, static_cast<int32_t>(n_seqs), tq, tile_seq, tile_q0, n_tiles, c->stream);
+  counted(c, 1);
+  ProfScope p(c, "attention", 0, 0);
+  if (tc) {
+    const int e = launch_attention_tc(qkv, T, seq_start, tile_seq, tile_q0, n_tiles_max, n_tiles, Hq, Hkv, hd, pkv, P,
+                                      out, c->d_err, c->num_sms, c->stream);
+    if (e != 0)
+      return fail(AIQ_ERR_CUDA, std::string("tcgen05 attention launch: ") +
+                                    cudaGetErrorString(static_cast<cudaError_t>(e)));
+  } else {
+    launch_attention(qkv, T, seq_start, tile_seq, tile_q0, n_tiles_max, n_tiles, Hq, Hkv, hd, pkv, P, out, c->d_err,
+                     c->stream);
+  }
+  counted(c, T > 0 && n_seqs > 0);
+  return AIQ_OK;
+}
+
 // ------------------------------------------------------------ validation ---
 
 aiq_status make_pred_set(const TableD& t, const aiq_pred* preds, int32_t n, PredSet* ps) {
@@ -401,8 +427,8 @@ aiq_status prefill_bufs(aiq_ctx* c, const ModelD& m, int64_t B, int64_t max_rows
   AIQ_TRY(ws(c, "pf.pos", B, &pb->pos));
   AIQ_TRY(ws(c, "pf.seq_start", B + 1, &pb->seq_start));
   AIQ_TRY(ws(c, "pf.last", B, &pb->last_idx));
-  AIQ_TRY(ws(c, "pf.tile_seq", B / 64 + B + 1, &pb->tile_seq));
-  AIQ_TRY(ws(c, "pf.tile_q0", B / 64 + B + 1, &pb->tile_q0));
+  AIQ_TRY(ws(c, "pf.tile_seq", B / 8 + B + 1, &pb->tile_seq));
+  AIQ_TRY(ws(c, "pf.tile_q0", B / 8 + B + 1, &pb->tile_q0));
   AIQ_TRY(ws(c, "pf.n_tiles", 1, &pb->n_tiles));
   AIQ_TRY(ws(c, "pf.resid", B * g.d_model, &pb->resid));
   AIQ_TRY(ws(c, "pf.xn", B * g.d_model, &pb->xn));
@@ -429,12 +455,10 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
   const int64_t ldkv = 2 * static_cast<int64_t>(Hkv) * hd;
   const int M = static_cast<int>(T);
   {
-    ProfScope p(c, "attn_tiles+embed", 0, 0);
-    launch_attn_tiles(b.seq_start, static_cast<int32_t>(n_seqs), b.tile_seq, b.tile_q0, b.n_tiles, nullptr, c->stream);
+    ProfScope p(c, "embed", 0, 0);
     launch_embed(b.tok, T, m.embed, d, b.resid, c->stream);
-    counted(c, 1 + (T > 0));
+    counted(c, T > 0);
   }
-  const int n_tiles_max = static_cast<int>((T + 63) / 64 + n_seqs);
   for (int l = 0; l < g.n_layers; ++l) {
     const LayerD& L = m.layers[l];
     {
@@ -456,12 +480,8 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
     if (pkv_out && T > 0)
       CUDA_TRY(cudaMemcpy2DAsync(pkv_out + l * T * ldkv, ldkv * sizeof(__half), b.qkv + Hq * hd,
                                  nqkv * sizeof(__half), ldkv * sizeof(__half), T, cudaMemcpyDeviceToDevice, c->stream));
-    {
-      ProfScope p(c, "attention", 0, 0);
-      launch_attention(b.qkv, T, b.seq_start, b.tile_seq, b.tile_q0, n_tiles_max, b.n_tiles, Hq, Hkv, hd,
-                       pkv_in ? pkv_in + l * P_in * ldkv : nullptr, P_in, b.att, c->d_err, c->stream);
-      counted(c, n_tiles_max > 0);
-    }
+    AIQ_TRY(attention(c, b.qkv, T, n_seqs, b.seq_start, b.tile_seq, b.tile_q0, b.n_tiles, Hq, Hkv, hd,
+                      pkv_in ? pkv_in + l * P_in * ldkv : nullptr, P_in, b.att));
     const bool prune = rows_only_last && l == g.n_layers - 1;
     const __half* att = b.att;
     float* resid = b.resid;
@@ -1175,6 +1195,10 @@ aiq_status aiq_set_option(aiq_ctx* c, const char* name, int64_t value) {
     c->gemm_pair = value != 0;
     return AIQ_OK;
   }
+  if (!std::strcmp(name, "attention_tc")) {
+    c->attention_tc = value != 0;
+    return AIQ_OK;
+  }
   return fail(AIQ_ERR_INVALID_ARG, std::string("unknown option ") + name);
 }
 
@@ -1250,16 +1274,16 @@ aiq_status aiq_op_attention(aiq_ctx* c, const void* qkv, int64_t T, const int32_
   if (n_seqs == 0 || T == 0) return AIQ_OK;
   CUDA_TRY(cudaSetDevice(c->device));
   int32_t *tile_seq, *tile_q0, *n_tiles;
-  const int64_t cap = T / 64 + n_seqs + 1;
+  const int64_t cap = T / 8 + n_seqs + 1;
   AIQ_TRY(ws(c, "op.tile_seq", cap, &tile_seq));
   AIQ_TRY(ws(c, "op.tile_q0", cap, &tile_q0));
   AIQ_TRY(ws(c, "op.n_tiles", 1, &n_tiles));
-  launch_attn_tiles(seq_start, n_seqs, tile_seq, tile_q0, n_tiles, nullptr, c->stream);
   if (P < 0 || (P > 0 && !prefix_kv)) return fail(AIQ_ERR_INVALID_ARG, "bad prefix");
-  launch_attention(static_cast<const __half*>(qkv), T, seq_start, tile_seq, tile_q0, static_cast<int>(cap - 1),
-                   n_tiles, Hq, Hkv, hd, static_cast<const __half*>(prefix_kv), P, static_cast<__half*>(out), c->d_err,
-                   c->stream);
-  return sync_and_check(c);
+  AIQ_TRY(attention(c, static_cast<const __half*>(qkv), T, n_seqs, seq_start, tile_seq, tile_q0, n_tiles, Hq, Hkv, hd,
+                    static_cast<const __half*>(prefix_kv), P, static_cast<__half*>(out)));
+  const aiq_status st = sync_and_check(c);
+  collect_profile(c);
+  return st;
 }
 
 }  // extern "C"

@@ -1,0 +1,487 @@
+// Causal grouped-query attention on the 5th-generation tensor cores.
+//
+// One work item = (32 consecutive tokens of one sequence) x (the 4 query heads
+// sharing one key/value head): its 128 query rows fill the M = 128 rows of a
+// tcgen05 MMA, so every key/value block is fetched once per head group.  The
+// keys of the shared prompt prefix (computed once per query, in prefix_kv)
+// come first, then the sequence's own keys up to the tile's last token.
+//
+//   warp 0    TMA: the Q tile (3-D box hd x heads x tokens), then K and V
+//             blocks of 64 keys into a two-slot ring (128-byte swizzle).
+//   warp 1    tcgen05.mma: S = Q K^T into one of two TMEM score buffers, and
+//             O += P V^T into the TMEM output accumulator.
+//   warps 2-5 one query row per thread: read its 64 scores with tcgen05.ld,
+//             apply the causal / prefix / length mask, keep the running max
+//             (the output is rescaled only when the max grows by more than
+//             2^8, so P never exceeds 256), write exp2(s - max) as fp16 into
+//             the swizzled P tile and transpose their quarter of the V block
+//             into the K-major V^T tile with ldmatrix.trans; at the end divide
+//             by the row sum and store the output row.
+// Work items are persistent per CTA; every wait is bounded.
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace aiq {
+namespace {
+
+constexpr int kThreadsTC = 192;
+constexpr int kKeys = 64;  // keys per block
+
+template <int HD>
+struct ACfg {
+  static constexpr int NC = HD / 64;             // 64-column sub-tiles of one head
+  static constexpr int Q_BYTES = 128 * HD * 2;   // 128 rows
+  static constexpr int SUB = 64 * 128;           // one [64 x 64] fp16 sub-tile
+  static constexpr int K_BYTES = NC * SUB;
+  static constexpr int VT_BYTES = HD * 128;      // HD rows x 64 keys
+  static constexpr int P_BYTES = 128 * 128;      // 128 rows x 64 keys
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = OFF_Q + Q_BYTES;
+  static constexpr int OFF_V = OFF_K + 2 * K_BYTES;
+  static constexpr int OFF_VT = OFF_V + 2 * K_BYTES;
+  static constexpr int OFF_P = OFF_VT + 2 * VT_BYTES;
+  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+  static constexpr int SMEM = 1024 + OFF_BAR + 256;
+  static constexpr int TMEM_COLS = 256;  // two 64-column score buffers + the output
+  static constexpr int O_COL = 128;
+};
+
+struct AttnArgs {
+  const int32_t* seq_start;
+  const int32_t* tile_seq;
+  const int32_t* tile_q0;
+  const int32_t* n_tiles;
+  int Hq, Hkv, G, TQ, P;
+  float scale_log2;
+  __half* out;
+  int* err;
+};
+
+__device__ __forceinline__ void load2x32_f(uint32_t ta, uint32_t tb, float* va, float* vb) {
+  uint32_t ra[32], rb[32];
+  tmem_ld_32x32b_x32(ta, ra);
+  tmem_ld_32x32b_x32(tb, rb);
+  tmem_ld_wait();
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    va[j] = __uint_as_float(ra[j]);
+    vb[j] = __uint_as_float(rb[j]);
+  }
+}
+
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t saddr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(saddr));
+}
+
+__device__ __forceinline__ void st_shared_u32(uint32_t saddr, uint32_t v) {
+  asm volatile("st.shared.u32 [%0], %1;" ::"r"(saddr), "r"(v) : "memory");
+}
+__device__ __forceinline__ void st_shared_v4(uint32_t saddr, uint4 v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(saddr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+
+template <int HD>
+__global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
+    k_attention_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
+                   const __grid_constant__ CUtensorMap tm_pre, AttnArgs a) {
+  using C = ACfg<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem + C::OFF_Q;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
+  uint64_t* q_full = bars + 0;
+  uint64_t* q_empty = bars + 1;
+  uint64_t* kv_full = bars + 2;   // [2]
+  uint64_t* kv_empty = bars + 4;  // [2]
+  uint64_t* s_full = bars + 6;    // [2]
+  uint64_t* p_full = bars + 8;    // [2]
+  uint64_t* o_done = bars + 10;   // [2]: PV of block g commits o_done[g & 1]
+  uint64_t* o_free = bars + 12;
+  uint64_t* mma_done = bars + 13;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 14);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  auto sK = [&](int b) { return smem + C::OFF_K + b * C::K_BYTES; };
+  auto sV = [&](int b) { return smem + C::OFF_V + b * C::K_BYTES; };
+  auto sVt = [&](int b) { return smem + C::OFF_VT + b * C::VT_BYTES; };
+  auto sP = [&](int b) { return smem + C::OFF_P + b * C::P_BYTES; };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  int* err = a.err;
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&kv_full[b], 1);
+      mbar_init(&kv_empty[b], 1);
+      mbar_init(&s_full[b], 1);
+      mbar_init(&p_full[b], 4);
+      mbar_init(&o_done[b], 1);
+    }
+    mbar_init(o_free, 4);
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_kv);
+    tma_prefetch_desc(&tm_pre);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+    tc_fence_before();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int n_work = *a.n_tiles * a.Hkv;
+  const int n_pre = (a.P + kKeys - 1) / kKeys;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA
+      uint32_t g = 0;  // key blocks issued so far (ring position)
+      int it = 0;
+      bool ok = true;
+      for (int w = blockIdx.x; w < n_work && ok; w += gridDim.x, ++it) {
+        const int tidx = w / a.Hkv, kvh = w % a.Hkv;
+        const int s = a.tile_seq[tidx], q0 = a.tile_q0[tidx];
+        const int st = a.seq_start[s], len = a.seq_start[s + 1] - st;
+        const int q_end = min(q0 + a.TQ, len);
+        const int n_kv = n_pre + (q_end + kKeys - 1) / kKeys;
+        if (!mbar_wait_bounded(q_empty, (it & 1) ^ 1, abort_flag, err)) break;
+        mbar_arrive_expect_tx(q_full, C::Q_BYTES);
+        for (int c = 0; c < C::NC; ++c) tma_load_3d(sQ + c * (128 * 128), &tm_q, q_full, c * 64, kvh * a.G, st + q0);
+        for (int j = 0; j < n_kv; ++j, ++g) {
+          const int b = g & 1;
+          if (!mbar_wait_bounded(&kv_empty[b], ((g >> 1) & 1) ^ 1, abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&kv_full[b], 2 * C::K_BYTES);
+          const bool pre = j < n_pre;
+          const CUtensorMap* map = pre ? &tm_pre : &tm_kv;
+          const int kcol = pre ? kvh * HD : (a.Hq + kvh) * HD;
+          const int vcol = pre ? (a.Hkv + kvh) * HD : (a.Hq + a.Hkv + kvh) * HD;
+          const int row = pre ? j * kKeys : st + (j - n_pre) * kKeys;
+          for (int c = 0; c < C::NC; ++c) {
+            tma_load_2d(sK(b) + c * C::SUB, map, &kv_full[b], kcol + c * 64, row);
+            tma_load_2d(sV(b) + c * C::SUB, map, &kv_full[b], vcol + c * 64, row);
+          }
+        }
+      }
+      if (!ok || *abort_flag) {
+        // let this thread's copies still in flight land before the CTA can exit
+        volatile int never = 0;
+        for (uint32_t i = g > 2 ? g - 2 : 0; i < g; ++i)
+          mbar_wait_bounded(&kv_full[i & 1], (i >> 1) & 1, &never, nullptr, 200000000ull);
+        mbar_wait_bounded(q_full, (it & 1), &never, nullptr, 200000000ull);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ MMA
+      constexpr uint32_t idesc_s = idesc_f16_f32(128, kKeys);
+      constexpr uint32_t idesc_o = idesc_f16_f32(128, HD);
+      uint32_t g = 0;
+      int it = 0;
+      bool ok = true;
+      auto issue_s = [&](uint32_t gg) -> bool {
+        const int b = gg & 1;
+        if (!mbar_wait_bounded(&kv_full[b], (gg >> 1) & 1, abort_flag, err)) return false;
+        tc_fence_after();
+        const uint32_t d = tmem_base + b * kKeys;
+#pragma unroll
+        for (int c = 0; c < C::NC; ++c)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_f16_ss(d, smem_desc_k_sw128(smem_u32(sQ + c * (128 * 128)) + k * 32),
+                        smem_desc_k_sw128(smem_u32(sK(b) + c * C::SUB) + k * 32), idesc_s, (c | k) != 0);
+        umma_commit(&s_full[b]);
+        return true;
+      };
+      for (int w = blockIdx.x; w < n_work && ok; w += gridDim.x, ++it) {
+        const int tidx = w / a.Hkv;
+        const int s = a.tile_seq[tidx], q0 = a.tile_q0[tidx];
+        const int len = a.seq_start[s + 1] - a.seq_start[s];
+        const int q_end = min(q0 + a.TQ, len);
+        const int n_kv = n_pre + (q_end + kKeys - 1) / kKeys;
+        if (!mbar_wait_bounded(q_full, it & 1, abort_flag, err)) break;
+        tc_fence_after();
+        // the softmax warps have read out the previous item's output
+        if (!mbar_wait_bounded(o_free, (it & 1) ^ 1, abort_flag, err)) break;
+        tc_fence_after();
+        if (!issue_s(g)) break;
+        for (int j = 0; j < n_kv; ++j, ++g) {
+          if (j + 1 < n_kv && !issue_s(g + 1)) {
+            ok = false;
+            break;
+          }
+          if (j + 1 == n_kv) umma_commit(q_empty);  // all S MMAs of this item issued
+          const int b = g & 1;
+          if (!mbar_wait_bounded(&p_full[b], (g >> 1) & 1, abort_flag, err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_f16_ss(tmem_base + C::O_COL, smem_desc_k_sw128(smem_u32(sP(b)) + k * 32),
+                        smem_desc_k_sw128(smem_u32(sVt(b)) + k * 32), idesc_o, (j | k) != 0);
+          umma_commit(&kv_empty[b]);
+          umma_commit(&o_done[b]);
+        }
+      }
+      umma_commit(mma_done);
+      volatile int never = 0;
+      mbar_wait_bounded(mma_done, 0, &never, err);
+    }
+  } else {
+    // ------------------------------------------------- softmax / epilogue
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;  // TMEM lane = query row of the tile
+    const int t = r / a.G, gq = r % a.G;
+    const uint32_t trow = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16);
+    uint32_t g = 0;
+    int it = 0;
+    bool ok = true;
+    for (int w = blockIdx.x; w < n_work && ok; w += gridDim.x, ++it) {
+      const int tidx = w / a.Hkv, kvh = w % a.Hkv;
+      const int s = a.tile_seq[tidx], q0 = a.tile_q0[tidx];
+      const int st = a.seq_start[s], len = a.seq_start[s + 1] - st;
+      const int q_end = min(q0 + a.TQ, len);
+      const int n_kv = n_pre + (q_end + kKeys - 1) / kKeys;
+      const int qpos = q0 + t;
+      float m_used = 0.f, l = 0.f;
+      for (int j = 0; j < n_kv; ++j, ++g) {
+        const int b = g & 1;
+        const uint32_t ph = (g >> 1) & 1;
+        if (!mbar_wait_bounded(&s_full[b], ph, abort_flag, err) ||
+            !mbar_wait_bounded(&kv_full[b], ph, abort_flag, err)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        float v[64];
+        load2x32_f(trow + b * kKeys, trow + b * kKeys + 32, v, v + 32);
+        const bool pre = j < n_pre;
+        const int key0 = (pre ? j : j - n_pre) * kKeys;
+        const bool need_mask = pre ? (key0 + kKeys > a.P) : (key0 + kKeys - 1 > q0 || key0 + kKeys > len);
+        float mx = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < 64; ++c) {
+          float x = v[c] * a.scale_log2;
+          if (need_mask) {
+            const int key = key0 + c;
+            if (pre ? key >= a.P : (key > qpos || key >= len)) x = -INFINITY;
+          }
+          v[c] = x;
+          mx = fmaxf(mx, x);
+        }
+        if (j == 0) {
+          m_used = mx == -INFINITY ? 0.f : mx;
+        } else {
+          const bool grow = mx > m_used + 8.f;
+          if (__any_sync(0xffffffffu, grow)) {
+            // rescale this warp's output rows once the previous block's PV is done
+            // (per-slot barrier: PV of block g-3 is already known complete and
+            // PV of block g+1 cannot start before this block's P, so the
+            // parity test cannot alias)
+            if (!mbar_wait_bounded(&o_done[(g - 1) & 1], ((g - 1) >> 1) & 1, abort_flag, err)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const float f = grow ? exp2f(m_used - mx) : 1.f;
+            if (grow) {
+              l *= f;
+              m_used = mx;
+            }
+#pragma unroll 1
+            for (int c = 0; c < HD; c += 32) {
+              uint32_t o[32];
+              tmem_ld_32x32b_x32(trow + C::O_COL + c, o);
+              tmem_ld_wait();
+#pragma unroll
+              for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
+              tmem_st_32x32b_x32(trow + C::O_COL + c, o);
+            }
+            tmem_st_wait();
+          }
+        }
+        // P slot b is free once the PV of two blocks ago has completed
+        if (!mbar_wait_bounded(&kv_empty[b], ph ^ 1, abort_flag, err)) {
+          ok = false;
+          break;
+        }
+        float rs = 0.f;
+        const uint32_t prow = smem_u32(sP(b)) + r * 128;
+#pragma unroll
+        for (int ch = 0; ch < 8; ++ch) {
+          uint32_t pk[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float p0 = exp2f(v[ch * 8 + 2 * i] - m_used);
+            const float p1 = exp2f(v[ch * 8 + 2 * i + 1] - m_used);
+            rs += p0 + p1;
+            __half2 h = __floats2half2_rn(p0, p1);
+            pk[i] = *reinterpret_cast<uint32_t*>(&h);
+          }
+          st_shared_v4(prow + ((ch ^ (r & 7)) << 4), make_uint4(pk[0], pk[1], pk[2], pk[3]));
+        }
+        l += rs;
+        // transpose this warp's 16 keys of the V block into the K-major V^T tile
+        {
+          const uint32_t vbase = smem_u32(sV(b));
+          const uint32_t tbase = smem_u32(sVt(b));
+          const int mi = lane >> 3, rr = lane & 7;
+#pragma unroll
+          for (int i = 0; i < HD / 16; ++i) {
+            const int q = 4 * i + mi;           // 8x8 block: key group (q / (HD/8)), dim group (q % (HD/8))
+            const int kg = q / (HD / 8), dg = q % (HD / 8);
+            const int key = quarter * 16 + kg * 8 + rr;
+            const int d = dg * 8;
+            const uint32_t src = vbase + (d / 64) * C::SUB + key * 128 + ((((d % 64) >> 3) ^ (key & 7)) << 4);
+            uint32_t x[4];
+            ldsm_x4_trans(x, src);
+#pragma unroll
+            for (int m = 0; m < 4; ++m) {
+              const int qm = 4 * i + m;
+              const int kgm = qm / (HD / 8), dgm = qm % (HD / 8);
+              const int dd = dgm * 8 + (lane >> 2);
+              const int kk = quarter * 16 + kgm * 8 + 2 * (lane & 3);
+              st_shared_u32(tbase + dd * 128 + ((((kk >> 3) ^ (dd & 7))) << 4) + (kk & 7) * 2, x[m]);
+            }
+          }
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[b]);
+      }
+      if (!ok) break;
+      // output row: O / l, stored for the tile's real tokens
+      if (!mbar_wait_bounded(&o_done[(g - 1) & 1], ((g - 1) >> 1) & 1, abort_flag, err)) break;
+      tc_fence_after();
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      const bool live = qpos < len;
+      __half* dst = a.out + static_cast<int64_t>(st + qpos) * (a.Hq * HD) + (kvh * a.G + gq) * HD;
+#pragma unroll 1
+      for (int c = 0; c < HD; c += 32) {
+        uint32_t o[32];
+        tmem_ld_32x32b_x32(trow + C::O_COL + c, o);
+        tmem_ld_wait();
+        if (live) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4) {
+            uint32_t pk[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              __half2 h = __floats2half2_rn(__uint_as_float(o[q4 * 8 + 2 * i]) * inv,
+                                            __uint_as_float(o[q4 * 8 + 2 * i + 1]) * inv);
+              pk[i] = *reinterpret_cast<uint32_t*>(&h);
+            }
+            d4[q4] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(o_free);
+    }
+  }
+
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn_attn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+bool map2d(CUtensorMap* m, const __half* base, int64_t rows, int64_t cols) {
+  auto fn = encode_fn_attn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols * 2)};
+  cuuint32_t box[2] = {64, 64};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// qkv viewed as [T][heads][hd]; box = 64 columns x G heads x TQ tokens.
+bool map3d_q(CUtensorMap* m, const __half* base, int64_t T, int heads, int hd, int G, int TQ) {
+  auto fn = encode_fn_attn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(hd), static_cast<cuuint64_t>(heads), static_cast<cuuint64_t>(T)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(hd * 2), static_cast<cuuint64_t>(int64_t(heads) * hd * 2)};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(G), static_cast<cuuint32_t>(TQ)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<__half*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int HD>
+int launch_tc(const CUtensorMap& mq, const CUtensorMap& mkv, const CUtensorMap& mpre, const AttnArgs& a,
+              int n_work_max, int num_sms, cudaStream_t s) {
+  using C = ACfg<HD>;
+  cudaError_t e = cudaFuncSetAttribute(k_attention_tc<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  const int per_sm = C::SMEM <= 113 * 1024 ? 2 : 1;
+  const int grid = n_work_max < num_sms * per_sm ? n_work_max : num_sms * per_sm;
+  if (grid <= 0) return 0;
+  k_attention_tc<HD><<<grid, kThreadsTC, C::SMEM, s>>>(mq, mkv, mpre, a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool attention_tc_supported(int hd, int Hq, int Hkv) {
+  if (hd != 64 && hd != 128) return false;
+  const int G = Hq / Hkv;
+  return Hq % Hkv == 0 && G >= 1 && G <= 128 && 128 % G == 0;
+}
+
+int attention_tc_tile_tokens(int Hq, int Hkv) { return 128 / (Hq / Hkv); }
+
+int launch_attention_tc(const __half* qkv, int64_t T, const int32_t* seq_start, const int32_t* tile_seq,
+                        const int32_t* tile_q0, int n_tiles_max, const int32_t* n_tiles_dev, int Hq, int Hkv, int hd,
+                        const __half* prefix_kv, int P, __half* out, int* err, int num_sms, cudaStream_t s) {
+  if (n_tiles_max <= 0 || T <= 0) return 0;
+  const int G = Hq / Hkv, TQ = 128 / G;
+  const int heads = Hq + 2 * Hkv;
+  CUtensorMap mq, mkv, mpre;
+  if (!map3d_q(&mq, qkv, T, heads, hd, G, TQ) || !map2d(&mkv, qkv, T, int64_t(heads) * hd)) return cudaErrorInvalidValue;
+  if (prefix_kv && P > 0) {
+    if (!map2d(&mpre, prefix_kv, P, int64_t(2) * Hkv * hd)) return cudaErrorInvalidValue;
+  } else {
+    mpre = mkv;
+    P = 0;
+  }
+  AttnArgs a{seq_start, tile_seq, tile_q0, n_tiles_dev, Hq, Hkv, G, TQ, P,
+             1.4426950408889634f / sqrtf(static_cast<float>(hd)), out, err};
+  const int n_work_max = n_tiles_max * Hkv;
+  return hd == 64 ? launch_tc<64>(mq, mkv, mpre, a, n_work_max, num_sms, s)
+                  : launch_tc<128>(mq, mkv, mpre, a, n_work_max, num_sms, s);
+}
+
+}  // namespace aiq

@@ -92,9 +92,9 @@ void launch_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* off
 // The shared prefix as a single sequence at positions 0..P-1.
 void launch_pack_prefix(const int32_t* prefix, int32_t P, int32_t* tok, int32_t* pos, int32_t* seq_start,
                         cudaStream_t s);
-// Attention work list of a chunk: one entry per (sequence, 64-row q block).
-void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t* tile_seq, int32_t* tile_q0,
-                       int32_t* n_tiles_dev, int32_t* scratch, cudaStream_t s);
+// Attention work list of a chunk: one entry per (sequence, block of tile_tokens query tokens).
+void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t tile_tokens, int32_t* tile_seq,
+                       int32_t* tile_q0, int32_t* n_tiles_dev, cudaStream_t s);
 
 // --------------------------------------------------------------- prefill ---
 void launch_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int interleave_block,
@@ -112,6 +112,13 @@ void launch_attention(const __half* qkv, int64_t T, const int32_t* seq_start, co
 // buffers for the final layer's row-only O-projection and MLP.
 void launch_gather_last(const __half* att, int ld_att, const float* resid, int d, const int32_t* last_idx, int64_t n,
                         __half* att_out, float* resid_out, int32_t* last_compact, cudaStream_t s);
+// tcgen05 attention (head_dim 64 or 128, query heads per KV head dividing 128):
+// work items of tile_tokens = 128 / (Hq / Hkv) tokens x one KV-head group.
+bool attention_tc_supported(int hd, int Hq, int Hkv);
+int attention_tc_tile_tokens(int Hq, int Hkv);
+int launch_attention_tc(const __half* qkv, int64_t T, const int32_t* seq_start, const int32_t* tile_seq,
+                        const int32_t* tile_q0, int n_tiles_max, const int32_t* n_tiles_dev, int Hq, int Hkv, int hd,
+                        const __half* prefix_kv, int P, __half* out, int* err, int num_sms, cudaStream_t s);
 // last_idx[r] < 0 reads prefix_last (fp32 [d]) instead of a row of resid.
 void launch_label_head(const float* resid, const int32_t* last_idx, const float* prefix_last, int64_t n_rows, int d,
                        const uint16_t* g, float eps, const uint16_t* lm_head, const uint16_t* lm_bias,

@@ -78,14 +78,14 @@ __global__ void k_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_
   }
 }
 
-// Attention work list: one entry per (sequence, 64-row query block), one block.
-__global__ void __launch_bounds__(1024) k_attn_tiles(const int32_t* seq_start, int32_t n, int32_t* tile_seq,
-                                                     int32_t* tile_q0, int32_t* n_tiles) {
+// Attention work list: one entry per (sequence, block of `tq` query tokens), one block.
+__global__ void __launch_bounds__(1024) k_attn_tiles(const int32_t* seq_start, int32_t n, int32_t tq,
+                                                     int32_t* tile_seq, int32_t* tile_q0, int32_t* n_tiles) {
   __shared__ int32_t sh[1024];
   int32_t carry = 0;
   for (int32_t b = 0; b < n; b += 1024) {
     const int32_t i = b + threadIdx.x;
-    const int32_t cnt = i < n ? (seq_start[i + 1] - seq_start[i] + 63) / 64 : 0;
+    const int32_t cnt = i < n ? (seq_start[i + 1] - seq_start[i] + tq - 1) / tq : 0;
     sh[threadIdx.x] = cnt;
     __syncthreads();
     for (int o = 1; o < 1024; o <<= 1) {
@@ -97,7 +97,7 @@ __global__ void __launch_bounds__(1024) k_attn_tiles(const int32_t* seq_start, i
     int32_t at = carry + sh[threadIdx.x] - cnt;
     for (int32_t q = 0; q < cnt; ++q) {
       tile_seq[at + q] = i;
-      tile_q0[at + q] = q * 64;
+      tile_q0[at + q] = q * tq;
     }
     carry += sh[1023];
     __syncthreads();
@@ -144,9 +144,9 @@ void launch_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* off
                                                                             tok, pos, seq_start, last_idx);
 }
 
-void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t* tile_seq, int32_t* tile_q0,
-                       int32_t* n_tiles_dev, int32_t* /*scratch*/, cudaStream_t s) {
-  k_attn_tiles<<<1, 1024, 0, s>>>(seq_start, n_seqs, tile_seq, tile_q0, n_tiles_dev);
+void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t tile_tokens, int32_t* tile_seq,
+                       int32_t* tile_q0, int32_t* n_tiles_dev, cudaStream_t s) {
+  k_attn_tiles<<<1, 1024, 0, s>>>(seq_start, n_seqs, tile_tokens, tile_seq, tile_q0, n_tiles_dev);
 }
 
 }  // namespace aiq

@@ -135,7 +135,7 @@ def test_rmsnorm(ctx, d):
     _close(_np64(out), ref, 1.5e-3, 1e-4, f"rmsnorm d{d}")
 
 
-@pytest.mark.parametrize("hd,Hq,Hkv", [(32, 4, 4), (64, 8, 2), (128, 4, 1)])
+@pytest.mark.parametrize("hd,Hq,Hkv", [(32, 4, 4), (64, 8, 2), (128, 4, 1), (64, 8, 8), (64, 4, 2), (128, 16, 2)])
 def test_attention_varlen(ctx, hd, Hq, Hkv):
     rng = np.random.default_rng(hd + Hq)
     lens = [1, 5, 64, 65, 130, 300, 17]
@@ -158,7 +158,8 @@ def test_attention_varlen(ctx, hd, Hq, Hkv):
         _close(got[s:s + n], ref, 4e-3, 4e-3, f"attention seq {i} len {n} hd {hd}")
 
 
-@pytest.mark.parametrize("hd,Hq,Hkv,P", [(32, 4, 4, 16), (64, 8, 2, 64), (64, 8, 2, 70), (128, 4, 1, 130)])
+@pytest.mark.parametrize("hd,Hq,Hkv,P", [(32, 4, 4, 16), (64, 8, 2, 64), (64, 8, 2, 70), (128, 4, 1, 130),
+                                         (64, 32, 8, 64), (128, 32, 8, 128)])
 def test_attention_with_shared_prefix(ctx, hd, Hq, Hkv, P):
     """Rows attend a shared prefix's keys/values plus their own: the output at
     each row token equals the oracle's attention over prefix ++ row at that position."""
@@ -238,3 +239,26 @@ def test_gemm_cta_pair_rope(ctx):
     qk = y[:, :rope_cols].reshape(M, Hq + Hkv, hd)
     ref = np.concatenate([tf.rope(qk, pos, 1.0e4).reshape(M, rope_cols), y[:, rope_cols:]], axis=1)
     _close(_np64(out), ref, 2e-3, 2e-3 * np.sqrt(K) * 0.05, "pair rope")
+
+
+def test_attention_tcgen05_matches_mma_sync_kernel(ctx):
+    """The tcgen05 and the mma.sync attention kernels agree on a GQA batch with a
+    shared prefix (both also match the oracle above)."""
+    rng = np.random.default_rng(5)
+    hd, Hq, Hkv, P = 64, 32, 8, 64
+    lens = [3, 40, 64, 97, 200, 1]
+    T = sum(lens)
+    W = (Hq + 2 * Hkv) * hd
+    pre = rng.standard_normal((P, W)).astype(np.float16)
+    rows = rng.standard_normal((T, W)).astype(np.float16)
+    pkv = np.ascontiguousarray(pre[:, Hq * hd:])
+    starts = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    dq, ds, dp = _h(rows), _h(starts), _h(pkv)
+    outs = []
+    for tc in (1, 0):
+        ctx.set_option("attention_tc", tc)
+        out = torch.zeros((T, Hq * hd), dtype=torch.float16, device="cuda")
+        ctx.op_attention(dq.data_ptr(), T, ds.data_ptr(), len(lens), Hq, Hkv, hd, out.data_ptr(), dp.data_ptr(), P)
+        outs.append(_np64(out))
+    ctx.set_option("attention_tc", 1)
+    _close(outs[0], outs[1], 4e-3, 4e-3, "tcgen05 vs mma.sync attention")
