@@ -71,6 +71,14 @@ __device__ __forceinline__ void load2x32_f(uint32_t ta, uint32_t tb, float* va, 
   }
 }
 
+// 2^x with the SFU's approximation (relative error ~2^-22, flushes
+// subnormals): plenty for probabilities that are rounded to fp16 next.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t saddr) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
@@ -271,18 +279,20 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         load2x32_f(trow + b * kKeys, trow + b * kKeys + 32, v, v + 32);
         const bool pre = j < n_pre;
         const int key0 = (pre ? j : j - n_pre) * kKeys;
+        // warp-uniform: only the prefix's last block and the causal diagonal /
+        // sequence end need a mask; then key c is visible iff c < lim
         const bool need_mask = pre ? (key0 + kKeys > a.P) : (key0 + kKeys - 1 > q0 || key0 + kKeys > len);
-        float mx = -INFINITY;
+        if (need_mask) {
+          const int lim = pre ? a.P - key0 : min(qpos + 1, len) - key0;
 #pragma unroll
-        for (int c = 0; c < 64; ++c) {
-          float x = v[c] * a.scale_log2;
-          if (need_mask) {
-            const int key = key0 + c;
-            if (pre ? key >= a.P : (key > qpos || key >= len)) x = -INFINITY;
-          }
-          v[c] = x;
-          mx = fmaxf(mx, x);
+          for (int c = 0; c < 64; ++c) v[c] = c < lim ? v[c] : -INFINITY;
         }
+        // running max on the raw scores; the softmax scale (with log2 e) is
+        // folded into one FFMA inside the exponent below
+        float mr = v[0];
+#pragma unroll
+        for (int c = 1; c < 64; ++c) mr = fmaxf(mr, v[c]);
+        const float mx = mr * a.scale_log2;
         if (j == 0) {
           m_used = mx == -INFINITY ? 0.f : mx;
         } else {
@@ -297,7 +307,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
               break;
             }
             tc_fence_after();
-            const float f = grow ? exp2f(m_used - mx) : 1.f;
+            const float f = grow ? ex2_approx(m_used - mx) : 1.f;
             if (grow) {
               l *= f;
               m_used = mx;
@@ -321,13 +331,14 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         }
         float rs = 0.f;
         const uint32_t prow = smem_u32(sP(b)) + r * 128;
+        const float sc = a.scale_log2, neg_m = -m_used;
 #pragma unroll
         for (int ch = 0; ch < 8; ++ch) {
           uint32_t pk[4];
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
-            const float p0 = exp2f(v[ch * 8 + 2 * i] - m_used);
-            const float p1 = exp2f(v[ch * 8 + 2 * i + 1] - m_used);
+            const float p0 = ex2_approx(fmaf(v[ch * 8 + 2 * i], sc, neg_m));
+            const float p1 = ex2_approx(fmaf(v[ch * 8 + 2 * i + 1], sc, neg_m));
             rs += p0 + p1;
             __half2 h = __floats2half2_rn(p0, p1);
             pk[i] = *reinterpret_cast<uint32_t*>(&h);
