@@ -6,8 +6,9 @@
 // (QKV, O, gate/up and down projections of each layer) run over every token
 // of the packed variable-length batch.
 //
-// Structure (one CTA per SM, persistent over 128 x BN output tiles, tile
-// index n-fastest so concurrently running CTAs share the weight panel in L2):
+// Structure (one CTA per SM, persistent over 128 x BN output tiles, tiles
+// ordered in bands of output columns so running CTAs share one L2-resident
+// slice of the weight matrix):
 //   warp 0  : TMA producer, STAGES-deep ring of (A 128x64, B BNx64) tiles,
 //             128-byte swizzle, one mbarrier per stage (full / empty).
 //   warp 1  : allocates 2*BN TMEM columns (two accumulators) and issues
@@ -45,6 +46,30 @@ struct KArgs {
   int M, N, K;
   GemmEpilogue ep;
 };
+
+// Tile order: bands of at most kBandTiles output-tile columns, all row tiles
+// of a band before the next band, columns fastest within a band.  Running
+// CTAs then share one band of the weight matrix (<= 32 MB for 2048-deep K)
+// that stays in L2 while the activation rows stream past, instead of sweeping
+// the whole weight matrix once per row tile.
+constexpr int kBandTiles = 32;
+
+__device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& mt, int& nt) {
+  const int bw = num_n < kBandTiles ? num_n : kBandTiles;
+  const int full_bands = num_n / bw;
+  const int per_band = num_m * bw;
+  const int band = tile / per_band;
+  if (band < full_bands) {
+    const int r = tile - band * per_band;
+    mt = r / bw;
+    nt = band * bw + r % bw;
+  } else {  // the narrower last band
+    const int w = num_n - full_bands * bw;
+    const int r = tile - full_bands * per_band;
+    mt = r / w;
+    nt = full_bands * bw + r % w;
+  }
+}
 
 __device__ __forceinline__ float u2f(uint32_t u) { return __uint_as_float(u); }
 
@@ -293,8 +318,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t issued = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-        const int m0 = (tile / num_n) * BM;
-        const int n0 = (tile % num_n) * BN;
+        int mt, nt;
+        tile_coords(tile, num_m, num_n, mt, nt);
+        const int m0 = mt * BM;
+        const int n0 = nt * BN;
         for (int kb = 0; kb < kblocks; ++kb) {
           const int s = issued % C::STAGES;
           const uint32_t ph = (issued / C::STAGES) & 1;
@@ -363,8 +390,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     int acc = 0;
     uint32_t acc_ph = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
-      const int m0 = (tile / num_n) * BM;
-      const int n0 = (tile % num_n) * BN;
+      int mt, nt;
+      tile_coords(tile, num_m, num_n, mt, nt);
+      const int m0 = mt * BM;
+      const int n0 = nt * BN;
       epilogue_prefetch<BN, EPI>(args, m0 + quarter * 32 + lane, n0);
       if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
       tc_fence_after();
@@ -466,8 +495,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t issued = 0;
       bool ok = true;
       for (int tile = pair; tile < num_tiles && ok; tile += n_pairs) {
-        const int m0 = (tile / num_n) * 2 * BM;
-        const int n0 = (tile % num_n) * BN;
+        int mt, nt;
+        tile_coords(tile, num_m, num_n, mt, nt);
+        const int m0 = mt * 2 * BM;
+        const int n0 = nt * BN;
         for (int kb = 0; kb < kblocks; ++kb) {
           const int s = issued % C::STAGES;
           const uint32_t ph = (issued / C::STAGES) & 1;
@@ -534,8 +565,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     int acc = 0;
     uint32_t acc_ph = 0;
     for (int tile = pair; tile < num_tiles; tile += n_pairs) {
-      const int m0 = (tile / num_n) * 2 * BM + rank * BM;
-      const int n0 = (tile % num_n) * BN;
+      int mt, nt;
+      tile_coords(tile, num_m, num_n, mt, nt);
+      const int m0 = mt * 2 * BM + rank * BM;
+      const int n0 = nt * BN;
       epilogue_prefetch<BN, EPI>(args, m0 + quarter * 32 + lane, n0);
       if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
       tc_fence_after();
