@@ -69,7 +69,7 @@ struct TableD {
 struct LayerD {
   uint16_t* attn_norm = nullptr;
   uint16_t* mlp_norm = nullptr;
-  __half* wqkv = nullptr;  // [(Hq + 2 Hkv) hd, d]
+  __half* wqkv = nullptr;  // [(Hq + 2 Hkv) hd, d], columns scaled by attn_norm's gain
   __half* wo = nullptr;    // [d, Hq hd]
   __half* wgu = nullptr;   // [2 f, d], gate/up interleaved in blocks of bn_gu / 2 rows
   __half* wd = nullptr;    // [d, f]
@@ -417,6 +417,7 @@ aiq_status ensure_rope(aiq_ctx* c, ModelD& m, int max_pos) {
 struct PrefillBufs {
   int32_t *tok, *pos, *seq_start, *last_idx, *tile_seq, *tile_q0, *n_tiles, *last_compact;
   float *resid, *resid_last;
+  float* ss_attn;  // per-128-column sums of squares of the residual, [T][d / 128]
   __half *xn, *qkv, *att, *act;
 };
 
@@ -436,6 +437,7 @@ aiq_status prefill_bufs(aiq_ctx* c, const ModelD& m, int64_t B, int64_t max_rows
   AIQ_TRY(ws(c, "pf.att", B * g.n_heads * g.head_dim, &pb->att));
   AIQ_TRY(ws(c, "pf.act", std::max(B, max_rows) * g.d_ffn, &pb->act));
   AIQ_TRY(ws(c, "pf.resid_last", max_rows * g.d_model, &pb->resid_last));
+  AIQ_TRY(ws(c, "pf.ss_attn", B * (g.d_model / 128), &pb->ss_attn));
   AIQ_TRY(ws(c, "pf.last_compact", max_rows, &pb->last_compact));
   return AIQ_OK;
 }
@@ -454,18 +456,20 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
   const int nqkv = (Hq + 2 * Hkv) * hd;
   const int64_t ldkv = 2 * static_cast<int64_t>(Hkv) * hd;
   const int M = static_cast<int>(T);
+  // The attention-side RMSNorm is fused: the embedding and every down
+  // projection leave the residual in b.xn as fp16 with its partial sums of
+  // squares in ss_attn, and the QKV GEMM (attn_norm gain folded into its
+  // weights) scales each row by 1/RMS in its epilogue.  The MLP-side norm is
+  // a standalone kernel: fusing it into the O-projection epilogue cost more
+  // there than the kernel it removed.
+  const int parts = d / 128;
   {
     ProfScope p(c, "embed", 0, 0);
-    launch_embed(b.tok, T, m.embed, d, b.resid, c->stream);
+    launch_embed(b.tok, T, m.embed, d, b.resid, b.xn, b.ss_attn, c->d_err, c->stream);
     counted(c, T > 0);
   }
   for (int l = 0; l < g.n_layers; ++l) {
     const LayerD& L = m.layers[l];
-    {
-      ProfScope p(c, "rmsnorm", 0, 0);
-      launch_rmsnorm(b.resid, T, d, L.attn_norm, g.rms_eps, b.xn, c->d_err, c->stream);
-      counted(c, T > 0);
-    }
     GemmEpilogue e1;
     e1.kind = EPI_ROPE_F16;
     e1.out = b.qkv;
@@ -476,6 +480,10 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
     e1.rope_cols = (Hq + Hkv) * hd;
     e1.head_dim = hd;
     e1.err = c->d_err;
+    e1.row_ss = b.ss_attn;
+    e1.ss_parts = parts;
+    e1.d_norm = static_cast<float>(d);
+    e1.eps = g.rms_eps;
     AIQ_TRY(gemm(c, "gemm_qkv_rope", b.xn, d, L.wqkv, d, M, nqkv, d, m.bn_qkv, e1));
     if (pkv_out && T > 0)
       CUDA_TRY(cudaMemcpy2DAsync(pkv_out + l * T * ldkv, ldkv * sizeof(__half), b.qkv + Hq * hd,
@@ -483,37 +491,51 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
     AIQ_TRY(attention(c, b.qkv, T, n_seqs, b.seq_start, b.tile_seq, b.tile_q0, b.n_tiles, Hq, Hkv, hd,
                       pkv_in ? pkv_in + l * P_in * ldkv : nullptr, P_in, b.att));
     const bool prune = rows_only_last && l == g.n_layers - 1;
-    const __half* att = b.att;
-    float* resid = b.resid;
-    int Mo = M;
-    if (prune) {
-      // the attention output is dead after this gather, so its rows are packed into b.qkv
-      ProfScope p(c, "gather_last", 0, 0);
-      launch_gather_last(b.att, Hq * hd, b.resid, d, b.last_idx, n_seqs, b.qkv, b.resid_last, b.last_compact,
-                         c->stream);
-      counted(c, n_seqs > 0);
-      att = b.qkv;
-      resid = b.resid_last;
-      Mo = static_cast<int>(n_seqs);
-    }
     GemmEpilogue e2;
     e2.kind = EPI_RESID_F32;
-    e2.out = resid;
     e2.ldo = d;
     e2.err = c->d_err;
-    AIQ_TRY(gemm(c, "gemm_o_resid", att, Hq * hd, L.wo, Hq * hd, Mo, d, Hq * hd, m.bn_o, e2));
-    {
-      ProfScope p(c, "rmsnorm", 0, 0);
-      launch_rmsnorm(resid, Mo, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
-      counted(c, Mo > 0);
-    }
+    e2.ss_parts = parts;
     GemmEpilogue e3;
     e3.kind = EPI_SWIGLU_F16;
     e3.out = b.act;
     e3.ldo = f;
     e3.err = c->d_err;
-    AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, d, L.wgu, d, Mo, 2 * f, d, m.bn_gu, e3));
-    AIQ_TRY(gemm(c, "gemm_down_resid", b.act, f, L.wd, f, Mo, d, f, m.bn_d, e2));
+    if (!prune) {
+      e2.out = b.resid;
+      AIQ_TRY(gemm(c, "gemm_o_resid", b.att, Hq * hd, L.wo, Hq * hd, M, d, Hq * hd, m.bn_o, e2));
+      {
+        ProfScope p(c, "rmsnorm", 0, 0);
+        launch_rmsnorm(b.resid, T, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+        counted(c, T > 0);
+      }
+      AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, d, L.wgu, d, M, 2 * f, d, m.bn_gu, e3));
+      // the down projection's epilogue prepares the next layer's attention norm
+      // (b.xn is free again: the gate/up GEMM before it has consumed it)
+      e2.xh_out = b.xn;
+      e2.ss_out = b.ss_attn;
+      AIQ_TRY(gemm(c, "gemm_down_resid", b.act, f, L.wd, f, M, d, f, m.bn_d, e2));
+    } else {
+      // final layer, rows only: gather each sequence's last token (the
+      // attention output is dead afterwards, so its rows are packed into
+      // b.qkv), then O-projection, RMSNorm and the MLP on those rows alone
+      {
+        ProfScope p(c, "gather_last", 0, 0);
+        launch_gather_last(b.att, Hq * hd, b.resid, d, b.last_idx, n_seqs, b.qkv, b.resid_last, b.last_compact,
+                           c->stream);
+        counted(c, n_seqs > 0);
+      }
+      const int Mo = static_cast<int>(n_seqs);
+      e2.out = b.resid_last;
+      AIQ_TRY(gemm(c, "gemm_o_resid", b.qkv, Hq * hd, L.wo, Hq * hd, Mo, d, Hq * hd, m.bn_o, e2));
+      {
+        ProfScope p(c, "rmsnorm", 0, 0);
+        launch_rmsnorm(b.resid_last, Mo, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+        counted(c, Mo > 0);
+      }
+      AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, d, L.wgu, d, Mo, 2 * f, d, m.bn_gu, e3));
+      AIQ_TRY(gemm(c, "gemm_down_resid", b.act, f, L.wd, f, Mo, d, f, m.bn_d, e2));
+    }
   }
   return AIQ_OK;
 }
@@ -1077,27 +1099,27 @@ aiq_status aiq_load_model(aiq_ctx* c, const aiq_model_config* cfg, const void* c
   for (int l = 0; l < g.n_layers; ++l) {
     LayerD& L = m.layers[l];
     M_TRY(up_bf16(tensors[ti++], d, &L.attn_norm));
-    // q, k, v stacked then converted: [(Hq + 2 Hkv) hd, d]
+    // q, k, v stacked then converted: [(Hq + 2 Hkv) hd, d], attn_norm gain folded in
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(qd) * d * 2, cudaMemcpyHostToDevice);
     cudaMemcpy(stage + size_t(qd) * d, tensors[ti++], size_t(kd) * d * 2, cudaMemcpyHostToDevice);
     cudaMemcpy(stage + size_t(qd + kd) * d, tensors[ti++], size_t(kd) * d * 2, cudaMemcpyHostToDevice);
     M_TRY(model_alloc(c, m, size_t(qd + 2 * kd) * d, &L.wqkv));
-    launch_bf16_to_f16(stage, L.wqkv, qd + 2 * kd, d, 0, 0, c->d_err, c->stream);
+    launch_bf16_to_f16(stage, L.wqkv, qd + 2 * kd, d, 0, 0, L.attn_norm, c->d_err, c->stream);
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(d) * qd * 2, cudaMemcpyHostToDevice);
     M_TRY(model_alloc(c, m, size_t(d) * qd, &L.wo));
-    launch_bf16_to_f16(stage, L.wo, d, qd, 0, 0, c->d_err, c->stream);
+    launch_bf16_to_f16(stage, L.wo, d, qd, 0, 0, nullptr, c->d_err, c->stream);
     M_TRY(up_bf16(tensors[ti++], d, &L.mlp_norm));
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(f) * d * 2, cudaMemcpyHostToDevice);
     cudaMemcpy(stage + size_t(f) * d, tensors[ti++], size_t(f) * d * 2, cudaMemcpyHostToDevice);
     M_TRY(model_alloc(c, m, size_t(2 * f) * d, &L.wgu));
-    launch_bf16_to_f16(stage, L.wgu, 2 * f, d, m.bn_gu / 2, f, c->d_err, c->stream);
+    launch_bf16_to_f16(stage, L.wgu, 2 * f, d, m.bn_gu / 2, f, nullptr, c->d_err, c->stream);
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(d) * f * 2, cudaMemcpyHostToDevice);
     M_TRY(model_alloc(c, m, size_t(d) * f, &L.wd));
-    launch_bf16_to_f16(stage, L.wd, d, f, 0, 0, c->d_err, c->stream);
+    launch_bf16_to_f16(stage, L.wd, d, f, 0, 0, nullptr, c->d_err, c->stream);
   }
   M_TRY(up_bf16(tensors[ti++], d, &m.final_norm));
   M_TRY(up_bf16(tensors[ti++], V * d, &m.lm_head));

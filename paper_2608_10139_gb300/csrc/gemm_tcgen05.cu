@@ -121,7 +121,8 @@ __device__ __forceinline__ void load_f32x32(const float* src, float* v) {
   }
 }
 
-__device__ __forceinline__ void add_store_f32x32(float* dst, const float* v) {
+// dst += v (fp32), and the new values are returned in out.
+__device__ __forceinline__ void add_store_f32x32(float* dst, const float* v, float* out) {
   float4* p = reinterpret_cast<float4*>(dst);
   float4 x[8];
 #pragma unroll
@@ -133,7 +134,32 @@ __device__ __forceinline__ void add_store_f32x32(float* dst, const float* v) {
     x[j].z += v[4 * j + 2];
     x[j].w += v[4 * j + 3];
     p[j] = x[j];
+    out[4 * j] = x[j].x;
+    out[4 * j + 1] = x[j].y;
+    out[4 * j + 2] = x[j].z;
+    out[4 * j + 3] = x[j].w;
   }
+}
+
+// 1 / RMS of an accumulator row from its partial sums of squares (fixed
+// summation order), or 1 when the GEMM's input is already normalised.
+__device__ __forceinline__ float row_inv_rms(const GemmEpilogue& ep, int row, bool live) {
+  if (!ep.row_ss || !live) return 1.f;
+  const float* p = ep.row_ss + static_cast<int64_t>(row) * ep.ss_parts;
+  float s = 0.f;
+  if ((ep.ss_parts & 3) == 0) {
+    const float4* p4 = reinterpret_cast<const float4*>(p);
+    for (int i = 0; i < ep.ss_parts / 4; ++i) {
+      const float4 v = __ldg(p4 + i);
+      s += v.x;
+      s += v.y;
+      s += v.z;
+      s += v.w;
+    }
+  } else {
+    for (int i = 0; i < ep.ss_parts; ++i) s += p[i];
+  }
+  return rsqrtf(s / ep.d_norm + ep.eps);
 }
 
 __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
@@ -158,20 +184,34 @@ __device__ __forceinline__ void epilogue_prefetch(const KArgs& a, int row, int n
   }
 }
 
+// inv: the row's 1/RMS (fused RMSNorm), computed by the caller before it
+// waits for the accumulator, so that its loads overlap the tile's MMAs.
 template <int BN, int EPI>
-__device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int row, int n0) {
+__device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int row, int n0, float inv) {
   const GemmEpilogue& ep = a.ep;
   const bool live = row < a.M;
   bool bad = false;
   if constexpr (EPI == EPI_RESID_F32) {
     float* o = static_cast<float*>(ep.out) + static_cast<int64_t>(row) * ep.ldo + n0;
+    float part = 0.f;  // sum of squares of the new residual over 128 columns
 #pragma unroll 1
     for (int c = 0; c < BN; c += 64) {
       float v0[32], v1[32];
       load2x32(trow + c, trow + c + 32, v0, v1);
       if (live) {
-        add_store_f32x32(o + c, v0);
-        add_store_f32x32(o + c + 32, v1);
+        add_store_f32x32(o + c, v0, v0);
+        add_store_f32x32(o + c + 32, v1, v1);
+        if (ep.xh_out) {
+          __half* xh = ep.xh_out + static_cast<int64_t>(row) * ep.ldo + n0 + c;
+          store_f16x32(xh, v0, bad);
+          store_f16x32(xh + 32, v1, bad);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) part += v0[j] * v0[j] + v1[j] * v1[j];
+          if ((c & 127) == 64) {
+            ep.ss_out[static_cast<int64_t>(row) * ep.ss_parts + (n0 + c) / 128] = part;
+            part = 0.f;
+          }
+        }
       }
     }
   } else if constexpr (EPI == EPI_SWIGLU_F16) {
@@ -181,7 +221,10 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
       float g[32], u[32];
       load2x32(trow + c, trow + BN / 2 + c, g, u);
 #pragma unroll
-      for (int j = 0; j < 32; ++j) g[j] = g[j] / (1.0f + expf(-g[j])) * u[j];
+      for (int j = 0; j < 32; ++j) {
+        const float gj = g[j] * inv;
+        g[j] = gj / (1.0f + expf(-gj)) * (u[j] * inv);
+      }
       if (live) store_f16x32(o + c, g, bad);
     }
   } else {
@@ -207,7 +250,7 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
             if (live) {
 #pragma unroll
               for (int j = 0; j < 32; ++j) {
-                const float a1 = x1[j], a2 = x2[j];
+                const float a1 = x1[j] * inv, a2 = x2[j] * inv;
                 x1[j] = a1 * cs[j] - a2 * sn[j];
                 x2[j] = a2 * cs[j] + a1 * sn[j];
               }
@@ -233,7 +276,7 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
           if (live) {
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
-              const float a1 = x[j], a2 = x[j + 16];
+              const float a1 = x[j] * inv, a2 = x[j + 16] * inv;
               x[j] = a1 * cs[j] - a2 * sn[j];
               x[j + 16] = a2 * cs[j] + a1 * sn[j];
             }
@@ -249,6 +292,11 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
       float v0[32], v1[32];
       load2x32(trow + c, trow + c + 32, v0, v1);
       if (live) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          v0[j] *= inv;
+          v1[j] *= inv;
+        }
         store_f16x32(o + c, v0, bad);
         store_f16x32(o + c + 32, v1, bad);
       }
@@ -256,7 +304,11 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
     if (c < BN) {
       float v[32];
       load32(trow + c, v);
-      if (live) store_f16x32(o + c, v, bad);
+      if (live) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] *= inv;
+        store_f16x32(o + c, v, bad);
+      }
     }
   }
   if (bad) set_dev_error(ep.err, DEVERR_FP16_RANGE);
@@ -395,10 +447,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int m0 = mt * BM;
       const int n0 = nt * BN;
       epilogue_prefetch<BN, EPI>(args, m0 + quarter * 32 + lane, n0);
+      const float inv = (EPI == EPI_ROPE_F16 || EPI == EPI_SWIGLU_F16)
+                            ? row_inv_rms(args.ep, m0 + quarter * 32 + lane, m0 + quarter * 32 + lane < args.M)
+                            : 1.f;
       if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
       tc_fence_after();
       const uint32_t trow = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-      epilogue_tile<BN, EPI>(args, trow, m0 + quarter * 32 + lane, n0);
+      epilogue_tile<BN, EPI>(args, trow, m0 + quarter * 32 + lane, n0, inv);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -570,10 +625,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int m0 = mt * 2 * BM + rank * BM;
       const int n0 = nt * BN;
       epilogue_prefetch<BN, EPI>(args, m0 + quarter * 32 + lane, n0);
+      const float inv = (EPI == EPI_ROPE_F16 || EPI == EPI_SWIGLU_F16)
+                            ? row_inv_rms(args.ep, m0 + quarter * 32 + lane, m0 + quarter * 32 + lane < args.M)
+                            : 1.f;
       if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
       tc_fence_after();
       const uint32_t trow = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-      epilogue_tile<BN, EPI>(args, trow, m0 + quarter * 32 + lane, n0);
+      epilogue_tile<BN, EPI>(args, trow, m0 + quarter * 32 + lane, n0, inv);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(tempty_leader + acc * 8);

@@ -26,6 +26,17 @@ struct GemmEpilogue {
   int rope_cols = 0;
   int head_dim = 0;
   int* err = nullptr;
+  // RMSNorm fused across GEMMs (the norm gain is folded into the weights):
+  //  - consumer (ROPE / SWIGLU): scale each accumulator row by
+  //    rsqrt(sum(row_ss[row][0..ss_parts)) / d_norm + eps) before the epilogue;
+  //  - producer (RESID): also write the new residual as fp16 (xh_out) and its
+  //    per-128-column sums of squares (ss_out [row][n / 128]).
+  const float* row_ss = nullptr;
+  int ss_parts = 0;
+  float d_norm = 1.f;
+  float eps = 0.f;
+  __half* xh_out = nullptr;
+  float* ss_out = nullptr;
 };
 
 // C = A[M,K] * B[N,K]^T with fp16 operands and fp32 accumulation on tcgen05.
@@ -97,10 +108,17 @@ void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t tile_to
                        int32_t* tile_q0, int32_t* n_tiles_dev, cudaStream_t s);
 
 // --------------------------------------------------------------- prefill ---
+// gain (optional, bf16 [cols]): dst[r][c] = fp16(src[r][c] * gain[c]), the product
+// formed exactly in fp32 and rounded once (an RMSNorm gain folded into the
+// following linear layer).
 void launch_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int interleave_block,
-                        int64_t half_rows, int* err, cudaStream_t s);
+                        int64_t half_rows, const uint16_t* gain, int* err, cudaStream_t s);
 void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, float theta, cudaStream_t s);
-void launch_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, cudaStream_t s);
+// Embedding rows into the fp32 residual; with xh/ss also its fp16 copy and
+// per-128-column sums of squares (the first layer's fused RMSNorm input).
+void launch_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, __half* xh, float* ss,
+                  int* err, cudaStream_t s);
+// g may be null (unit gain).
 void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int* err,
                     cudaStream_t s);
 // prefix_kv (optional): [P, 2 Hkv hd] fp16 keys then values of a shared prefix that

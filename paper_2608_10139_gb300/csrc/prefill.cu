@@ -18,7 +18,7 @@ __device__ __forceinline__ float bf16_bits_to_float(uint16_t b) {
 // matrices (gate then up) and dst rows alternate blocks of ib gate rows and
 // ib up rows, so that one GEMM output tile holds matching gate/up columns.
 __global__ void k_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int ib, int64_t half_rows,
-                              int* err) {
+                              const uint16_t* gain, int* err) {
   const int64_t n = rows * cols;
   bool bad = false;
   for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < n;
@@ -29,7 +29,8 @@ __global__ void k_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, in
       const int64_t b = r / (2 * ib), w = r % (2 * ib);
       sr = w < ib ? b * ib + w : half_rows + b * ib + (w - ib);
     }
-    const float v = bf16_bits_to_float(src[sr * cols + c]);
+    float v = bf16_bits_to_float(src[sr * cols + c]);
+    if (gain) v *= bf16_bits_to_float(gain[c]);  // exact: two 8-bit significands
     bad |= !(fabsf(v) <= 65504.f);
     dst[e] = __float2half_rn(v);
   }
@@ -49,25 +50,52 @@ __global__ void k_rope_table(float* cos_t, float* sin_t, int max_pos, int hd, do
   }
 }
 
-// One warp per token; 8 bf16 (16 bytes) per lane per step.
-__global__ void k_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid) {
+// One warp per token; 8 bf16 (16 bytes) per lane per step.  With xh / ss the
+// row is also written as fp16 and its sums of squares per 128 columns (16
+// lanes x 8 values) are stored, in a fixed order, for the fused RMSNorm.
+__global__ void k_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, __half* xh, float* ss,
+                        int* err) {
   const int64_t t = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (t >= T) return;
   const uint4* src = reinterpret_cast<const uint4*>(emb + static_cast<int64_t>(tok[t]) * d);
   float4* dst = reinterpret_cast<float4*>(resid + t * d);
-  for (int c = lane; c < d / 8; c += 32) {
-    const uint4 v = src[c];
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  bool bad = false;
+  for (int c0 = 0; c0 < d / 8; c0 += 32) {
+    const int c = c0 + lane;
     float f[8];
+    float part = 0.f;
+    if (c < d / 8) {
+      const uint4 v = src[c];
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      f[2 * j] = __uint_as_float(w[j] << 16);
-      f[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+      for (int j = 0; j < 4; ++j) {
+        f[2 * j] = __uint_as_float(w[j] << 16);
+        f[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+      }
+      dst[2 * c] = make_float4(f[0], f[1], f[2], f[3]);
+      dst[2 * c + 1] = make_float4(f[4], f[5], f[6], f[7]);
+      if (xh) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          bad |= !(fabsf(f[2 * j]) <= 65504.f) || !(fabsf(f[2 * j + 1]) <= 65504.f);
+          __half2 h = __floats2half2_rn(f[2 * j], f[2 * j + 1]);
+          pk[j] = *reinterpret_cast<uint32_t*>(&h);
+          part += f[2 * j] * f[2 * j] + f[2 * j + 1] * f[2 * j + 1];
+        }
+        reinterpret_cast<uint4*>(xh + t * d)[c] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      }
     }
-    dst[2 * c] = make_float4(f[0], f[1], f[2], f[3]);
-    dst[2 * c + 1] = make_float4(f[4], f[5], f[6], f[7]);
+    if (ss) {
+      // lanes 16k .. 16k+15 hold columns [128 * (c0 / 16 + k), +128): reduce within the half-warp
+#pragma unroll
+      for (int o = 8; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+      const int slot = (c0 * 8 + (lane >> 4) * 128) / 128;
+      if ((lane & 15) == 0 && c < d / 8) ss[t * (d / 128) + slot] = part;
+    }
   }
+  if (bad) set_dev_error(err, DEVERR_FP16_RANGE);
 }
 
 // One warp per row: fp32 statistics, fp16 output for the next GEMM.
@@ -91,9 +119,14 @@ __global__ void k_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, f
 #pragma unroll
   for (int j = 0; j < PER_LANE; ++j) {
     const int c = (lane + 32 * j) * 4;
-    const uint2 gg = *reinterpret_cast<const uint2*>(g + c);
-    const float g0 = __uint_as_float(gg.x << 16), g1 = __uint_as_float(gg.x & 0xFFFF0000u);
-    const float g2 = __uint_as_float(gg.y << 16), g3 = __uint_as_float(gg.y & 0xFFFF0000u);
+    float g0 = 1.f, g1 = 1.f, g2 = 1.f, g3 = 1.f;
+    if (g) {
+      const uint2 gg = *reinterpret_cast<const uint2*>(g + c);
+      g0 = __uint_as_float(gg.x << 16);
+      g1 = __uint_as_float(gg.x & 0xFFFF0000u);
+      g2 = __uint_as_float(gg.y << 16);
+      g3 = __uint_as_float(gg.y & 0xFFFF0000u);
+    }
     const float a = v[j].x * inv * g0, b = v[j].y * inv * g1, cc = v[j].z * inv * g2, e = v[j].w * inv * g3;
     bad |= !(fabsf(a) <= 65504.f) || !(fabsf(b) <= 65504.f) || !(fabsf(cc) <= 65504.f) || !(fabsf(e) <= 65504.f);
     __half2 h0 = __floats2half2_rn(a, b), h1 = __floats2half2_rn(cc, e);
@@ -114,7 +147,7 @@ __global__ void k_rmsnorm_any(const float* x, int64_t T, int d, const uint16_t* 
   const float inv = rsqrtf(ss / d + eps);
   bool bad = false;
   for (int c = lane; c < d; c += 32) {
-    const float v = row[c] * inv * bf16_bits_to_float(g[c]);
+    const float v = row[c] * inv * (g ? bf16_bits_to_float(g[c]) : 1.f);
     bad |= !(fabsf(v) <= 65504.f);
     out[t * d + c] = __float2half_rn(v);
   }
@@ -168,12 +201,12 @@ inline unsigned grid_for(int64_t threads) { return static_cast<unsigned>((thread
 }  // namespace
 
 void launch_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int interleave_block,
-                        int64_t half_rows, int* err, cudaStream_t s) {
+                        int64_t half_rows, const uint16_t* gain, int* err, cudaStream_t s) {
   const int64_t n = rows * cols;
   if (n <= 0) return;
   unsigned g = grid_for(n);
   if (g > 8192) g = 8192;
-  k_bf16_to_f16<<<g, 256, 0, s>>>(src, dst, rows, cols, interleave_block, half_rows, err);
+  k_bf16_to_f16<<<g, 256, 0, s>>>(src, dst, rows, cols, interleave_block, half_rows, gain, err);
 }
 
 void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, float theta, cudaStream_t s) {
@@ -184,9 +217,10 @@ void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, fl
   k_rope_table<<<g, 256, 0, s>>>(cos_t, sin_t, max_pos, head_dim, static_cast<double>(theta));
 }
 
-void launch_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, cudaStream_t s) {
+void launch_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, __half* xh, float* ss,
+                  int* err, cudaStream_t s) {
   if (T <= 0) return;
-  k_embed<<<grid_for(T * 32), 256, 0, s>>>(tok, T, emb, d, resid);
+  k_embed<<<grid_for(T * 32), 256, 0, s>>>(tok, T, emb, d, resid, xh, ss, err);
 }
 
 void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int* err,
