@@ -269,8 +269,38 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       for (int j = 0; j < n_kv; ++j, ++g) {
         const int b = g & 1;
         const uint32_t ph = (g >> 1) & 1;
-        if (!mbar_wait_bounded(&s_full[b], ph, abort_flag, err) ||
-            !mbar_wait_bounded(&kv_full[b], ph, abort_flag, err)) {
+        // the V block has landed and the V^T / P slot is free once the PV of
+        // two blocks ago has completed: transpose before the scores are ready
+        if (!mbar_wait_bounded(&kv_full[b], ph, abort_flag, err) ||
+            !mbar_wait_bounded(&kv_empty[b], ph ^ 1, abort_flag, err)) {
+          ok = false;
+          break;
+        }
+        // transpose this warp's 16 keys of the V block into the K-major V^T tile
+        {
+          const uint32_t vbase = smem_u32(sV(b));
+          const uint32_t tbase = smem_u32(sVt(b));
+          const int mi = lane >> 3, rr = lane & 7;
+#pragma unroll
+          for (int i = 0; i < HD / 16; ++i) {
+            const int q = 4 * i + mi;           // 8x8 block: key group (q / (HD/8)), dim group (q % (HD/8))
+            const int kg = q / (HD / 8), dg = q % (HD / 8);
+            const int key = quarter * 16 + kg * 8 + rr;
+            const int d = dg * 8;
+            const uint32_t src = vbase + (d / 64) * C::SUB + key * 128 + ((((d % 64) >> 3) ^ (key & 7)) << 4);
+            uint32_t x[4];
+            ldsm_x4_trans(x, src);
+#pragma unroll
+            for (int m = 0; m < 4; ++m) {
+              const int qm = 4 * i + m;
+              const int kgm = qm / (HD / 8), dgm = qm % (HD / 8);
+              const int dd = dgm * 8 + (lane >> 2);
+              const int kk = quarter * 16 + kgm * 8 + 2 * (lane & 3);
+              st_shared_u32(tbase + dd * 128 + ((((kk >> 3) ^ (dd & 7))) << 4) + (kk & 7) * 2, x[m]);
+            }
+          }
+        }
+        if (!mbar_wait_bounded(&s_full[b], ph, abort_flag, err)) {
           ok = false;
           break;
         }
@@ -289,9 +319,14 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         }
         // running max on the raw scores; the softmax scale (with log2 e) is
         // folded into one FFMA inside the exponent below
-        float mr = v[0];
+        // (eight independent partial maxima keep the FMNMX chain short)
+        float pm[8];
 #pragma unroll
-        for (int c = 1; c < 64; ++c) mr = fmaxf(mr, v[c]);
+        for (int c = 0; c < 8; ++c) pm[c] = v[c];
+#pragma unroll
+        for (int c = 8; c < 64; ++c) pm[c & 7] = fmaxf(pm[c & 7], v[c]);
+        const float mr = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
         const float mx = mr * a.scale_log2;
         if (j == 0) {
           m_used = mx == -INFINITY ? 0.f : mx;
@@ -324,12 +359,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
             tmem_st_wait();
           }
         }
-        // P slot b is free once the PV of two blocks ago has completed
-        if (!mbar_wait_bounded(&kv_empty[b], ph ^ 1, abort_flag, err)) {
-          ok = false;
-          break;
-        }
-        float rs = 0.f;
+        float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         const uint32_t prow = smem_u32(sP(b)) + r * 128;
         const float sc = a.scale_log2, neg_m = -m_used;
 #pragma unroll
@@ -339,37 +369,14 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
           for (int i = 0; i < 4; ++i) {
             const float p0 = ex2_approx(fmaf(v[ch * 8 + 2 * i], sc, neg_m));
             const float p1 = ex2_approx(fmaf(v[ch * 8 + 2 * i + 1], sc, neg_m));
-            rs += p0 + p1;
+            ps[2 * i] += p0;
+            ps[2 * i + 1] += p1;
             __half2 h = __floats2half2_rn(p0, p1);
             pk[i] = *reinterpret_cast<uint32_t*>(&h);
           }
           st_shared_v4(prow + ((ch ^ (r & 7)) << 4), make_uint4(pk[0], pk[1], pk[2], pk[3]));
         }
-        l += rs;
-        // transpose this warp's 16 keys of the V block into the K-major V^T tile
-        {
-          const uint32_t vbase = smem_u32(sV(b));
-          const uint32_t tbase = smem_u32(sVt(b));
-          const int mi = lane >> 3, rr = lane & 7;
-#pragma unroll
-          for (int i = 0; i < HD / 16; ++i) {
-            const int q = 4 * i + mi;           // 8x8 block: key group (q / (HD/8)), dim group (q % (HD/8))
-            const int kg = q / (HD / 8), dg = q % (HD / 8);
-            const int key = quarter * 16 + kg * 8 + rr;
-            const int d = dg * 8;
-            const uint32_t src = vbase + (d / 64) * C::SUB + key * 128 + ((((d % 64) >> 3) ^ (key & 7)) << 4);
-            uint32_t x[4];
-            ldsm_x4_trans(x, src);
-#pragma unroll
-            for (int m = 0; m < 4; ++m) {
-              const int qm = 4 * i + m;
-              const int kgm = qm / (HD / 8), dgm = qm % (HD / 8);
-              const int dd = dgm * 8 + (lane >> 2);
-              const int kk = quarter * 16 + kgm * 8 + 2 * (lane & 3);
-              st_shared_u32(tbase + dd * 128 + ((((kk >> 3) ^ (dd & 7))) << 4) + (kk & 7) * 2, x[m]);
-            }
-          }
-        }
+        l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&p_full[b]);
