@@ -12,6 +12,11 @@ Parity status per function:
   transformer.causal_attention  pinned (torch SDPA, identical-key prefix mean)
   transformer.label_logits      pinned (zero-weight bias closed form,
                           identity-layer closed form, causality, GQA duplication)
+  transformer.vocab_logits  pinned (label rows equal the pinned label head,
+                          row t equals the logits of the first t+1 tokens)
+  transformer.greedy_generate  pinned (zero-weight bias closed form, the
+                          permutation-head closed form y_t = pi^(t+1)(x), eos/pad)
+  relational.like_contains     pinned (delimited-string containment, edge cases)
   whole-model numerics at random weights: parity unpinned beyond the
                           component pins (the paper prints no model outputs).
 """

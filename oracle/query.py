@@ -3,7 +3,11 @@
 TEST INFRASTRUCTURE ONLY (tests, smoke check, benchmark CPU-baseline leg).
 
 ``run_select`` follows Table 2 Q1/Q2 with Fig. 2's decision: WHERE relational
-terms AND AI_IF(text) = 1, then the aggregate.  ``run_join_select`` adds the
+terms AND AI_IF(text) = 1, then the aggregate.  ``run_transform`` follows
+Table 2 Q3 (SELECT AI_TRANSFORM(text) ... WHERE relational terms: greedy
+generation for every candidate row) and Q5 (COUNT(*) of the rows whose
+generated text is LIKE '%pattern%', with the matching rows' outputs as the
+debug payload).  ``run_join_select`` adds the
 reviews-movies equi-join on movie id of Section 4's datasets paragraph, with
 the build-side (movies) predicate, and groups the yes rows by movie.
 
@@ -102,3 +106,42 @@ def run_join_select(probe, build, probe_key: str, build_key: str, probe_preds,
                                    build_preds, brute_force)
     return _finish(model, prefix, probe, cand, cand_b, labels, agg, sample,
                    build.cols[build_key])
+
+
+@dataclass
+class TransformResult:
+    cand_rows: np.ndarray          # rows that reach the LM, ascending
+    sample: np.ndarray             # candidate positions the LM was run on
+    tokens: np.ndarray             # [len(sample), n_new] generated ids (pad after eos)
+    text_len: np.ndarray           # [len(sample)] tokens before the eos
+    match: Optional[np.ndarray]    # LIKE result per sampled candidate (None: no LIKE)
+    agg: Optional[dict]            # LIKE: count and matching row ids, when every candidate ran
+
+
+def like_aggregate(match: np.ndarray, cand_rows: np.ndarray) -> dict:
+    """Table 2 Q5: COUNT(*) of the LIKE matches and their row ids (ascending)."""
+    match = np.asarray(match, dtype=bool)
+    return {"count": int(match.sum()), "row_ids": np.asarray(cand_rows)[match].astype(np.int32)}
+
+
+def run_transform(table, prefix, preds, model: tf.Model, n_new: int, eos: int = -1,
+                  pad: int = 0, like: Optional[Sequence[int]] = None,
+                  sample: Optional[np.ndarray] = None) -> TransformResult:
+    """WHERE ``preds``, then greedy AI_TRANSFORM of each candidate's prompt
+    (prefix ++ row tokens), then the optional LIKE '%like%' filter applied to
+    each output's text (the tokens before its eos)."""
+    cand = rel.compact(rel.predicate_mask(table.cols, preds, table.n_rows))
+    n = len(cand)
+    sample = np.arange(n) if sample is None else np.asarray(sample, dtype=np.int64)
+    seqs = prompts(prefix, table.offsets, table.tokens, cand[sample])
+    toks = np.zeros((len(seqs), n_new), dtype=np.int64)
+    lens = np.zeros(len(seqs), dtype=np.int64)
+    for i, q in enumerate(seqs):
+        toks[i], lens[i] = tf.greedy_generate(model, q, n_new, eos, pad)
+    match = None
+    agg = None
+    if like is not None:
+        match = np.array([rel.like_contains(toks[i, :lens[i]], like) for i in range(len(seqs))], dtype=bool)
+        if len(sample) == n and np.array_equal(sample, np.arange(n)):
+            agg = like_aggregate(match, cand)
+    return TransformResult(cand, sample, toks, lens, match, agg)

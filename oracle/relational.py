@@ -169,3 +169,13 @@ def group_build_counts(decision: np.ndarray, cand_build_rows: np.ndarray,
     return (np.array(rows, dtype=np.int32),
             np.array([build_keys[m] for m in rows], dtype=np.int64),
             np.array([counts[m] for m in rows], dtype=np.int64))
+
+
+def like_contains(text: Sequence[int], pattern: Sequence[int]) -> bool:
+    """SQL ``text LIKE '%pattern%'`` on token sequences (Table 2 Q5): true iff
+    ``pattern`` occurs as a contiguous run of ``text``; an empty pattern
+    matches every text, the empty one included."""
+    t, p = list(text), list(pattern)
+    if not p:
+        return True
+    return any(t[i:i + len(p)] == p for i in range(len(t) - len(p) + 1))

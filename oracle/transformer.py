@@ -14,8 +14,9 @@ common Llama-style reading:
   * causal grouped-query attention, scale 1/sqrt(hd), query head h reads
     key/value head h // (H_q / H_kv);
   * SwiGLU MLP W_d(silu(W_g x) * W_u x); no biases except the LM-head bias;
-  * untied LM head; only the label rows of it are ever needed (Fig. 2 slices
-    the last position's logits at the label ids).
+  * untied LM head; AI_IF needs only its label rows (Fig. 2 slices the last
+    position's logits at the label ids), AI_TRANSFORM (Table 1) its full
+    vocabulary for greedy decoding.
 Weights arrive as bf16 bit patterns and are upcast exactly; all arithmetic is
 float64.  Each row is run alone: no packing, no padding.
 """
@@ -143,3 +144,42 @@ def label_logits(m: Model, seqs: List[np.ndarray], labels: Sequence[int]) -> np.
         h = rmsnorm(x[-1], g, m.s.rms_eps)
         out[i] = w_lab @ h + b_lab
     return out
+
+
+def vocab_logits(m: Model, seqs: List[np.ndarray]) -> np.ndarray:
+    """Full-vocabulary logits at every position of one sequence [T, V]:
+    final RMSNorm of each hidden state, times the whole LM head, plus its
+    bias.  Row t is the next-token distribution after seq[:t+1] (causal)."""
+    assert len(seqs) == 1
+    x = hidden_states(m, seqs)[0]
+    h = rmsnorm(x, m.get("final_norm"), m.s.rms_eps)
+    return h @ bf16_to_f64(m.w["lm_head"]).T + bf16_to_f64(m.w["lm_bias"])
+
+
+def first_argmax(z: np.ndarray) -> int:
+    """Index of the largest value; the lowest index among equal maxima."""
+    return int(np.flatnonzero(z == z.max())[0])
+
+
+def greedy_generate(m: Model, prompt: np.ndarray, n_new: int, eos: int = -1,
+                    pad: int = 0):
+    """AI_TRANSFORM (Table 1: causal-LM forward with generative decoding,
+    output masked with a pad id): ``n_new`` greedy steps, each one a full
+    forward over prompt ++ tokens generated so far (no key/value cache) and
+    the first argmax of the last position's vocabulary logits.  Once the
+    model emits ``eos`` the remaining positions hold ``pad``.
+
+    Returns (tokens [n_new] int64, text_len): text_len counts the tokens
+    before the eos (n_new when none was emitted)."""
+    seq = [int(t) for t in prompt]
+    out = np.full(n_new, pad, dtype=np.int64)
+    text_len = n_new
+    for t in range(n_new):
+        z = vocab_logits(m, [np.asarray(seq, dtype=np.int64)])[-1]
+        y = first_argmax(z)
+        out[t] = y
+        if y == eos:
+            text_len = t
+            break
+        seq.append(y)
+    return out, text_len
