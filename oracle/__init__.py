@@ -17,6 +17,10 @@ Parity status per function:
   transformer.greedy_generate  pinned (zero-weight bias closed form, the
                           permutation-head closed form y_t = pi^(t+1)(x), eos/pad)
   relational.like_contains     pinned (delimited-string containment, edge cases)
+  relational.self_join_pairs   pinned (hand-worked fixture, grouped 2-combinations,
+                          sum of C(n_g, 2) closed form)
+  query.run_pair_select   pinned (pair prompt layout, zero-weight bias closed form,
+                          logits equal the concatenated prompt's label logits)
   whole-model numerics at random weights: parity unpinned beyond the
                           component pins (the paper prints no model outputs).
 """

@@ -7,7 +7,9 @@ terms AND AI_IF(text) = 1, then the aggregate.  ``run_transform`` follows
 Table 2 Q3 (SELECT AI_TRANSFORM(text) ... WHERE relational terms: greedy
 generation for every candidate row) and Q5 (COUNT(*) of the rows whose
 generated text is LIKE '%pattern%', with the matching rows' outputs as the
-debug payload).  ``run_join_select`` adds the
+debug payload).  ``run_pair_select`` follows Q4: the selected rows are
+self-joined on a key (A.id = B.id AND A.review_id < B.review_id) and every
+pair gets one AI_IF call on prefix ++ text(A) ++ text(B).  ``run_join_select`` adds the
 reviews-movies equi-join on movie id of Section 4's datasets paragraph, with
 the build-side (movies) predicate, and groups the yes rows by movie.
 
@@ -145,3 +147,42 @@ def run_transform(table, prefix, preds, model: tf.Model, n_new: int, eos: int = 
         if len(sample) == n and np.array_equal(sample, np.arange(n)):
             agg = like_aggregate(match, cand)
     return TransformResult(cand, sample, toks, lens, match, agg)
+
+
+def pair_prompts(prefix: np.ndarray, offsets: np.ndarray, tokens: np.ndarray,
+                 pairs: Sequence[Tuple[int, int]]) -> List[np.ndarray]:
+    """Q4's prompt for a pair: the shared prefix, then A's text, then B's."""
+    return [np.concatenate([prefix, tokens[offsets[a]:offsets[a + 1]],
+                            tokens[offsets[b]:offsets[b + 1]]]).astype(np.int64) for a, b in pairs]
+
+
+@dataclass
+class PairResult:
+    pairs: np.ndarray          # [n_pairs, 2] (a, b), ascending
+    sample: np.ndarray         # pair positions the LM was run on
+    logits: np.ndarray         # [len(sample), K]
+    decision: np.ndarray       # decisions of the sampled pairs
+    agg: Optional[dict]        # COUNT and the yes pairs, when every pair ran
+
+
+def pair_aggregate(decision: np.ndarray, pairs: np.ndarray) -> dict:
+    """COUNT(*) of the pairs decided yes and those pairs, ascending."""
+    yes = np.asarray(decision) == 1
+    return {"count": int(yes.sum()), "yes_pairs": np.asarray(pairs).reshape(-1, 2)[yes]}
+
+
+def run_pair_select(table, key: str, preds, prefix, labels, model: tf.Model,
+                    sample: Optional[np.ndarray] = None) -> PairResult:
+    """WHERE ``preds`` on both sides (the predicate filters the relation before
+    it is joined with itself), the key self-join, then AI_IF per pair."""
+    cand = rel.compact(rel.predicate_mask(table.cols, preds, table.n_rows))
+    pairs = np.array(rel.self_join_pairs(table.cols[key], cand), dtype=np.int64).reshape(-1, 2)
+    n = len(pairs)
+    sample = np.arange(n) if sample is None else np.asarray(sample, dtype=np.int64)
+    seqs = pair_prompts(prefix, table.offsets, table.tokens, [tuple(p) for p in pairs[sample]])
+    logits = tf.label_logits(model, seqs, labels)
+    decision = rel.decide(logits) if len(seqs) else np.zeros(0, np.int32)
+    agg = None
+    if len(sample) == n and np.array_equal(sample, np.arange(n)):
+        agg = pair_aggregate(decision, pairs)
+    return PairResult(pairs, sample, logits, decision, agg)

@@ -15,6 +15,8 @@ Every function restates a passage of the paper:
   * Table 1, SELECT row and Fig. 2: the aggregate is a masked reduction over
     the decision mask (COUNT, the selected ids, or a GROUP BY count).
   * Section 4, datasets paragraph: reviews joined with movies on movie id.
+  * Table 2 Q4: the self-join A.id = B.id AND A.review_id < B.review_id whose
+    row pairs each get one AI_IF call on the concatenated texts.
 """
 from __future__ import annotations
 
@@ -179,3 +181,16 @@ def like_contains(text: Sequence[int], pattern: Sequence[int]) -> bool:
     if not p:
         return True
     return any(t[i:i + len(p)] == p for i in range(len(t) - len(p) + 1))
+
+
+def self_join_pairs(keys: np.ndarray, rows: Sequence[int]) -> List[Tuple[int, int]]:
+    """Table 2 Q4's self-join over the selected rows: every (a, b) with
+    keys[a] == keys[b] and a < b (the row index is the review id), each
+    unordered pair once, in ascending (a, b) order.  Nested loop."""
+    rows = sorted(int(r) for r in rows)
+    out = []
+    for i, a in enumerate(rows):
+        for b in rows[i + 1:]:
+            if keys[a] == keys[b]:
+                out.append((a, b))
+    return out
