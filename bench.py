@@ -55,6 +55,9 @@ def parse():
                    help="relational: predicate + compaction alone on a 2^28-row table, against HBM bandwidth")
     p.add_argument("--micro-rows", type=int, default=1 << 28)
     p.add_argument("--sweep", default="", help="selectivity sweep: 'fixed', 'lognormal' or 'both'")
+    p.add_argument("--transform", type=int, default=0,
+                   help="AI_TRANSFORM: greedy tokens per candidate row (0: the AI_IF query)")
+    p.add_argument("--like", default="", help="AI_TRANSFORM ... LIKE pattern, comma-separated token ids")
     return p.parse_args()
 
 
@@ -421,6 +424,76 @@ def sweep(args):
     ctx.close()
 
 
+def transform_bench(args):
+    """AI_TRANSFORM over the workload's candidate rows (Table 2 Q3; Q5 with
+    --like): greedy decoding of --transform tokens per row after the chunked
+    prefill, everything on the device.  One JSON line with generated tokens/s
+    and the decode kernels' rooflines; not the headline metric."""
+    import torch
+    from paper_2608_10139_gb300 import aiq
+    from paper_2608_10139_gb300 import build as _build
+    _build.build()
+    w = workload(args)
+    q = synth.make_inputs(w)
+    W = synth.make_weights(w.model, w.weight_seed)
+    ctx = aiq.Context(0)
+    model = ctx.load_model(w.model, [W[n] for n, _, _ in synth.weight_specs(w.model)])
+    table = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+    preds = [(p.column, p.op, p.value) for p in w.preds]
+    like = [int(x) for x in args.like.split(",")] if args.like else None
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+
+    def run():
+        return ctx.run_transform(table, model, preds, q.prefix, args.transform, like=like)
+
+    for _ in range(args.warmup):
+        run()
+    clocks = ClockSampler(0)
+    ctx.reset_kernel_stats()
+    ctx.set_option("profile", 1)
+    clocks.start()
+    res = []
+    for _ in range(args.steps):
+        flush.add_(1.0)
+        torch.cuda.synchronize()
+        res.append(run())
+    clk = clocks.stop()
+    ctx.set_option("profile", 0)
+    stats = ctx.kernel_stats()
+    r = res[-1]
+    ms = statistics.median([x.ms_total for x in res])
+    dec_ms = statistics.median([x.ms_decode for x in res])
+    gen_tokens = r.n_candidates * args.transform
+    pk, src = peaks()
+    att = stats.get("decode_attention", {"total_ms": 0, "bytes": 0, "launches": 0})
+    att_gbs = att["bytes"] / (att["total_ms"] / 1000.0) / 1e9 if att["total_ms"] else None
+    dg = [v for k, v in stats.items() if k.startswith("dec_gemm_") or k == "gemm_lm_argmax"]
+    dg_ms = sum(v["total_ms"] for v in dg)
+    dg_tf = sum(v["flops"] for v in dg) / (dg_ms / 1000.0) / 1e12 if dg_ms else None
+    line = {"metric": "AI_TRANSFORM generated tokens/s", "value": gen_tokens / (ms / 1000.0), "unit": "tokens/s",
+            "higher_is_better": True, "steps": args.steps, "warmup": args.warmup, "dtype": "f16xf16->f32",
+            "data": "synthetic",
+            "config": {"workload": w.name, "rows": w.n_rows, "candidates": r.n_candidates,
+                       "max_new_tokens": args.transform, "like": like, "chunks": r.n_chunks},
+            "input_rows_per_s": w.n_rows / (ms / 1000.0), "p50_latency_ms": ms, "decode_ms_p50": dec_ms,
+            "prefill_ms_p50": statistics.median([x.ms_prefill - x.ms_decode for x in res]),
+            "decode_tflops": r.decode_flops / (dec_ms / 1000.0) / 1e12 if dec_ms else None,
+            "like_count": r.count,
+            "kernel_ms_per_step": {k: round(v["total_ms"] / args.steps, 3) for k, v in sorted(stats.items())},
+            "roofline": {
+                "decode_attention": {"bound": "hbm", "achieved": att_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                                     "frac": att_gbs / pk["hbm_gbs"] if att_gbs else None,
+                                     "launches": att["launches"], "peak_source": f"{src} hbm_gbs"},
+                "decode_gemms": {"bound": "tensor", "achieved": dg_tf,
+                                 "peak": pk.get("bf16_tflops_sustained", pk["bf16_tflops"]), "unit": "TFLOP/s",
+                                 "frac": dg_tf / pk.get("bf16_tflops_sustained", pk["bf16_tflops"]) if dg_tf else None,
+                                 "peak_source": f"{src} bf16_tflops_sustained"}},
+            "clocks": clk}
+    print(json.dumps(line), flush=True)
+    ctx.free_table(table)
+    ctx.close()
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -429,6 +502,8 @@ def main():
         micro_relational(args)
     elif args.sweep:
         sweep(args)
+    elif args.transform:
+        transform_bench(args)
     else:
         ours(args)
 

@@ -128,6 +128,15 @@ typedef struct {
   double prefill_flops; /* executed: 2*params per token + 4*Hq*hd*L per causal pair + head */
   int64_t n_launches;   /* CUDA kernels this query launched */
   int64_t n_prefill_tokens; /* tokens run through the decoder: the shared prefix once + every row's text */
+  /* aiq_run_transform only (zero / NULL otherwise) */
+  int32_t gen_max_new;        /* columns of gen_tokens: the generate spec's max_new_tokens */
+  int64_t n_gen_rows;         /* rows of gen_tokens */
+  const int32_t* gen_row_ids; /* [n_gen_rows] ascending table rows */
+  const int32_t* gen_tokens;  /* [n_gen_rows, gen_max_new]: greedy tokens, the eos, then pad_id */
+  const int32_t* gen_text_len; /* [n_gen_rows]: generated tokens before the eos (max_new without one) */
+  float ms_decode;            /* device time of the decode steps (inside ms_prefill) */
+  double decode_flops;        /* 2*params per decoded token + attention over cached keys + full LM head */
+  int64_t n_decode_steps;     /* sum over prefill chunks of max_new_tokens */
 } aiq_result_view;
 
 typedef struct aiq_ctx aiq_ctx;
@@ -175,6 +184,39 @@ aiq_status aiq_run_select(aiq_ctx* ctx, aiq_table table, aiq_model model, const 
 aiq_status aiq_run_join_select(aiq_ctx* ctx, aiq_table build, int32_t build_key, const aiq_pred* build_preds,
                                int32_t n_build_preds, aiq_table probe, int32_t probe_key, aiq_model model,
                                const aiq_select* probe_side, aiq_result_h* out);
+
+/* AI_TRANSFORM (Table 1: causal-LM forward with generative decoding, output
+ * masked with a pad id; Table 2 Q3 and Q5).  Greedy decoding: every step
+ * appends the first index of the largest full-vocabulary logit (final RMSNorm,
+ * LM head, bias) at the row's last position.  After a row emits eos_id, its
+ * remaining positions hold pad_id; eos_id < 0 disables the stop.
+ * like_len > 0 adds Q5's filter: a row matches when the pattern occurs as a
+ * contiguous run of its generated tokens before the eos (SQL LIKE '%...%' on
+ * token ids); like_len == 0 with a non-NULL like_tokens matches every row. */
+typedef struct {
+  int32_t max_new_tokens;     /* 1..4096 */
+  int32_t eos_id;             /* -1: none */
+  int32_t pad_id;
+  const int32_t* like_tokens; /* host; NULL: no LIKE filter (Q3 form) */
+  int32_t like_len;           /* 0..256 */
+  int32_t flags;              /* AIQ_GEN_* */
+} aiq_generate;
+
+enum {
+  AIQ_GEN_MATCH_TOKENS = 1 /* with LIKE: also return the matching rows' tokens (the "debug outputs") */
+};
+
+/* Table 2 Q3: SELECT AI_TRANSFORM(text, prefix) FROM table WHERE <preds>:
+ *   gen_row_ids = the candidate rows, gen_tokens / gen_text_len per row, count = -1.
+ * Table 2 Q5: SELECT COUNT(*) ... WHERE <preds> AND AI_TRANSFORM(...) LIKE '%p%':
+ *   count = matching rows, row_ids = their ids; with AIQ_GEN_MATCH_TOKENS the
+ *   gen_* arrays hold the matching rows only.
+ * Uses q's preds, text_column and prefix; its labels, agg and flags are ignored.
+ * Token ids of the prefix and the rows must be < vocab; pad_id and eos_id too
+ * (when set).  The whole generation runs on the device: only the results
+ * cross PCIe. */
+aiq_status aiq_run_transform(aiq_ctx* ctx, aiq_table table, aiq_model model, const aiq_select* q,
+                             const aiq_generate* gen, aiq_result_h* out);
 
 aiq_status aiq_result(aiq_ctx* ctx, aiq_result_h result, aiq_result_view* out);
 aiq_status aiq_result_free(aiq_ctx* ctx, aiq_result_h result);

@@ -60,6 +60,21 @@ aiq_status aiq_op_rmsnorm(aiq_ctx* ctx, const float* x, int64_t T, int32_t d, co
 aiq_status aiq_op_attention(aiq_ctx* ctx, const void* qkv, int64_t T, const int32_t* seq_start, int32_t n_seqs,
                             int32_t Hq, int32_t Hkv, int32_t hd, const void* prefix_kv, int32_t P, void* out);
 
+/* One decode step of causal grouped-query attention (AI_TRANSFORM, Table 1:
+ * generative decoding; each row attends every earlier token of its own
+ * sequence).  R rows, one new token each: qkv fp16 [R, (Hq + 2 Hkv) * hd]
+ * (rotary embeddings applied).  Row r's keys/values, every cache fp16 with
+ * rows of [2 Hkv hd] (keys, then values):
+ *   prefix_kv [P] shared by every row (may be NULL when P == 0);
+ *   own_kv rows [seq_start[r], seq_start[r+1]) (seq_start int32 [R + 1], device);
+ *   gen_kv [R, gen_cap] slots 0 .. slot of row r, where slot `slot` first
+ *   receives this step's key and value (written by the call).
+ * out fp16 [R, Hq * hd].  hd in {32, 64, 128}, Hq / Hkv <= 8.  All pointers are
+ * device memory owned by the caller; the call synchronises its stream. */
+aiq_status aiq_op_decode_attention(aiq_ctx* ctx, const void* qkv, int32_t R, int32_t Hq, int32_t Hkv, int32_t hd,
+                                   const void* prefix_kv, int32_t P, const void* own_kv, const int32_t* seq_start,
+                                   void* gen_kv, int32_t gen_cap, int32_t slot, void* out);
+
 /* One relational term for aiq_filter_compact_static: `column op constant` on a
  * caller-owned device column of n_rows values (16-byte aligned).  INT32 and
  * INT64 columns compare with `ivalue`, FLOAT32 columns with `fvalue`. */

@@ -22,6 +22,7 @@ INT32, INT64, FLOAT32, TOKENS = 0, 1, 2, 3
 LT, LE, GT, GE, EQ, NE = 0, 1, 2, 3, 4, 5
 AGG_COUNT, AGG_ROW_IDS, AGG_GROUP_LABEL, AGG_GROUP_BUILD_KEY = 0, 1, 2, 3
 FLAG_LOGITS, FLAG_RELATIONAL_ONLY = 1, 2
+GEN_MATCH_TOKENS = 1
 EPI_F16, EPI_ROPE_F16, EPI_RESID_F32, EPI_SWIGLU_F16 = 0, 1, 2, 3
 
 
@@ -63,7 +64,15 @@ class _View(C.Structure):
                 ("label_logits", C.POINTER(C.c_float)), ("decisions", C.POINTER(C.c_int32)),
                 ("ms_relational", C.c_float), ("ms_prefill", C.c_float), ("ms_aggregate", C.c_float),
                 ("ms_total", C.c_float), ("prefill_flops", C.c_double), ("n_launches", C.c_int64),
-                ("n_prefill_tokens", C.c_int64)]
+                ("n_prefill_tokens", C.c_int64),
+                ("gen_max_new", C.c_int32), ("n_gen_rows", C.c_int64), ("gen_row_ids", C.POINTER(C.c_int32)),
+                ("gen_tokens", C.POINTER(C.c_int32)), ("gen_text_len", C.POINTER(C.c_int32)),
+                ("ms_decode", C.c_float), ("decode_flops", C.c_double), ("n_decode_steps", C.c_int64)]
+
+
+class _Generate(C.Structure):
+    _fields_ = [("max_new_tokens", C.c_int32), ("eos_id", C.c_int32), ("pad_id", C.c_int32),
+                ("like_tokens", C.POINTER(C.c_int32)), ("like_len", C.c_int32), ("flags", C.c_int32)]
 
 
 class _Term(C.Structure):
@@ -89,6 +98,8 @@ _SIGS = {
     "aiq_run_select": [C.c_void_p, C.c_int64, C.c_int64, C.POINTER(_Select), C.POINTER(C.c_int64)],
     "aiq_run_join_select": [C.c_void_p, C.c_int64, C.c_int32, C.POINTER(_Pred), C.c_int32, C.c_int64, C.c_int32,
                             C.c_int64, C.POINTER(_Select), C.POINTER(C.c_int64)],
+    "aiq_run_transform": [C.c_void_p, C.c_int64, C.c_int64, C.POINTER(_Select), C.POINTER(_Generate),
+                          C.POINTER(C.c_int64)],
     "aiq_result": [C.c_void_p, C.c_int64, C.POINTER(_View)],
     "aiq_result_free": [C.c_void_p, C.c_int64],
     "aiq_last_error": [],
@@ -103,6 +114,8 @@ _SIGS = {
     "aiq_op_rmsnorm": [C.c_void_p, C.c_void_p, C.c_int64, C.c_int32, C.c_void_p, C.c_float, C.c_void_p],
     "aiq_op_attention": [C.c_void_p, C.c_void_p, C.c_int64, C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32,
                          C.c_void_p, C.c_int32, C.c_void_p],
+    "aiq_op_decode_attention": [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_void_p,
+                                C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p],
     "aiq_filter_compact_static": [C.POINTER(_Term), C.c_int32, C.c_int64, C.c_void_p, C.c_void_p, C.c_void_p],
 }
 
@@ -182,6 +195,27 @@ class Result:
     prefill_flops: float
     n_launches: int
     n_prefill_tokens: int
+
+
+@dataclass
+class TransformResult:
+    n_input_rows: int
+    n_candidates: int
+    count: int                 # LIKE matches (-1 without LIKE)
+    row_ids: np.ndarray        # LIKE: matching rows, ascending
+    gen_row_ids: np.ndarray    # rows of gen_tokens
+    gen_tokens: np.ndarray     # [n_gen_rows, max_new]
+    gen_text_len: np.ndarray   # [n_gen_rows]
+    ms_relational: float
+    ms_prefill: float          # prefill and decode
+    ms_decode: float
+    ms_aggregate: float
+    ms_total: float
+    prefill_flops: float
+    decode_flops: float
+    n_decode_steps: int
+    n_launches: int
+    n_chunks: int
 
 
 def _arr(ptr, n, dtype, shape=None):
@@ -322,6 +356,33 @@ class Context:
                                             probe.col(probe_key), model, C.byref(sel), C.byref(h)))
         return self._fetch(h, len(labels))
 
+    def run_transform(self, table: TableRef, model: int, preds, prefix, max_new: int, eos: int = -1,
+                      pad: int = 0, like=None, match_tokens: bool = False,
+                      text_name: str = "text") -> TransformResult:
+        """AI_TRANSFORM (greedy) of every candidate row; with ``like`` (a token
+        sequence) only the COUNT / ids of the rows whose output contains it."""
+        sel, keep = self._select(table, preds, prefix, [], AGG_COUNT, 0, text_name)
+        pat = _i32(like if like is not None else [])
+        buf = pat if pat.size else np.zeros(1, np.int32)   # a non-NULL pointer for the empty pattern
+        g = _Generate(max_new, eos, pad,
+                      buf.ctypes.data_as(C.POINTER(C.c_int32)) if like is not None else None,
+                      len(pat), GEN_MATCH_TOKENS if match_tokens else 0)
+        h = C.c_int64()
+        _check(self.lib.aiq_run_transform(self.h, table.handle, model, C.byref(sel), C.byref(g), C.byref(h)))
+        v = _View()
+        try:
+            _check(self.lib.aiq_result(self.h, h, C.byref(v)))
+            n, w = v.n_gen_rows, v.gen_max_new
+            return TransformResult(
+                v.n_input_rows, v.n_candidates, v.count, _arr(v.row_ids, v.n_row_ids, np.int32),
+                _arr(v.gen_row_ids, n, np.int32),
+                _arr(v.gen_tokens, n * w, np.int32, (n, w)) if n else np.zeros((0, w), np.int32),
+                _arr(v.gen_text_len, n, np.int32),
+                v.ms_relational, v.ms_prefill, v.ms_decode, v.ms_aggregate, v.ms_total, v.prefill_flops,
+                v.decode_flops, v.n_decode_steps, v.n_launches, v.n_chunks)
+        finally:
+            self.lib.aiq_result_free(self.h, h)
+
     # -------------------------------------------------------------- options
     def set_option(self, name: str, value: int):
         _check(self.lib.aiq_set_option(self.h, name.encode(), int(value)))
@@ -355,3 +416,8 @@ class Context:
     def op_attention(self, qkv: int, T: int, seq_start: int, n_seqs: int, Hq: int, Hkv: int, hd: int, out: int,
                      prefix_kv: int = 0, P: int = 0):
         _check(self.lib.aiq_op_attention(self.h, qkv, T, seq_start, n_seqs, Hq, Hkv, hd, prefix_kv or None, P, out))
+
+    def op_decode_attention(self, qkv: int, R: int, Hq: int, Hkv: int, hd: int, own_kv: int, seq_start: int,
+                            gen_kv: int, gen_cap: int, slot: int, out: int, prefix_kv: int = 0, P: int = 0):
+        _check(self.lib.aiq_op_decode_attention(self.h, qkv, R, Hq, Hkv, hd, prefix_kv or None, P, own_kv, seq_start,
+                                                gen_kv, gen_cap, slot, out))

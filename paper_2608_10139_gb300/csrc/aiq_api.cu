@@ -87,6 +87,11 @@ struct ModelD {
   DevBuf rope_cos, rope_sin;
   int rope_max_pos = 0;
   double linear_flops_per_token = 0;
+  // full-vocabulary LM head for generation, made on first use: fp16 [vpad, d]
+  // (zero rows past the vocabulary) and an fp32 bias with -inf past it
+  __half* lm_f16 = nullptr;
+  float* lm_bias_f32 = nullptr;
+  int vpad = 0;
 };
 
 struct ResultH {
@@ -94,6 +99,8 @@ struct ResultH {
   std::vector<int32_t> row_ids, group_rows, cand_ids, cand_build, decisions;
   std::vector<int64_t> group_keys, group_counts, label_counts;
   std::vector<float> logits;
+  std::vector<int32_t> gen_ids, gen_tok, gen_len;
+  int32_t gen_max_new = 0;
 };
 
 struct ProfRec {
@@ -549,16 +556,179 @@ struct QueryState {
   int64_t P = 0;                            // prefix tokens, run once
 };
 
-aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_select* q, QueryState* st) {
+// Generation state of an AI_TRANSFORM query (Table 1): greedy decoding of
+// every candidate row after its chunk's prefill.
+struct GenPlan {
+  int max_new = 0, eos = -1, pad = 0;
+  int32_t* tok = nullptr;  // [S, max_new] generated tokens (device)
+  int32_t* len = nullptr;  // [S] tokens before the eos (device)
+  std::vector<std::pair<cudaEvent_t, cudaEvent_t>> spans;  // decode time per chunk
+  double flops = 0;
+  int64_t steps = 0;
+};
+
+// Full-vocabulary LM head in the GEMM's operand format, made once per model.
+aiq_status ensure_lm_f16(aiq_ctx* c, ModelD& m) {
+  if (m.lm_f16) return AIQ_OK;
+  const aiq_model_config& g = m.cfg;
+  const int vpad = (g.vocab + 255) / 256 * 256;
+  __half* w = nullptr;
+  float* b = nullptr;
+  void* p = nullptr;
+  AIQ_TRY(dalloc(c, &p, static_cast<size_t>(vpad) * g.d_model * sizeof(__half)));
+  w = static_cast<__half*>(p);
+  m.allocs.push_back(DevBuf{p, std::max<size_t>(static_cast<size_t>(vpad) * g.d_model * sizeof(__half), 256)});
+  AIQ_TRY(dalloc(c, &p, static_cast<size_t>(vpad) * sizeof(float)));
+  b = static_cast<float*>(p);
+  m.allocs.push_back(DevBuf{p, std::max<size_t>(static_cast<size_t>(vpad) * sizeof(float), 256)});
+  CUDA_TRY(cudaMemsetAsync(w, 0, static_cast<size_t>(vpad) * g.d_model * sizeof(__half), c->stream));
+  launch_bf16_to_f16(m.lm_head, w, g.vocab, g.d_model, 0, 0, nullptr, c->d_err, c->stream);
+  launch_bias_f32(m.lm_bias, g.vocab, vpad, b, c->stream);
+  counted(c, 2);
+  AIQ_TRY(sync_and_check(c));
+  m.lm_f16 = w;
+  m.lm_bias_f32 = b;
+  m.vpad = vpad;
+  return AIQ_OK;
+}
+
+struct DecodeBufs {
+  __half *kvc, *gkv;  // [L][Tc][2 kd] prompt keys/values of the chunk; [L][R][gcap][2 kd] generated ones
+  int gcap;
+  unsigned long long* best;
+  int32_t *done, *next, *pos;
+};
+
+// Greedy tokens of the LM head for R rows of normalised hidden states in b.xn.
+aiq_status lm_argmax_select(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const DecodeBufs& d, int R, int t,
+                            GenPlan* gp, int64_t r0, int P) {
+  GemmEpilogue e;
+  e.kind = EPI_ARGMAX;
+  e.bias = m.lm_bias_f32;
+  e.best = d.best;
+  e.err = c->d_err;
+  AIQ_TRY(gemm(c, "gemm_lm_argmax", b.xn, m.cfg.d_model, m.lm_f16, m.cfg.d_model, R, m.vpad, m.cfg.d_model, 256, e));
+  ProfScope p(c, "decode_select", 0, 0);
+  launch_decode_select(d.best, R, t, gp->max_new, gp->eos, gp->pad, m.cfg.vocab, d.done,
+                       gp->tok + r0 * gp->max_new, gp->len + r0, d.next, d.pos, b.seq_start, P, c->d_err, c->stream);
+  counted(c, 1);
+  return AIQ_OK;
+}
+
+// One decoder pass over R single-token rows (each row's newest token, at its
+// own position), keys/values appended to generated slot `slot`.
+aiq_status decode_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const DecodeBufs& d, int R, int64_t Tc,
+                         const __half* pkv, int P, int slot) {
+  const aiq_model_config& g = m.cfg;
+  const int dm = g.d_model, hd = g.head_dim, Hq = g.n_heads, Hkv = g.n_kv_heads, f = g.d_ffn;
+  const int nqkv = (Hq + 2 * Hkv) * hd;
+  const int64_t ldkv = 2 * static_cast<int64_t>(Hkv) * hd;
+  const int parts = dm / 128;
+  {
+    ProfScope p(c, "embed", 0, 0);
+    launch_embed(d.next, R, m.embed, dm, b.resid, b.xn, b.ss_attn, c->d_err, c->stream);
+    counted(c, 1);
+  }
+  for (int l = 0; l < g.n_layers; ++l) {
+    const LayerD& L = m.layers[l];
+    GemmEpilogue e1;
+    e1.kind = EPI_ROPE_F16;
+    e1.out = b.qkv;
+    e1.ldo = nqkv;
+    e1.positions = d.pos;
+    e1.rope_cos = static_cast<const float*>(m.rope_cos.p);
+    e1.rope_sin = static_cast<const float*>(m.rope_sin.p);
+    e1.rope_cols = (Hq + Hkv) * hd;
+    e1.head_dim = hd;
+    e1.err = c->d_err;
+    e1.row_ss = b.ss_attn;
+    e1.ss_parts = parts;
+    e1.d_norm = static_cast<float>(dm);
+    e1.eps = g.rms_eps;
+    AIQ_TRY(gemm(c, "dec_gemm_qkv_rope", b.xn, dm, L.wqkv, dm, R, nqkv, dm, m.bn_qkv, e1));
+    {
+      // keys read per row: P + len + slot + 1; summed over the rows: R (P + slot + 1) + Tc
+      const double keys = double(R) * (P + slot + 1) + double(Tc);
+      ProfScope p(c, "decode_attention", 4.0 * Hq * hd * keys,
+                  keys * ldkv * 2.0 + double(R) * (nqkv + Hq * hd + ldkv) * 2.0);
+      const int e = launch_decode_attention(b.qkv, nqkv, R, Hq, Hkv, hd, pkv ? pkv + l * P * ldkv : nullptr, P,
+                                            d.kvc + l * Tc * ldkv, b.seq_start,
+                                            d.gkv + static_cast<int64_t>(l) * R * d.gcap * ldkv, d.gcap, slot, b.att,
+                                            c->d_err, c->stream);
+      counted(c, 1);
+      if (e != 0)
+        return fail(AIQ_ERR_CUDA, std::string("decode attention launch: ") +
+                                      cudaGetErrorString(static_cast<cudaError_t>(e)));
+    }
+    GemmEpilogue e2;
+    e2.kind = EPI_RESID_F32;
+    e2.out = b.resid;
+    e2.ldo = dm;
+    e2.err = c->d_err;
+    e2.ss_parts = parts;
+    AIQ_TRY(gemm(c, "dec_gemm_o_resid", b.att, Hq * hd, L.wo, Hq * hd, R, dm, Hq * hd, m.bn_o, e2));
+    {
+      ProfScope p(c, "rmsnorm", 0, 0);
+      launch_rmsnorm(b.resid, R, dm, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+      counted(c, 1);
+    }
+    GemmEpilogue e3;
+    e3.kind = EPI_SWIGLU_F16;
+    e3.out = b.act;
+    e3.ldo = f;
+    e3.err = c->d_err;
+    AIQ_TRY(gemm(c, "dec_gemm_gateup_swiglu", b.xn, dm, L.wgu, dm, R, 2 * f, dm, m.bn_gu, e3));
+    e2.xh_out = b.xn;
+    e2.ss_out = b.ss_attn;
+    AIQ_TRY(gemm(c, "dec_gemm_down_resid", b.act, f, L.wd, f, R, dm, f, m.bn_d, e2));
+  }
+  return AIQ_OK;
+}
+
+// max_new greedy steps for the R rows of one chunk whose prefill just ran
+// (final hidden state of each row's last prompt token in b.resid_last).
+aiq_status decode_chunk(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const DecodeBufs& d, int R, int64_t Tc,
+                        const __half* pkv, int P, const float* prefix_last, int64_t r0, GenPlan* gp) {
+  const aiq_model_config& g = m.cfg;
+  launch_patch_empty_rows(b.resid_last, b.last_compact, prefix_last, R, g.d_model, c->stream);
+  {
+    ProfScope p(c, "rmsnorm", 0, 0);
+    launch_rmsnorm(b.resid_last, R, g.d_model, m.final_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+    counted(c, 2);
+  }
+  AIQ_TRY(lm_argmax_select(c, m, b, d, R, 0, gp, r0, P));
+  for (int t = 1; t < gp->max_new; ++t) {
+    AIQ_TRY(decode_layers(c, m, b, d, R, Tc, pkv, P, t - 1));
+    {
+      ProfScope p(c, "rmsnorm", 0, 0);
+      launch_rmsnorm(b.resid, R, g.d_model, m.final_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+      counted(c, 1);
+    }
+    AIQ_TRY(lm_argmax_select(c, m, b, d, R, t, gp, r0, P));
+  }
+  // executed FLOPs: full LM head every step; decoder passes with attention over
+  // P + len + t keys per row (sum over rows: R (P + t) + Tc)
+  const double hq_hd = double(g.n_heads) * g.head_dim;
+  gp->flops += double(gp->max_new) * 2.0 * g.d_model * m.vpad * R;
+  for (int t = 1; t < gp->max_new; ++t)
+    gp->flops += m.linear_flops_per_token * R + 4.0 * hq_hd * g.n_layers * (double(R) * (P + t) + double(Tc));
+  gp->steps += gp->max_new;
+  return AIQ_OK;
+}
+
+aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_select* q, QueryState* st,
+                         GenPlan* gp = nullptr) {
   const ColD& col = t.cols[q->text_column];
-  const int K = q->n_labels;
+  const int K = gp ? 0 : q->n_labels;
   const int64_t S = st->S;
   const int32_t P = q->prefix_len;
-  float* logits;
-  AIQ_TRY(ws(c, "q.logits", std::max<int64_t>(S * K, 1), &logits));
-  st->logits = logits;
+  float* logits = nullptr;
+  if (!gp) {
+    AIQ_TRY(ws(c, "q.logits", std::max<int64_t>(S * K, 1), &logits));
+    st->logits = logits;
+  }
   if (S == 0) return AIQ_OK;
-  int32_t *lens, *prefix_d, *labels_d;
+  int32_t *lens, *prefix_d, *labels_d = nullptr;
   int64_t *cu, *scan_scratch;
   unsigned long long* pairs_d;
   AIQ_TRY(ws(c, "q.lens", S, &lens));
@@ -566,9 +736,11 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
   AIQ_TRY(ws(c, "q.scan", 2 * (S / kRowsPerBlock + 2), &scan_scratch));
   AIQ_TRY(ws(c, "q.pairs", 1, &pairs_d));
   AIQ_TRY(ws(c, "q.prefix", std::max<int32_t>(P, 1), &prefix_d));
-  AIQ_TRY(ws(c, "q.labels", K, &labels_d));
   if (P > 0) CUDA_TRY(cudaMemcpyAsync(prefix_d, q->prefix, P * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
-  CUDA_TRY(cudaMemcpyAsync(labels_d, q->label_ids, K * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
+  if (K > 0) {
+    AIQ_TRY(ws(c, "q.labels", K, &labels_d));
+    CUDA_TRY(cudaMemcpyAsync(labels_d, q->label_ids, K * sizeof(int32_t), cudaMemcpyHostToDevice, c->stream));
+  }
   CUDA_TRY(cudaMemsetAsync(pairs_d, 0, sizeof(unsigned long long), c->stream));
   {
     ProfScope p(c, "pack_plan", 0, 0);
@@ -599,16 +771,29 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
     Bmax = std::max(Bmax, chunks[2 * (i + 1) + 1] - chunks[2 * i + 1]);
     Rmax = std::max(Rmax, chunks[2 * (i + 1)] - chunks[2 * i]);
   }
-  AIQ_TRY(ensure_rope(c, m, static_cast<int>(P + max_len)));
+  AIQ_TRY(ensure_rope(c, m, static_cast<int>(P + max_len + (gp ? gp->max_new : 0))));
   PrefillBufs pb;
   AIQ_TRY(prefill_bufs(c, m, std::max<int64_t>(Bmax, 64), Rmax, &pb));
   const aiq_model_config& g = m.cfg;
+  const int64_t ldkv = 2 * static_cast<int64_t>(g.n_kv_heads) * g.head_dim;
+  DecodeBufs db{};
+  if (gp) {
+    AIQ_TRY(ensure_lm_f16(c, m));
+    db.gcap = std::max(gp->max_new - 1, 1);
+    AIQ_TRY(ws(c, "g.kvc", static_cast<int64_t>(g.n_layers) * std::max<int64_t>(Bmax, 1) * ldkv, &db.kvc));
+    AIQ_TRY(ws(c, "g.gkv", static_cast<int64_t>(g.n_layers) * Rmax * db.gcap * ldkv, &db.gkv));
+    AIQ_TRY(ws(c, "g.best", Rmax, &db.best));
+    AIQ_TRY(ws(c, "g.done", Rmax, &db.done));
+    AIQ_TRY(ws(c, "g.next", Rmax, &db.next));
+    AIQ_TRY(ws(c, "g.pos", Rmax, &db.pos));
+    CUDA_TRY(cudaMemsetAsync(db.best, 0, Rmax * sizeof(unsigned long long), c->stream));
+  }
   __half* pkv = nullptr;
   float* prefix_last;
   AIQ_TRY(ws(c, "pf.prefix_last", g.d_model, &prefix_last));
   if (P > 0) {
     // the shared prefix once: its per-layer keys/values and its last hidden state
-    AIQ_TRY(ws(c, "pf.prefix_kv", static_cast<int64_t>(g.n_layers) * P * 2 * g.n_kv_heads * g.head_dim, &pkv));
+    AIQ_TRY(ws(c, "pf.prefix_kv", static_cast<int64_t>(g.n_layers) * P * ldkv, &pkv));
     launch_pack_prefix(prefix_d, P, pb.tok, pb.pos, pb.seq_start, c->stream);
     counted(c, 1);
     AIQ_TRY(run_layers(c, m, pb, P, 1, nullptr, 0, pkv, false));
@@ -625,8 +810,15 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
                         pb.seq_start, pb.last_idx, c->stream);
       counted(c, 1);
     }
-    AIQ_TRY(run_layers(c, m, pb, Tc, r1 - r0, pkv, static_cast<int>(P), nullptr, true));
-    {
+    // generation keeps every layer's prompt keys/values of the chunk for the decode steps
+    AIQ_TRY(run_layers(c, m, pb, Tc, r1 - r0, pkv, static_cast<int>(P), gp ? db.kvc : nullptr, true));
+    if (gp) {
+      cudaEvent_t e0 = take_event(c), e1 = take_event(c);
+      CUDA_TRY(cudaEventRecord(e0, c->stream));
+      AIQ_TRY(decode_chunk(c, m, pb, db, static_cast<int>(r1 - r0), Tc, pkv, P, prefix_last, r0, gp));
+      CUDA_TRY(cudaEventRecord(e1, c->stream));
+      gp->spans.push_back({e0, e1});
+    } else {
       ProfScope p(c, "label_head", 0, 0);
       launch_label_head(pb.resid_last, pb.last_compact, prefix_last, r1 - r0, g.d_model, m.final_norm, g.rms_eps,
                         m.lm_head, m.lm_bias, labels_d, K, logits + r0 * K, c->stream);
@@ -742,13 +934,16 @@ void finish_view(ResultH& R, const QueryState& st, int64_t n_input, int K, int a
   v.cand_build_rows = R.cand_build.empty() ? nullptr : R.cand_build.data();
   v.label_logits = R.logits.empty() ? nullptr : R.logits.data();
   v.decisions = R.decisions.empty() ? nullptr : R.decisions.data();
+  v.gen_max_new = R.gen_max_new;
+  v.n_gen_rows = static_cast<int64_t>(R.gen_ids.size());
+  v.gen_row_ids = R.gen_ids.empty() ? nullptr : R.gen_ids.data();
+  v.gen_tokens = R.gen_tok.empty() ? nullptr : R.gen_tok.data();
+  v.gen_text_len = R.gen_len.empty() ? nullptr : R.gen_len.data();
   (void)agg;
 }
 
-aiq_status validate_select(aiq_ctx* c, const TableD& t, const ModelD* m, const aiq_select* q) {
-  if (!q) return fail(AIQ_ERR_INVALID_ARG, "select is NULL");
-  const bool rel_only = q->flags & AIQ_FLAG_RELATIONAL_ONLY;
-  if (rel_only) return AIQ_OK;
+// The prompt half of a query: text column, token ids, prefix, length limits.
+aiq_status validate_prompt(const TableD& t, const ModelD* m, const aiq_select* q, int64_t extra_positions) {
   if (!m) return fail(AIQ_ERR_NOT_FOUND, "unknown model handle");
   if (q->text_column < 0 || q->text_column >= static_cast<int32_t>(t.cols.size()) ||
       t.cols[q->text_column].type != AIQ_TOKENS)
@@ -758,6 +953,19 @@ aiq_status validate_select(aiq_ctx* c, const TableD& t, const ModelD* m, const a
   if (q->prefix_len < 0 || (q->prefix_len > 0 && !q->prefix)) return fail(AIQ_ERR_INVALID_ARG, "bad prefix");
   for (int i = 0; i < q->prefix_len; ++i)
     if (q->prefix[i] < 0 || q->prefix[i] >= V) return fail(AIQ_ERR_INVALID_ARG, "prefix token id out of range");
+  if (q->prefix_len == 0 && t.cols[q->text_column].min_len == 0)
+    return fail(AIQ_ERR_INVALID_ARG, "a row with empty text needs a non-empty prefix (its prompt would be empty)");
+  if (q->prefix_len + t.cols[q->text_column].max_len + extra_positions > (1 << 20))
+    return fail(AIQ_ERR_UNSUPPORTED, "a prompt is longer than 2^20 tokens");
+  return AIQ_OK;
+}
+
+aiq_status validate_select(aiq_ctx* c, const TableD& t, const ModelD* m, const aiq_select* q) {
+  if (!q) return fail(AIQ_ERR_INVALID_ARG, "select is NULL");
+  const bool rel_only = q->flags & AIQ_FLAG_RELATIONAL_ONLY;
+  if (rel_only) return AIQ_OK;
+  AIQ_TRY(validate_prompt(t, m, q, 0));
+  const int V = m->cfg.vocab;
   if (q->n_labels < 2 || q->n_labels > 16 || !q->label_ids) return fail(AIQ_ERR_INVALID_ARG, "n_labels must be 2..16");
   for (int i = 0; i < q->n_labels; ++i)
     if (q->label_ids[i] < 0 || q->label_ids[i] >= V) return fail(AIQ_ERR_INVALID_ARG, "label id out of range");
@@ -766,10 +974,6 @@ aiq_status validate_select(aiq_ctx* c, const TableD& t, const ModelD* m, const a
     return fail(AIQ_ERR_INVALID_ARG, "COUNT / ROW_IDS need exactly 2 labels (yes, no)");
   if (q->agg == AIQ_AGG_GROUP_BUILD_KEY && q->n_labels != 2)
     return fail(AIQ_ERR_INVALID_ARG, "GROUP_BUILD_KEY needs exactly 2 labels (yes, no)");
-  const int64_t max_len = q->prefix_len + t.cols[q->text_column].max_len;
-  if (q->prefix_len == 0 && t.cols[q->text_column].min_len == 0)
-    return fail(AIQ_ERR_INVALID_ARG, "a row with empty text needs a non-empty prefix (its prompt would be empty)");
-  if (max_len > (1 << 20)) return fail(AIQ_ERR_UNSUPPORTED, "a prompt is longer than 2^20 tokens");
   (void)c;
   return AIQ_OK;
 }
@@ -869,6 +1073,138 @@ aiq_status run_query(aiq_ctx* c, const TableD* build, int32_t build_key, const a
   dst.v.ms_aggregate = t23;
   dst.v.ms_total = t03;
   if (!rel_only && m) dst.v.prefill_flops = R.v.prefill_flops;
+  dst.v.n_launches = c->launches;
+  return AIQ_OK;
+}
+
+// Table 2 Q3 / Q5: relational phase, prefill + greedy decoding per chunk,
+// then the LIKE filter and the result arrays.
+aiq_status run_transform(aiq_ctx* c, const TableD& t, ModelD* m, const aiq_select* q, const aiq_generate* gen,
+                         aiq_result_h* out) {
+  AIQ_TRY(validate_prompt(t, m, q, gen->max_new_tokens));
+  const int V = m->cfg.vocab;
+  if (gen->max_new_tokens < 1 || gen->max_new_tokens > 4096)
+    return fail(AIQ_ERR_INVALID_ARG, "max_new_tokens must be 1..4096");
+  if (gen->eos_id < -1 || gen->eos_id >= V) return fail(AIQ_ERR_INVALID_ARG, "eos_id must be -1 or a token id");
+  if (gen->pad_id < 0 || gen->pad_id >= V) return fail(AIQ_ERR_INVALID_ARG, "pad_id must be a token id");
+  const bool like = gen->like_tokens != nullptr;
+  if (like && (gen->like_len < 0 || gen->like_len > 256)) return fail(AIQ_ERR_INVALID_ARG, "like_len must be 0..256");
+  for (int i = 0; like && i < gen->like_len; ++i)
+    if (gen->like_tokens[i] < 0 || gen->like_tokens[i] >= V)
+      return fail(AIQ_ERR_INVALID_ARG, "LIKE pattern token id out of range");
+  PredSet ps{};
+  AIQ_TRY(make_pred_set(t, q->preds, q->n_preds, &ps));
+
+  c->launches = 0;
+  cudaEvent_t ev[4];
+  for (auto& e : ev) e = take_event(c);
+  CUDA_TRY(cudaEventRecord(ev[0], c->stream));
+  QueryState st;
+  AIQ_TRY(filter_compact(c, t, ps, ProbeSpec{}, "sel", &st.S, &st.ids, nullptr));
+  CUDA_TRY(cudaEventRecord(ev[1], c->stream));
+  const int64_t S = st.S;
+  const int W = gen->max_new_tokens;
+  GenPlan gp;
+  gp.max_new = W;
+  gp.eos = gen->eos_id;
+  gp.pad = gen->pad_id;
+  AIQ_TRY(ws(c, "g.tok", std::max<int64_t>(S * W, 1), &gp.tok));
+  AIQ_TRY(ws(c, "g.len", std::max<int64_t>(S, 1), &gp.len));
+  AIQ_TRY(prefill_phase(c, t, *m, q, &st, &gp));
+  CUDA_TRY(cudaEventRecord(ev[2], c->stream));
+
+  ResultH R;
+  R.gen_max_new = W;
+  if (!like) {
+    R.gen_ids.resize(S);
+    R.gen_tok.resize(S * W);
+    R.gen_len.resize(S);
+    if (S) {
+      CUDA_TRY(cudaMemcpyAsync(R.gen_ids.data(), st.ids, S * 4, cudaMemcpyDeviceToHost, c->stream));
+      CUDA_TRY(cudaMemcpyAsync(R.gen_tok.data(), gp.tok, S * W * 4, cudaMemcpyDeviceToHost, c->stream));
+      CUDA_TRY(cudaMemcpyAsync(R.gen_len.data(), gp.len, S * 4, cudaMemcpyDeviceToHost, c->stream));
+    }
+  } else if (S > 0) {
+    // LIKE on the device; only the matches' ids (and, if asked, their tokens) come back
+    const int64_t nb = (S + kRowsPerBlock - 1) / kRowsPerBlock;
+    int32_t *pat, *match, *bcnt, *pos, *rows;
+    uint32_t* bits;
+    int64_t* boff;
+    AIQ_TRY(ws(c, "g.like", std::max(gen->like_len, 1), &pat));
+    AIQ_TRY(ws(c, "g.match", S, &match));
+    AIQ_TRY(ws(c, "g.bits", nb * (kRowsPerBlock / 32), &bits));
+    AIQ_TRY(ws(c, "g.bcnt", nb, &bcnt));
+    AIQ_TRY(ws(c, "g.boff", nb + 1, &boff));
+    if (gen->like_len > 0)
+      CUDA_TRY(cudaMemcpyAsync(pat, gen->like_tokens, gen->like_len * 4, cudaMemcpyHostToDevice, c->stream));
+    {
+      ProfScope p(c, "like_match", 0, 0);
+      launch_like_match(gp.tok, gp.len, S, W, pat, gen->like_len, match, c->stream);
+      launch_flag_mask(match, S, bits, bcnt, c->stream);
+      launch_scan_counts(bcnt, nb, boff, c->stream);
+      counted(c, 3);
+    }
+    AIQ_TRY(read_i64(c, boff + nb, 1, c->h_pin));
+    const int64_t Y = c->h_pin[0];
+    AIQ_TRY(ws(c, "g.mpos", std::max<int64_t>(Y, 1), &pos));
+    AIQ_TRY(ws(c, "g.mrows", std::max<int64_t>(Y, 1), &rows));
+    launch_compact(bits, boff, S, pos, st.ids, rows, c->stream);
+    counted(c, 1);
+    R.row_ids.resize(Y);
+    if (Y) CUDA_TRY(cudaMemcpyAsync(R.row_ids.data(), rows, Y * 4, cudaMemcpyDeviceToHost, c->stream));
+    R.label_counts.clear();
+    if ((gen->flags & AIQ_GEN_MATCH_TOKENS) && Y > 0) {
+      int32_t *mtok, *mlen;
+      AIQ_TRY(ws(c, "g.mtok", Y * W, &mtok));
+      AIQ_TRY(ws(c, "g.mlen", Y, &mlen));
+      launch_gather_rows_i32(gp.tok, W, pos, Y, mtok, c->stream);
+      launch_gather_rows_i32(gp.len, 1, pos, Y, mlen, c->stream);
+      counted(c, 2);
+      R.gen_ids = R.row_ids;
+      R.gen_tok.resize(Y * W);
+      R.gen_len.resize(Y);
+      CUDA_TRY(cudaMemcpyAsync(R.gen_tok.data(), mtok, Y * W * 4, cudaMemcpyDeviceToHost, c->stream));
+      CUDA_TRY(cudaMemcpyAsync(R.gen_len.data(), mlen, Y * 4, cudaMemcpyDeviceToHost, c->stream));
+    }
+  }
+  CUDA_TRY(cudaEventRecord(ev[3], c->stream));
+  AIQ_TRY(sync_and_check(c));
+  float t01 = 0, t12 = 0, t23 = 0, t03 = 0, tdec = 0;
+  cudaEventElapsedTime(&t01, ev[0], ev[1]);
+  cudaEventElapsedTime(&t12, ev[1], ev[2]);
+  cudaEventElapsedTime(&t23, ev[2], ev[3]);
+  cudaEventElapsedTime(&t03, ev[0], ev[3]);
+  for (auto& e : ev) c->ev_pool.push_back(e);
+  for (auto& sp : gp.spans) {
+    float ms = 0;
+    cudaEventElapsedTime(&ms, sp.first, sp.second);
+    tdec += ms;
+    c->ev_pool.push_back(sp.first);
+    c->ev_pool.push_back(sp.second);
+  }
+  collect_profile(c);
+  ResultH& dst = new_result(c, out);
+  dst = std::move(R);
+  finish_view(dst, st, t.n_rows, 0, -1);
+  dst.v.count = like ? static_cast<int64_t>(dst.row_ids.size()) : -1;
+  dst.v.ms_relational = t01;
+  dst.v.ms_prefill = t12;
+  dst.v.ms_aggregate = t23;
+  dst.v.ms_total = t03;
+  dst.v.ms_decode = tdec;
+  dst.v.decode_flops = gp.flops;
+  dst.v.n_decode_steps = gp.steps;
+  {
+    const aiq_model_config& g = m->cfg;
+    const double pre = S > 0 ? static_cast<double>(st.P) : 0.0;
+    const double d = g.d_model, qd = double(g.n_heads) * g.head_dim, kd = double(g.n_kv_heads) * g.head_dim;
+    const double per_layer = m->linear_flops_per_token / g.n_layers;
+    const double tail = 2.0 * (qd * d + 3.0 * d * g.d_ffn);
+    dst.v.prefill_flops = per_layer * (g.n_layers - 1) * (static_cast<double>(st.T) + pre) +
+                          2.0 * d * (qd + 2 * kd) * static_cast<double>(st.T) + tail * static_cast<double>(S) +
+                          per_layer * pre +
+                          4.0 * g.n_heads * g.head_dim * g.n_layers * (static_cast<double>(st.pairs) + pre * (pre + 1) / 2);
+  }
   dst.v.n_launches = c->launches;
   return AIQ_OK;
 }
@@ -1184,6 +1520,17 @@ aiq_status aiq_run_join_select(aiq_ctx* c, aiq_table build, int32_t build_key, c
   return run_query(c, &b->second, build_key, build_preds, n_build_preds, p->second, probe_key, m, q, out);
 }
 
+aiq_status aiq_run_transform(aiq_ctx* c, aiq_table table, aiq_model model, const aiq_select* q,
+                             const aiq_generate* gen, aiq_result_h* out) {
+  if (!c || !q || !gen || !out) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
+  auto t = c->tables.find(table);
+  if (t == c->tables.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown table handle");
+  auto mi = c->models.find(model);
+  if (mi == c->models.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown model handle");
+  CUDA_TRY(cudaSetDevice(c->device));
+  return run_transform(c, t->second, &mi->second, q, gen, out);
+}
+
 aiq_status aiq_result(aiq_ctx* c, aiq_result_h h, aiq_result_view* out) {
   if (!c || !out) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
   auto it = c->results.find(h);
@@ -1306,6 +1653,25 @@ aiq_status aiq_op_attention(aiq_ctx* c, const void* qkv, int64_t T, const int32_
   const aiq_status st = sync_and_check(c);
   collect_profile(c);
   return st;
+}
+
+aiq_status aiq_op_decode_attention(aiq_ctx* c, const void* qkv, int32_t R, int32_t Hq, int32_t Hkv, int32_t hd,
+                                   const void* prefix_kv, int32_t P, const void* own_kv, const int32_t* seq_start,
+                                   void* gen_kv, int32_t gen_cap, int32_t slot, void* out) {
+  if (!c || !qkv || !own_kv || !seq_start || !gen_kv || !out || R < 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv ||
+      P < 0 || (P > 0 && !prefix_kv) || gen_cap < 1 || slot < 0 || slot >= gen_cap)
+    return fail(AIQ_ERR_INVALID_ARG, "bad args");
+  if (!(hd == 32 || hd == 64 || hd == 128) || Hq / Hkv > 8)
+    return fail(AIQ_ERR_UNSUPPORTED, "hd must be 32, 64 or 128 and Hq / Hkv <= 8");
+  if (R == 0) return AIQ_OK;
+  CUDA_TRY(cudaSetDevice(c->device));
+  const int e = launch_decode_attention(static_cast<const __half*>(qkv), static_cast<int64_t>(Hq + 2 * Hkv) * hd, R,
+                                        Hq, Hkv, hd, static_cast<const __half*>(prefix_kv), P,
+                                        static_cast<const __half*>(own_kv), seq_start, static_cast<__half*>(gen_kv),
+                                        gen_cap, slot, static_cast<__half*>(out), c->d_err, c->stream);
+  if (e != 0) return fail(AIQ_ERR_CUDA, std::string("decode attention launch: ") +
+                                            cudaGetErrorString(static_cast<cudaError_t>(e)));
+  return sync_and_check(c);
 }
 
 }  // extern "C"

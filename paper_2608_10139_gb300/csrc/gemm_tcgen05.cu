@@ -214,6 +214,42 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
         }
       }
     }
+  } else if constexpr (EPI == EPI_ARGMAX) {
+    // logits = acc + bias; strictly-greater keeps the first column of a tie
+    float best = -INFINITY;
+    int bcol = -1;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 64) {
+      float v0[32], v1[32];
+      load2x32(trow + c, trow + c + 32, v0, v1);
+      if (live) {
+        float b0[32], b1[32];
+        load_f32x32(ep.bias + n0 + c, b0);
+        load_f32x32(ep.bias + n0 + c + 32, b1);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const float x = v0[j] + b0[j];
+          if (x > best) {
+            best = x;
+            bcol = n0 + c + j;
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const float x = v1[j] + b1[j];
+          if (x > best) {
+            best = x;
+            bcol = n0 + c + 32 + j;
+          }
+        }
+      }
+    }
+    if (live && bcol >= 0) {
+      const uint32_t u = __float_as_uint(best);
+      const uint32_t ord = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+      atomicMax(ep.best + row,
+                (static_cast<unsigned long long>(ord) << 32) | (0xFFFFFFFFu - static_cast<uint32_t>(bcol)));
+    }
   } else if constexpr (EPI == EPI_SWIGLU_F16) {
     __half* o = static_cast<__half*>(ep.out) + static_cast<int64_t>(row) * ep.ldo + n0 / 2;
 #pragma unroll 1
@@ -715,6 +751,7 @@ int dispatch_pair(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, 
     case EPI_ROPE_F16: return launch_pair<EPI_ROPE_F16>(ma, mb, a, num_sms, s);
     case EPI_RESID_F32: return launch_pair<EPI_RESID_F32>(ma, mb, a, num_sms, s);
     case EPI_SWIGLU_F16: return launch_pair<EPI_SWIGLU_F16>(ma, mb, a, num_sms, s);
+    case EPI_ARGMAX: return launch_pair<EPI_ARGMAX>(ma, mb, a, num_sms, s);
   }
   return cudaErrorInvalidValue;
 }
@@ -726,6 +763,7 @@ int dispatch_epi(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, i
     case EPI_ROPE_F16: return launch<BN, EPI_ROPE_F16>(ma, mb, a, num_sms, s);
     case EPI_RESID_F32: return launch<BN, EPI_RESID_F32>(ma, mb, a, num_sms, s);
     case EPI_SWIGLU_F16: return launch<BN, EPI_SWIGLU_F16>(ma, mb, a, num_sms, s);
+    case EPI_ARGMAX: return launch<BN, EPI_ARGMAX>(ma, mb, a, num_sms, s);
   }
   return cudaErrorInvalidValue;
 }
@@ -743,6 +781,7 @@ int gemm_f16_tcgen05(const __half* A, int64_t lda, const __half* B, int64_t ldb,
     const int hd = ep.head_dim;
     if (!(hd == 32 || hd == 64 || hd == 128) || bn % hd != 0 || !ep.positions || !ep.rope_cos) return cudaErrorInvalidValue;
   }
+  if (ep.kind == EPI_ARGMAX && (!ep.bias || !ep.best)) return cudaErrorInvalidValue;
   CUtensorMap ma, mb;
   if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, B, N, K, ldb, pair ? 128 : bn)) return cudaErrorInvalidValue;
   KArgs a{M, N, K, ep};

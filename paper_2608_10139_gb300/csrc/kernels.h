@@ -14,6 +14,8 @@ enum GemmEpi : int {
   EPI_ROPE_F16 = 1,   // as EPI_F16, rotary embedding applied to columns < rope_cols
   EPI_RESID_F32 = 2,  // out fp32 [M, N] += acc  (residual stream update)
   EPI_SWIGLU_F16 = 3, // B interleaves gate/up blocks of BN/2 rows: out fp16 [M, N/2] = silu(g) * u
+  EPI_ARGMAX = 4,     // per row: max over columns of acc + bias[col] and its first column, folded into
+                      // best[row] with a 64-bit atomicMax of (order-preserving value bits, ~col)
 };
 
 struct GemmEpilogue {
@@ -37,6 +39,9 @@ struct GemmEpilogue {
   float eps = 0.f;
   __half* xh_out = nullptr;
   float* ss_out = nullptr;
+  // EPI_ARGMAX: fp32 bias [N] (-inf marks padding columns) and the per-row packed result
+  const float* bias = nullptr;
+  unsigned long long* best = nullptr;
 };
 
 // C = A[M,K] * B[N,K]^T with fp16 operands and fp32 accumulation on tcgen05.
@@ -156,6 +161,30 @@ void launch_nonzero_mask(const unsigned long long* counts, int64_t n, uint32_t* 
 void launch_gather_groups(const int32_t* rows, int64_t g, const int64_t* build_keys,
                           const unsigned long long* counts, int64_t* keys_out, int64_t* counts_out,
                           cudaStream_t s);
+
+// ---------------------------------------------------------------- decode ---
+// Decode attention of R single-token rows (row r's token: q/k/v in qkv row r).
+// Keys of row r: the P shared-prefix rows of pkv, its own prompt rows
+// kvc[seq_start[r] .. seq_start[r+1]), then its generated slots gkv[r][0 .. slot]
+// (this step's key/value are first written to slot `slot`).  Layouts [.][2 Hkv hd]
+// (keys then values).  Returns 0 or a cudaError_t value.
+int launch_decode_attention(const __half* qkv, int64_t ldq, int R, int Hq, int Hkv, int hd, const __half* pkv, int P,
+                            const __half* kvc, const int32_t* seq_start, __half* gkv, int gcap, int slot, __half* out,
+                            int* err, cudaStream_t s);
+// Token of step t for every row from the packed LM-head argmax (best[] is reset
+// to 0), pad after an eos, and the fed-back position P + len + t.
+void launch_decode_select(unsigned long long* best, int R, int t, int max_new, int eos, int pad, int V, int32_t* done,
+                          int32_t* gen_tok, int32_t* gen_len, int32_t* next_tok, int32_t* pos,
+                          const int32_t* seq_start, int P, int* err, cudaStream_t s);
+void launch_patch_empty_rows(float* resid, const int32_t* last_idx, const float* prefix_last, int R, int d,
+                             cudaStream_t s);
+void launch_bias_f32(const uint16_t* b, int V, int Vpad, float* out, cudaStream_t s);
+void launch_like_match(const int32_t* gen_tok, const int32_t* gen_len, int64_t S, int max_new, const int32_t* pattern,
+                       int plen, int32_t* match, cudaStream_t s);
+void launch_gather_rows_i32(const int32_t* src, int width, const int32_t* pos, int64_t n, int32_t* out,
+                            cudaStream_t s);
+// bits / per-block counts of the non-zero entries of an int32 flag array.
+void launch_flag_mask(const int32_t* flags, int64_t n, uint32_t* bits, int32_t* block_counts, cudaStream_t s);
 
 // Sets the thread-local message that aiq_last_error() returns.
 void set_error_message(const char* msg);

@@ -394,6 +394,16 @@ __global__ void __launch_bounds__(kThreads) k_decide(const float* logits, int64_
   if (threadIdx.x < K && hist[threadIdx.x]) atomicAdd(label_counts + threadIdx.x, (unsigned long long)hist[threadIdx.x]);
 }
 
+__global__ void __launch_bounds__(kThreads) k_flag_mask(const int32_t* flags, int64_t n, uint32_t* bits,
+                                                         int32_t* block_counts) {
+  __shared__ int red[kThreads / 32];
+  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock + threadIdx.x * 8;
+  uint32_t byte = 0;
+  for (int j = 0; j < 8 && r0 + j < n; ++j) byte |= static_cast<uint32_t>(flags[r0 + j] != 0) << j;
+  const int total = write_words_and_count(byte, bits + static_cast<int64_t>(blockIdx.x) * (kRowsPerBlock / 32), red);
+  if (threadIdx.x == 0) block_counts[blockIdx.x] = total;
+}
+
 __global__ void k_group_build(const int32_t* decision, const int32_t* build_rows, int64_t S,
                               unsigned long long* counts) {
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
@@ -485,6 +495,11 @@ void launch_decide(const float* logits, int64_t S, int K, int32_t* decision, uin
   if (S <= 0) return;
   k_decide<<<blocks_for(S, kRowsPerBlock), kThreads, 0, s>>>(logits, S, K, decision, yes_bits, block_counts,
                                                              label_counts);
+}
+
+void launch_flag_mask(const int32_t* flags, int64_t n, uint32_t* bits, int32_t* block_counts, cudaStream_t s) {
+  if (n <= 0) return;
+  k_flag_mask<<<blocks_for(n, kRowsPerBlock), kThreads, 0, s>>>(flags, n, bits, block_counts);
 }
 
 void launch_group_build(const int32_t* decision, const int32_t* cand_build_rows, int64_t S,
