@@ -154,6 +154,7 @@ struct aiq_ctx {
   bool profile = false;
   bool gemm_pair = true;  // CTA-pair (cta_group::2) GEMM tiles where the shape allows
   bool attention_tc = true;  // tcgen05 attention where the head shape allows
+  int64_t decode_rows = 2048;  // generation: target rows per prefill chunk (= decode batch)
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
   std::map<std::string, StatAcc> stats;
@@ -755,7 +756,14 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
   st->pairs = c->h_pin[1];
   st->P = P;
   const int64_t max_len = col.max_len;  // longest row text; the prefix runs on its own
-  const int64_t B = std::max<int64_t>(std::max<int64_t>(c->token_budget, max_len), P);
+  int64_t budget = c->token_budget;
+  if (gp) {
+    // a chunk's rows decode together, one token each per step: size the chunks
+    // for about decode_rows rows so that the decode GEMMs have M of that order
+    const int64_t per_row = T / S + 1;
+    budget = std::max(budget, std::min<int64_t>(c->decode_rows * per_row, int64_t(1) << 20));
+  }
+  const int64_t B = std::max<int64_t>(std::max<int64_t>(budget, max_len), P);
   const int64_t step = B - max_len + 1;
   const int64_t n_chunks = std::max<int64_t>(1, (T + step - 1) / step);
   st->n_chunks = n_chunks;
@@ -1562,6 +1570,11 @@ aiq_status aiq_set_option(aiq_ctx* c, const char* name, int64_t value) {
   }
   if (!std::strcmp(name, "gemm_pair")) {
     c->gemm_pair = value != 0;
+    return AIQ_OK;
+  }
+  if (!std::strcmp(name, "decode_rows")) {
+    if (value < 1 || value > (int64_t(1) << 20)) return fail(AIQ_ERR_INVALID_ARG, "decode_rows must be 1..2^20");
+    c->decode_rows = value;
     return AIQ_OK;
   }
   if (!std::strcmp(name, "attention_tc")) {

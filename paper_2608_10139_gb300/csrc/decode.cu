@@ -15,8 +15,7 @@
 namespace aiq {
 namespace {
 
-constexpr int kDecThreads = 128;  // 4 warps per (row, KV head)
-constexpr int kDecMaxG = 8;       // query heads per KV head
+constexpr int kDecThreads = 256;  // 8 warps per (row, KV head)
 
 struct DecArgs {
   const __half* qkv;  // [R][ldq]: q heads, k heads, v heads of this step's token
@@ -46,21 +45,27 @@ __device__ __forceinline__ float warp_sum(float v) {
 }
 
 // One block per (row, KV head): the G query heads of the group against all
-// of the row's keys.  Warp w takes key blocks w, w + 4, ... of 32 keys; in a
-// block each lane scores one key for all G heads (q from shared memory),
-// then the warp accumulates P V with each lane owning HD / 32 output columns.
-// The four warps' partial (max, sum, output) are merged at the end.
-template <int HD>
+// of the row's keys.  Warp w takes key blocks w, w + 8, ... of KB keys.  In a
+// block every lane (a pair of lanes for head_dim 128) holds one key: the key
+// row and all KB value rows of the block are loaded together, so a block costs
+// one memory round trip; the scores of the G heads come from q in shared
+// memory, then P V accumulates with each lane owning HD / 32 output columns.
+// The eight warps' partial (max, sum, output) are merged at the end.
+template <int HD, int G>
 __global__ void __launch_bounds__(kDecThreads) k_decode_attention(DecArgs a) {
-  constexpr int DPL = HD / 32;  // output columns per lane
-  __shared__ __align__(16) float sq[kDecMaxG * HD];
-  __shared__ float sp[4][kDecMaxG][32];
-  __shared__ float sm_m[4][kDecMaxG], sm_l[4][kDecMaxG];
-  __shared__ __align__(16) float so[4][kDecMaxG][HD];
+  constexpr int NW = kDecThreads / 32;
+  constexpr int DPL = HD / 32;           // output columns per lane
+  constexpr int LPK = HD == 128 ? 2 : 1; // lanes per key
+  constexpr int KB = 32 / LPK;           // keys per warp block
+  constexpr int KC = HD / 8 / LPK;       // 16-byte chunks of a key row per lane
+  constexpr int VW = (DPL + 1) / 2;      // 32-bit words of packed halves per value slice
+  __shared__ __align__(16) float sq[G * HD];
+  __shared__ float sp[NW][G][KB];
+  __shared__ float sm_m[NW][G], sm_l[NW][G];
+  __shared__ __align__(16) float so[NW][G * HD];
 
   const int r = blockIdx.x / a.Hkv, h = blockIdx.x % a.Hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int G = a.G;
   const int kd = a.Hkv * HD;
   const int64_t ld = 2 * static_cast<int64_t>(kd);
   const __half* qrow = a.qkv + static_cast<int64_t>(r) * a.ldq;
@@ -77,17 +82,18 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_attention(DecArgs a) {
   __syncthreads();  // the slot written above is read back by this block below
 
   const int n_keys = a.P + len + a.slot + 1;
-  float m_run[kDecMaxG], l_lane[kDecMaxG], o[kDecMaxG][DPL];
+  float m_run[G], l_lane[G], o[G][DPL];
 #pragma unroll
-  for (int g = 0; g < kDecMaxG; ++g) {
+  for (int g = 0; g < G; ++g) {
     m_run[g] = -INFINITY;
     l_lane[g] = 0.f;
 #pragma unroll
     for (int e = 0; e < DPL; ++e) o[g][e] = 0.f;
   }
+  const int kslot = lane / LPK, part = lane % LPK;  // this lane's key in the block, its half of the row
 
-  for (int blk = warp; blk * 32 < n_keys; blk += 4) {
-    const int j = blk * 32 + lane;
+  for (int blk = warp; blk * KB < n_keys; blk += NW) {
+    const int j = blk * KB + kslot;
     const bool valid = j < n_keys;
     // key row of key j: shared prefix, then the row's prompt, then its generated tokens
     const __half* krow = nullptr;
@@ -100,107 +106,122 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_attention(DecArgs a) {
         krow = a.gkv + (static_cast<int64_t>(r) * a.gcap + (j - a.P - len)) * ld;
       krow += h * HD;
     }
-    float s[kDecMaxG];
-#pragma unroll
-    for (int g = 0; g < kDecMaxG; ++g) s[g] = 0.f;
+    const int nvalid = min(KB, n_keys - blk * KB);
+    // issue every load of the block: this lane's part of its key row, and its
+    // column slice of all KB value rows (plain loads: the newest slot was
+    // written by this block a moment ago)
+    uint4 kr[KC];
     if (valid) {
 #pragma unroll
-      for (int c = 0; c < HD / 8; ++c) {
-        // plain loads: this block wrote the newest slot a moment ago
-        const uint4 kv = reinterpret_cast<const uint4*>(krow)[c];
-        const __half2* k2 = reinterpret_cast<const __half2*>(&kv);
-        float kf[8];
+      for (int c = 0; c < KC; ++c) kr[c] = reinterpret_cast<const uint4*>(krow + part * (HD / 2))[c];
+    } else {
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 f = __half22float2(k2[e]);
-          kf[2 * e] = f.x;
-          kf[2 * e + 1] = f.y;
-        }
+      for (int c = 0; c < KC; ++c) kr[c] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    const unsigned long long my_v = reinterpret_cast<unsigned long long>(krow ? krow + kd : nullptr);
+    uint32_t vr[KB][VW];
 #pragma unroll
-        for (int g = 0; g < kDecMaxG; ++g) {
-          if (g < G) {
-            const float4 q0 = *reinterpret_cast<const float4*>(&sq[g * HD + 8 * c]);
-            const float4 q1 = *reinterpret_cast<const float4*>(&sq[g * HD + 8 * c + 4]);
-            s[g] += q0.x * kf[0] + q0.y * kf[1] + q0.z * kf[2] + q0.w * kf[3] + q1.x * kf[4] + q1.y * kf[5] +
-                    q1.z * kf[6] + q1.w * kf[7];
-          }
+    for (int jb = 0; jb < KB; ++jb) {
+      const __half* vrow = reinterpret_cast<const __half*>(__shfl_sync(0xffffffffu, my_v, jb * LPK));
+      if (jb < nvalid) {
+        if constexpr (DPL == 1) {
+          vr[jb][0] = reinterpret_cast<const uint16_t*>(vrow)[lane];
+        } else if constexpr (DPL == 2) {
+          vr[jb][0] = reinterpret_cast<const uint32_t*>(vrow)[lane];
+        } else {
+          const uint2 u = reinterpret_cast<const uint2*>(vrow)[lane];
+          vr[jb][0] = u.x;
+          vr[jb][1] = u.y;
         }
+      } else {
+#pragma unroll
+        for (int e = 0; e < VW; ++e) vr[jb][e] = 0u;
+      }
+    }
+    // scores of the G heads for this lane's key (partial over its half of the row for hd 128)
+    float s[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) s[g] = 0.f;
+#pragma unroll
+    for (int c = 0; c < KC; ++c) {
+      const __half2* k2 = reinterpret_cast<const __half2*>(&kr[c]);
+      float kf[8];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 f = __half22float2(k2[e]);
+        kf[2 * e] = f.x;
+        kf[2 * e + 1] = f.y;
+      }
+      const int d0 = part * (HD / 2) + 8 * c;
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        const float4 q0 = *reinterpret_cast<const float4*>(&sq[g * HD + d0]);
+        const float4 q1 = *reinterpret_cast<const float4*>(&sq[g * HD + d0 + 4]);
+        s[g] += q0.x * kf[0] + q0.y * kf[1] + q0.z * kf[2] + q0.w * kf[3] + q1.x * kf[4] + q1.y * kf[5] +
+                q1.z * kf[6] + q1.w * kf[7];
       }
     }
 #pragma unroll
-    for (int g = 0; g < kDecMaxG; ++g) {
-      if (g < G) {
-        const float sv = valid ? s[g] : -INFINITY;
-        const float m_new = fmaxf(m_run[g], warp_max(sv));  // finite: key blk * 32 is valid
-        const float f = exp2f(m_run[g] - m_new);
-        const float p = valid ? exp2f(sv - m_new) : 0.f;
-        l_lane[g] = l_lane[g] * f + p;
+    for (int g = 0; g < G; ++g) {
+      if constexpr (LPK == 2) s[g] += __shfl_xor_sync(0xffffffffu, s[g], 1);
+      const float sv = valid ? s[g] : -INFINITY;
+      const float m_new = fmaxf(m_run[g], warp_max(sv));  // finite: the block's first key is valid
+      const float f = exp2f(m_run[g] - m_new);
+      const float p = valid ? exp2f(sv - m_new) : 0.f;
+      l_lane[g] = l_lane[g] * f + (part == 0 ? p : 0.f);
 #pragma unroll
-        for (int e = 0; e < DPL; ++e) o[g][e] *= f;
-        m_run[g] = m_new;
-        sp[warp][g][lane] = p;
-      }
+      for (int e = 0; e < DPL; ++e) o[g][e] *= f;
+      m_run[g] = m_new;
+      if (part == 0) sp[warp][g][kslot] = p;
     }
     __syncwarp();
-    const int nvalid = min(32, n_keys - blk * 32);
-    const unsigned long long my_v = reinterpret_cast<unsigned long long>(krow ? krow + kd : nullptr);
-#pragma unroll 4
-    for (int jj = 0; jj < nvalid; ++jj) {
-      const __half* vrow = reinterpret_cast<const __half*>(__shfl_sync(0xffffffffu, my_v, jj));
+#pragma unroll
+    for (int jb = 0; jb < KB; ++jb) {
       float vf[DPL];
       if constexpr (DPL == 1) {
-        vf[0] = __half2float(vrow[lane]);
-      } else if constexpr (DPL == 2) {
-        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(vrow + 2 * lane));
-        vf[0] = f.x;
-        vf[1] = f.y;
+        vf[0] = __half2float(__ushort_as_half(static_cast<unsigned short>(vr[jb][0])));
       } else {
-        const uint2 u = *reinterpret_cast<const uint2*>(vrow + 4 * lane);
-        const float2 f0 = __half22float2(*reinterpret_cast<const __half2*>(&u.x));
-        const float2 f1 = __half22float2(*reinterpret_cast<const __half2*>(&u.y));
-        vf[0] = f0.x;
-        vf[1] = f0.y;
-        vf[2] = f1.x;
-        vf[3] = f1.y;
+#pragma unroll
+        for (int e = 0; e < VW; ++e) {
+          const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&vr[jb][e]));
+          vf[2 * e] = f.x;
+          vf[2 * e + 1] = f.y;
+        }
       }
 #pragma unroll
-      for (int g = 0; g < kDecMaxG; ++g) {
-        if (g < G) {
-          const float p = sp[warp][g][jj];
+      for (int g = 0; g < G; ++g) {
+        const float p = sp[warp][g][jb];  // 0 for keys past the end
 #pragma unroll
-          for (int e = 0; e < DPL; ++e) o[g][e] += p * vf[e];
-        }
+        for (int e = 0; e < DPL; ++e) o[g][e] += p * vf[e];
       }
     }
     __syncwarp();
   }
 
-  // merge the four warps' partial softmax states
+  // merge the warps' partial softmax states
 #pragma unroll
-  for (int g = 0; g < kDecMaxG; ++g) {
-    if (g < G) {
-      const float l = warp_sum(l_lane[g]);
-      if (lane == 0) {
-        sm_m[warp][g] = m_run[g];
-        sm_l[warp][g] = l;
-      }
-#pragma unroll
-      for (int e = 0; e < DPL; ++e) so[warp][g][lane * DPL + e] = o[g][e];
+  for (int g = 0; g < G; ++g) {
+    const float l = warp_sum(l_lane[g]);
+    if (lane == 0) {
+      sm_m[warp][g] = m_run[g];
+      sm_l[warp][g] = l;
     }
+#pragma unroll
+    for (int e = 0; e < DPL; ++e) so[warp][g * HD + lane * DPL + e] = o[g][e];
   }
   __syncthreads();
   __half* orow = a.out + static_cast<int64_t>(r) * a.Hq * HD + h * G * HD;
   for (int i = tid; i < G * HD; i += kDecThreads) {
-    const int g = i / HD, dd = i % HD;
+    const int g = i / HD;
     float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) M = fmaxf(M, sm_m[w][g]);
+    for (int w = 0; w < NW; ++w) M = fmaxf(M, sm_m[w][g]);
     float L = 0.f, O = 0.f;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) {
+    for (int w = 0; w < NW; ++w) {
       const float f = sm_m[w][g] == -INFINITY ? 0.f : exp2f(sm_m[w][g] - M);  // a warp without keys
       L += sm_l[w][g] * f;
-      O += so[w][g][dd] * f;
+      O += so[w][i] * f;
     }
     orow[i] = __float2half_rn(O / L);
   }
@@ -268,10 +289,21 @@ __global__ void k_gather_rows_i32(const int32_t* src, int width, const int32_t* 
   for (int i = threadIdx.x; i < width; i += blockDim.x) out[k * width + i] = s[i];
 }
 
-template <int HD>
+template <int HD, int G>
 int launch_dec(const DecArgs& a, int R, cudaStream_t s) {
-  k_decode_attention<HD><<<R * a.Hkv, kDecThreads, 0, s>>>(a);
+  k_decode_attention<HD, G><<<R * a.Hkv, kDecThreads, 0, s>>>(a);
   return cudaGetLastError();
+}
+
+template <int HD>
+int launch_dec_g(const DecArgs& a, int R, cudaStream_t s) {
+  switch (a.G) {
+    case 1: return launch_dec<HD, 1>(a, R, s);
+    case 2: return launch_dec<HD, 2>(a, R, s);
+    case 4: return launch_dec<HD, 4>(a, R, s);
+    case 8: return launch_dec<HD, 8>(a, R, s);
+  }
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace
@@ -280,14 +312,16 @@ int launch_decode_attention(const __half* qkv, int64_t ldq, int R, int Hq, int H
                             const __half* kvc, const int32_t* seq_start, __half* gkv, int gcap, int slot, __half* out,
                             int* err, cudaStream_t s) {
   if (R <= 0) return 0;
-  if (Hq % Hkv || Hq / Hkv > kDecMaxG || !(hd == 32 || hd == 64 || hd == 128) || slot < 0 || slot >= gcap)
+  const int G = Hkv > 0 ? Hq / Hkv : 0;
+  if (Hkv <= 0 || Hq % Hkv || !(G == 1 || G == 2 || G == 4 || G == 8) || !(hd == 32 || hd == 64 || hd == 128) ||
+      slot < 0 || slot >= gcap)
     return cudaErrorInvalidValue;
   DecArgs a{qkv, ldq, Hq, Hkv, Hq / Hkv, pkv, P, kvc, seq_start, gkv, gcap, slot,
             1.4426950408889634f / sqrtf(static_cast<float>(hd)), out, err};
   switch (hd) {
-    case 32: return launch_dec<32>(a, R, s);
-    case 64: return launch_dec<64>(a, R, s);
-    default: return launch_dec<128>(a, R, s);
+    case 32: return launch_dec_g<32>(a, R, s);
+    case 64: return launch_dec_g<64>(a, R, s);
+    default: return launch_dec_g<128>(a, R, s);
   }
 }
 
