@@ -33,195 +33,225 @@ struct DecArgs {
   int* err;
 };
 
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
+__device__ __forceinline__ void cp_async16(uint32_t saddr, const void* gmem, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(saddr), "l"(gmem), "r"(valid ? 16 : 0)
+               : "memory");
 }
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t saddr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(saddr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], uint32_t saddr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(saddr));
+}
+__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&x)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(x[0]), "r"(x[1]), "r"(x[2]), "r"(x[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_h2(float x, float y) {
+  __half2 v = __floats2half2_rn(x, y);
+  return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// One block per (row, KV head): the G query heads of the group against all
-// of the row's keys.  Warp w takes key blocks w, w + 8, ... of KB keys.  In a
-// block every lane (a pair of lanes for head_dim 128) holds one key: the key
-// row and all KB value rows of the block are loaded together, so a block costs
-// one memory round trip; the scores of the G heads come from q in shared
-// memory, then P V accumulates with each lane owning HD / 32 output columns.
-// The eight warps' partial (max, sum, output) are merged at the end.
-template <int HD, int G>
+template <int HD>
+struct DecCfg {
+  static constexpr int NW = kDecThreads / 32;
+  static constexpr int KB = HD == 128 ? 16 : 32;  // keys per warp block
+  static constexpr int LDS = HD + 8;    // padded smem row (halves): conflict-free ldmatrix
+  static constexpr int Q_HALVES = 16 * LDS;
+  static constexpr int WARP_HALVES = 2 * KB * LDS;  // K block then V block
+  static constexpr int SMEM = (Q_HALVES + NW * WARP_HALVES) * 2;
+};
+
+// One block per (row, KV head): the G <= 8 query heads of the group against
+// all of the row's keys, on m16n8k16 tensor-core MMAs (the heads are the
+// rows of the A tile, the rest of its 16 rows are zero).  Warp w takes key
+// blocks w, w + 8, ... of 32 keys (16 at head_dim 128): it stages the block's
+// K and V rows in its own shared-memory slice with cp.async (all rows of both
+// at once), then
+// S = Q K^T, the online softmax on the accumulator fragments and O += P V
+// with V read through ldmatrix.trans.  The eight warps' partial (max, sum,
+// output) are merged at the end.
+template <int HD>
 __global__ void __launch_bounds__(kDecThreads) k_decode_attention(DecArgs a) {
-  constexpr int NW = kDecThreads / 32;
-  constexpr int DPL = HD / 32;           // output columns per lane
-  constexpr int LPK = HD == 128 ? 2 : 1; // lanes per key
-  constexpr int KB = 32 / LPK;           // keys per warp block
-  constexpr int KC = HD / 8 / LPK;       // 16-byte chunks of a key row per lane
-  constexpr int VW = (DPL + 1) / 2;      // 32-bit words of packed halves per value slice
-  __shared__ __align__(16) float sq[G * HD];
-  __shared__ float sp[NW][G][KB];
-  __shared__ float sm_m[NW][G], sm_l[NW][G];
-  __shared__ __align__(16) float so[NW][G * HD];
+  using C = DecCfg<HD>;
+  constexpr int NW = C::NW, KB = C::KB, LDS = C::LDS;
+  constexpr int KS = HD / 16;  // k-steps of Q K^T
+  constexpr int DN = HD / 8;   // 8-wide output column tiles
+  constexpr int CH = HD / 8;   // 16-byte chunks per row
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  __half* sQ = reinterpret_cast<__half*>(smem_raw);
 
   const int r = blockIdx.x / a.Hkv, h = blockIdx.x % a.Hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int G = a.G;
   const int kd = a.Hkv * HD;
   const int64_t ld = 2 * static_cast<int64_t>(kd);
   const __half* qrow = a.qkv + static_cast<int64_t>(r) * a.ldq;
   const int st = a.seq_start[r], len = a.seq_start[r + 1] - st;
   __half* slot = a.gkv + (static_cast<int64_t>(r) * a.gcap + a.slot) * ld;
+  __half* sK = sQ + C::Q_HALVES + warp * C::WARP_HALVES;
+  __half* sV = sK + KB * LDS;
 
-  // this token's key and value into its cache slot; its G query heads (scaled) into shared memory
+  // this token's key and value into its cache slot; the G query heads as the
+  // first rows of a zero-padded 16-row tile
   for (int i = tid; i < HD / 8; i += kDecThreads) {
     reinterpret_cast<uint4*>(slot + h * HD)[i] = reinterpret_cast<const uint4*>(qrow + (a.Hq + h) * HD)[i];
     reinterpret_cast<uint4*>(slot + kd + h * HD)[i] =
         reinterpret_cast<const uint4*>(qrow + (a.Hq + a.Hkv + h) * HD)[i];
   }
-  for (int i = tid; i < G * HD; i += kDecThreads) sq[i] = __half2float(qrow[h * G * HD + i]) * a.scale_log2;
-  __syncthreads();  // the slot written above is read back by this block below
+  for (int i = tid; i < 16 * CH; i += kDecThreads) {
+    const int row = i / CH, c = i % CH;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (row < G) v = reinterpret_cast<const uint4*>(qrow + (h * G + row) * HD)[c];
+    *reinterpret_cast<uint4*>(sQ + row * LDS + c * 8) = v;
+  }
+  __syncthreads();  // the slot written above is read back by this block below; sQ complete
 
   const int n_keys = a.P + len + a.slot + 1;
-  float m_run[G], l_lane[G], o[G][DPL];
+  const int gq = lane >> 2, tq = lane & 3;
+  uint32_t qf[KS][4];
 #pragma unroll
-  for (int g = 0; g < G; ++g) {
-    m_run[g] = -INFINITY;
-    l_lane[g] = 0.f;
-#pragma unroll
-    for (int e = 0; e < DPL; ++e) o[g][e] = 0.f;
+  for (int kk = 0; kk < KS; ++kk) {
+    const int mat = lane >> 3;
+    const int row = (lane & 7) + 8 * (mat & 1);
+    const int col = kk * 16 + 8 * (mat >> 1);
+    ldsm_x4(qf[kk], smem_u32(sQ + row * LDS + col));
   }
-  const int kslot = lane / LPK, part = lane % LPK;  // this lane's key in the block, its half of the row
+  float o[DN][4];
+#pragma unroll
+  for (int i = 0; i < DN; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float m0 = -INFINITY, l0 = 0.f;  // row gq (a head when gq < G); rows 8..15 are padding
 
   for (int blk = warp; blk * KB < n_keys; blk += NW) {
-    const int j = blk * KB + kslot;
-    const bool valid = j < n_keys;
-    // key row of key j: shared prefix, then the row's prompt, then its generated tokens
-    const __half* krow = nullptr;
-    if (valid) {
-      if (j < a.P)
-        krow = a.pkv + j * ld;
-      else if (j < a.P + len)
-        krow = a.kvc + (st + j - a.P) * ld;
-      else
-        krow = a.gkv + (static_cast<int64_t>(r) * a.gcap + (j - a.P - len)) * ld;
-      krow += h * HD;
-    }
-    const int nvalid = min(KB, n_keys - blk * KB);
-    // issue every load of the block: this lane's part of its key row, and its
-    // column slice of all KB value rows (plain loads: the newest slot was
-    // written by this block a moment ago)
-    uint4 kr[KC];
-    if (valid) {
+    const int key0 = blk * KB;
+    // stage K and V of keys key0 .. key0 + KB - 1: shared prefix, the row's prompt, its generated tokens
 #pragma unroll
-      for (int c = 0; c < KC; ++c) kr[c] = reinterpret_cast<const uint4*>(krow + part * (HD / 2))[c];
-    } else {
-#pragma unroll
-      for (int c = 0; c < KC; ++c) kr[c] = make_uint4(0u, 0u, 0u, 0u);
-    }
-    const unsigned long long my_v = reinterpret_cast<unsigned long long>(krow ? krow + kd : nullptr);
-    uint32_t vr[KB][VW];
-#pragma unroll
-    for (int jb = 0; jb < KB; ++jb) {
-      const __half* vrow = reinterpret_cast<const __half*>(__shfl_sync(0xffffffffu, my_v, jb * LPK));
-      if (jb < nvalid) {
-        if constexpr (DPL == 1) {
-          vr[jb][0] = reinterpret_cast<const uint16_t*>(vrow)[lane];
-        } else if constexpr (DPL == 2) {
-          vr[jb][0] = reinterpret_cast<const uint32_t*>(vrow)[lane];
-        } else {
-          const uint2 u = reinterpret_cast<const uint2*>(vrow)[lane];
-          vr[jb][0] = u.x;
-          vr[jb][1] = u.y;
-        }
+    for (int i = 0; i < KB * CH / 32; ++i) {
+      const int c = lane + 32 * i;
+      const int kr = c / CH, part = c % CH;
+      const int j = key0 + kr;
+      const bool valid = j < n_keys;
+      const __half* krow = a.pkv;  // any mapped address when the chunk is zero-filled
+      if (valid) {
+        if (j < a.P)
+          krow = a.pkv + j * ld;
+        else if (j < a.P + len)
+          krow = a.kvc + (st + j - a.P) * ld;
+        else
+          krow = a.gkv + (static_cast<int64_t>(r) * a.gcap + (j - a.P - len)) * ld;
+        krow += h * HD;
       } else {
-#pragma unroll
-        for (int e = 0; e < VW; ++e) vr[jb][e] = 0u;
+        krow = slot;
       }
+      cp_async16(smem_u32(sK + kr * LDS + part * 8), krow + part * 8, valid);
+      cp_async16(smem_u32(sV + kr * LDS + part * 8), krow + kd + part * 8, valid);
     }
-    // scores of the G heads for this lane's key (partial over its half of the row for hd 128)
-    float s[G];
-#pragma unroll
-    for (int g = 0; g < G; ++g) s[g] = 0.f;
-#pragma unroll
-    for (int c = 0; c < KC; ++c) {
-      const __half2* k2 = reinterpret_cast<const __half2*>(&kr[c]);
-      float kf[8];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float2 f = __half22float2(k2[e]);
-        kf[2 * e] = f.x;
-        kf[2 * e + 1] = f.y;
-      }
-      const int d0 = part * (HD / 2) + 8 * c;
-#pragma unroll
-      for (int g = 0; g < G; ++g) {
-        const float4 q0 = *reinterpret_cast<const float4*>(&sq[g * HD + d0]);
-        const float4 q1 = *reinterpret_cast<const float4*>(&sq[g * HD + d0 + 4]);
-        s[g] += q0.x * kf[0] + q0.y * kf[1] + q0.z * kf[2] + q0.w * kf[3] + q1.x * kf[4] + q1.y * kf[5] +
-                q1.z * kf[6] + q1.w * kf[7];
-      }
-    }
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      if constexpr (LPK == 2) s[g] += __shfl_xor_sync(0xffffffffu, s[g], 1);
-      const float sv = valid ? s[g] : -INFINITY;
-      const float m_new = fmaxf(m_run[g], warp_max(sv));  // finite: the block's first key is valid
-      const float f = exp2f(m_run[g] - m_new);
-      const float p = valid ? exp2f(sv - m_new) : 0.f;
-      l_lane[g] = l_lane[g] * f + (part == 0 ? p : 0.f);
-#pragma unroll
-      for (int e = 0; e < DPL; ++e) o[g][e] *= f;
-      m_run[g] = m_new;
-      if (part == 0) sp[warp][g][kslot] = p;
-    }
+    cp_async_wait_all();
     __syncwarp();
+    float sc[KB / 8][4];
 #pragma unroll
-    for (int jb = 0; jb < KB; ++jb) {
-      float vf[DPL];
-      if constexpr (DPL == 1) {
-        vf[0] = __half2float(__ushort_as_half(static_cast<unsigned short>(vr[jb][0])));
-      } else {
+    for (int n = 0; n < KB / 8; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
 #pragma unroll
-        for (int e = 0; e < VW; ++e) {
-          const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&vr[jb][e]));
-          vf[2 * e] = f.x;
-          vf[2 * e + 1] = f.y;
-        }
-      }
+    for (int kk = 0; kk < KS; ++kk) {
 #pragma unroll
-      for (int g = 0; g < G; ++g) {
-        const float p = sp[warp][g][jb];  // 0 for keys past the end
-#pragma unroll
-        for (int e = 0; e < DPL; ++e) o[g][e] += p * vf[e];
+      for (int np = 0; np < KB / 16; ++np) {
+        const int mat = lane >> 3;
+        const int key = np * 16 + (lane & 7) + 8 * (mat >> 1);
+        const int dim = kk * 16 + 8 * (mat & 1);
+        uint32_t bb[4];
+        ldsm_x4(bb, smem_u32(sK + key * LDS + dim));
+        mma16816(sc[2 * np], qf[kk], bb[0], bb[1]);
+        mma16816(sc[2 * np + 1], qf[kk], bb[2], bb[3]);
       }
     }
-    __syncwarp();
+    // log2 units, keys past the end masked; row gq uses elements 0 and 1
+    float mx = -INFINITY;
+#pragma unroll
+    for (int n = 0; n < KB / 8; ++n) {
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int key = key0 + n * 8 + 2 * tq + e;
+        const float v = key < n_keys ? sc[n][e] * a.scale_log2 : -INFINITY;
+        sc[n][e] = v;
+        mx = fmaxf(mx, v);
+      }
+    }
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+    const float mn = fmaxf(m0, mx);  // finite: key0 < n_keys
+    const float c0 = exp2f(m0 - mn);
+    m0 = mn;
+    float rs = 0.f;
+#pragma unroll
+    for (int n = 0; n < KB / 8; ++n) {
+      sc[n][0] = exp2f(sc[n][0] - mn);
+      sc[n][1] = exp2f(sc[n][1] - mn);
+      rs += sc[n][0] + sc[n][1];
+    }
+    l0 = l0 * c0 + rs;
+#pragma unroll
+    for (int i = 0; i < DN; ++i) {
+      o[i][0] *= c0;
+      o[i][1] *= c0;
+    }
+#pragma unroll
+    for (int k2 = 0; k2 < KB / 16; ++k2) {
+      uint32_t pa[4];
+      pa[0] = pack_h2(sc[2 * k2][0], sc[2 * k2][1]);
+      pa[1] = 0u;  // padding rows 8..15
+      pa[2] = pack_h2(sc[2 * k2 + 1][0], sc[2 * k2 + 1][1]);
+      pa[3] = 0u;
+#pragma unroll
+      for (int dp = 0; dp < DN / 2; ++dp) {
+        const int mat = lane >> 3;
+        const int key = k2 * 16 + (lane & 7) + 8 * (mat & 1);
+        const int dim = dp * 16 + 8 * (mat >> 1);
+        uint32_t bb[4];
+        ldsm_x4_t(bb, smem_u32(sV + key * LDS + dim));
+        mma16816(o[2 * dp], pa, bb[0], bb[1]);
+        mma16816(o[2 * dp + 1], pa, bb[2], bb[3]);
+      }
+    }
+    __syncwarp();  // every lane is done with this warp's staging before it is refilled
   }
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
 
-  // merge the warps' partial softmax states
+  // merge the warps' partial softmax states (the staging area is reused)
+  __syncthreads();
+  float* mm = reinterpret_cast<float*>(smem_raw + C::Q_HALVES * 2);  // [NW][8] max, [NW][8] sum, [NW][8][HD]
+  float* ll = mm + NW * 8;
+  float* oo = ll + NW * 8;
+  if (tq == 0) {
+    mm[warp * 8 + gq] = m0;
+    ll[warp * 8 + gq] = l0;
+  }
 #pragma unroll
-  for (int g = 0; g < G; ++g) {
-    const float l = warp_sum(l_lane[g]);
-    if (lane == 0) {
-      sm_m[warp][g] = m_run[g];
-      sm_l[warp][g] = l;
-    }
-#pragma unroll
-    for (int e = 0; e < DPL; ++e) so[warp][g * HD + lane * DPL + e] = o[g][e];
+  for (int i = 0; i < DN; ++i) {
+    oo[(warp * 8 + gq) * HD + i * 8 + 2 * tq] = o[i][0];
+    oo[(warp * 8 + gq) * HD + i * 8 + 2 * tq + 1] = o[i][1];
   }
   __syncthreads();
   __half* orow = a.out + static_cast<int64_t>(r) * a.Hq * HD + h * G * HD;
   for (int i = tid; i < G * HD; i += kDecThreads) {
-    const int g = i / HD;
+    const int g = i / HD, dd = i % HD;
     float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < NW; ++w) M = fmaxf(M, sm_m[w][g]);
+    for (int w = 0; w < NW; ++w) M = fmaxf(M, mm[w * 8 + g]);
     float L = 0.f, O = 0.f;
 #pragma unroll
     for (int w = 0; w < NW; ++w) {
-      const float f = sm_m[w][g] == -INFINITY ? 0.f : exp2f(sm_m[w][g] - M);  // a warp without keys
-      L += sm_l[w][g] * f;
-      O += so[w][i] * f;
+      const float f = mm[w * 8 + g] == -INFINITY ? 0.f : exp2f(mm[w * 8 + g] - M);  // a warp without keys
+      L += ll[w * 8 + g] * f;
+      O += oo[(w * 8 + g) * HD + dd] * f;
     }
     orow[i] = __float2half_rn(O / L);
   }
@@ -289,21 +319,13 @@ __global__ void k_gather_rows_i32(const int32_t* src, int width, const int32_t* 
   for (int i = threadIdx.x; i < width; i += blockDim.x) out[k * width + i] = s[i];
 }
 
-template <int HD, int G>
-int launch_dec(const DecArgs& a, int R, cudaStream_t s) {
-  k_decode_attention<HD, G><<<R * a.Hkv, kDecThreads, 0, s>>>(a);
-  return cudaGetLastError();
-}
-
 template <int HD>
-int launch_dec_g(const DecArgs& a, int R, cudaStream_t s) {
-  switch (a.G) {
-    case 1: return launch_dec<HD, 1>(a, R, s);
-    case 2: return launch_dec<HD, 2>(a, R, s);
-    case 4: return launch_dec<HD, 4>(a, R, s);
-    case 8: return launch_dec<HD, 8>(a, R, s);
-  }
-  return cudaErrorInvalidValue;
+int launch_dec(const DecArgs& a, int R, cudaStream_t s) {
+  using C = DecCfg<HD>;
+  cudaError_t e = cudaFuncSetAttribute(k_decode_attention<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  k_decode_attention<HD><<<R * a.Hkv, kDecThreads, C::SMEM, s>>>(a);
+  return cudaGetLastError();
 }
 
 }  // namespace
@@ -319,9 +341,9 @@ int launch_decode_attention(const __half* qkv, int64_t ldq, int R, int Hq, int H
   DecArgs a{qkv, ldq, Hq, Hkv, Hq / Hkv, pkv, P, kvc, seq_start, gkv, gcap, slot,
             1.4426950408889634f / sqrtf(static_cast<float>(hd)), out, err};
   switch (hd) {
-    case 32: return launch_dec_g<32>(a, R, s);
-    case 64: return launch_dec_g<64>(a, R, s);
-    default: return launch_dec_g<128>(a, R, s);
+    case 32: return launch_dec<32>(a, R, s);
+    case 64: return launch_dec<64>(a, R, s);
+    default: return launch_dec<128>(a, R, s);
   }
 }
 
