@@ -65,9 +65,8 @@ struct DecCfg {
   static constexpr int NW = kDecThreads / 32;
   static constexpr int KB = HD == 128 ? 16 : 32;  // keys per warp block
   static constexpr int LDS = HD + 8;    // padded smem row (halves): conflict-free ldmatrix
-  static constexpr int Q_HALVES = 16 * LDS;
   static constexpr int WARP_HALVES = 2 * KB * LDS;  // K block then V block
-  static constexpr int SMEM = (Q_HALVES + NW * WARP_HALVES) * 2;
+  static constexpr int SMEM = NW * WARP_HALVES * 2;
 };
 
 // One block per (row, KV head): the G <= 8 query heads of the group against
@@ -80,14 +79,13 @@ struct DecCfg {
 // with V read through ldmatrix.trans.  The eight warps' partial (max, sum,
 // output) are merged at the end.
 template <int HD>
-__global__ void __launch_bounds__(kDecThreads) k_decode_attention(DecArgs a) {
+__global__ void __launch_bounds__(kDecThreads, HD == 128 ? 2 : 3) k_decode_attention(DecArgs a) {
   using C = DecCfg<HD>;
   constexpr int NW = C::NW, KB = C::KB, LDS = C::LDS;
   constexpr int KS = HD / 16;  // k-steps of Q K^T
   constexpr int DN = HD / 8;   // 8-wide output column tiles
   constexpr int CH = HD / 8;   // 16-byte chunks per row
   extern __shared__ __align__(16) uint8_t smem_raw[];
-  __half* sQ = reinterpret_cast<__half*>(smem_raw);
 
   const int r = blockIdx.x / a.Hkv, h = blockIdx.x % a.Hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -97,33 +95,31 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_attention(DecArgs a) {
   const __half* qrow = a.qkv + static_cast<int64_t>(r) * a.ldq;
   const int st = a.seq_start[r], len = a.seq_start[r + 1] - st;
   __half* slot = a.gkv + (static_cast<int64_t>(r) * a.gcap + a.slot) * ld;
-  __half* sK = sQ + C::Q_HALVES + warp * C::WARP_HALVES;
+  __half* sK = reinterpret_cast<__half*>(smem_raw) + warp * C::WARP_HALVES;
   __half* sV = sK + KB * LDS;
 
-  // this token's key and value into its cache slot; the G query heads as the
-  // first rows of a zero-padded 16-row tile
+  // this token's key and value into its cache slot, for the later steps; this
+  // step reads them straight from the qkv row (no wait on the store)
   for (int i = tid; i < HD / 8; i += kDecThreads) {
     reinterpret_cast<uint4*>(slot + h * HD)[i] = reinterpret_cast<const uint4*>(qrow + (a.Hq + h) * HD)[i];
     reinterpret_cast<uint4*>(slot + kd + h * HD)[i] =
         reinterpret_cast<const uint4*>(qrow + (a.Hq + a.Hkv + h) * HD)[i];
   }
-  for (int i = tid; i < 16 * CH; i += kDecThreads) {
-    const int row = i / CH, c = i % CH;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (row < G) v = reinterpret_cast<const uint4*>(qrow + (h * G + row) * HD)[c];
-    *reinterpret_cast<uint4*>(sQ + row * LDS + c * 8) = v;
-  }
-  __syncthreads();  // the slot written above is read back by this block below; sQ complete
 
   const int n_keys = a.P + len + a.slot + 1;
   const int gq = lane >> 2, tq = lane & 3;
+  // A fragments of the query tile straight from global memory: row gq is query
+  // head h G + gq (rows >= G and 8..15 are zero padding)
   uint32_t qf[KS][4];
+  {
+    const uint32_t* q32 = reinterpret_cast<const uint32_t*>(qrow + (h * G + gq) * HD);
 #pragma unroll
-  for (int kk = 0; kk < KS; ++kk) {
-    const int mat = lane >> 3;
-    const int row = (lane & 7) + 8 * (mat & 1);
-    const int col = kk * 16 + 8 * (mat >> 1);
-    ldsm_x4(qf[kk], smem_u32(sQ + row * LDS + col));
+    for (int kk = 0; kk < KS; ++kk) {
+      qf[kk][0] = gq < G ? q32[(kk * 16 + 2 * tq) / 2] : 0u;
+      qf[kk][1] = 0u;
+      qf[kk][2] = gq < G ? q32[(kk * 16 + 8 + 2 * tq) / 2] : 0u;
+      qf[kk][3] = 0u;
+    }
   }
   float o[DN][4];
 #pragma unroll
@@ -139,17 +135,19 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_attention(DecArgs a) {
       const int kr = c / CH, part = c % CH;
       const int j = key0 + kr;
       const bool valid = j < n_keys;
-      const __half* krow = a.pkv;  // any mapped address when the chunk is zero-filled
+      const __half* krow;
       if (valid) {
         if (j < a.P)
           krow = a.pkv + j * ld;
         else if (j < a.P + len)
           krow = a.kvc + (st + j - a.P) * ld;
-        else
+        else if (j < n_keys - 1)
           krow = a.gkv + (static_cast<int64_t>(r) * a.gcap + (j - a.P - len)) * ld;
+        else
+          krow = qrow + a.Hq * HD;  // this step's token: its k heads, then (kd further) its v heads
         krow += h * HD;
       } else {
-        krow = slot;
+        krow = qrow;  // zero-filled chunk: any mapped address
       }
       cp_async16(smem_u32(sK + kr * LDS + part * 8), krow + part * 8, valid);
       cp_async16(smem_u32(sV + kr * LDS + part * 8), krow + kd + part * 8, valid);
@@ -227,7 +225,7 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_attention(DecArgs a) {
 
   // merge the warps' partial softmax states (the staging area is reused)
   __syncthreads();
-  float* mm = reinterpret_cast<float*>(smem_raw + C::Q_HALVES * 2);  // [NW][8] max, [NW][8] sum, [NW][8][HD]
+  float* mm = reinterpret_cast<float*>(smem_raw);  // [NW][8] max, [NW][8] sum, [NW][8][HD]
   float* ll = mm + NW * 8;
   float* oo = ll + NW * 8;
   if (tq == 0) {
