@@ -58,6 +58,7 @@ def parse():
     p.add_argument("--transform", type=int, default=0,
                    help="AI_TRANSFORM: greedy tokens per candidate row (0: the AI_IF query)")
     p.add_argument("--like", default="", help="AI_TRANSFORM ... LIKE pattern, comma-separated token ids")
+    p.add_argument("--decode-rows", type=int, default=0, help="AI_TRANSFORM rows per decode batch (0: library default)")
     return p.parse_args()
 
 
@@ -441,6 +442,8 @@ def transform_bench(args):
     table = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
     preds = [(p.column, p.op, p.value) for p in w.preds]
     like = [int(x) for x in args.like.split(",")] if args.like else None
+    if args.decode_rows:
+        ctx.set_option("decode_rows", args.decode_rows)
     flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
 
     def run():
@@ -474,7 +477,8 @@ def transform_bench(args):
             "higher_is_better": True, "steps": args.steps, "warmup": args.warmup, "dtype": "f16xf16->f32",
             "data": "synthetic",
             "config": {"workload": w.name, "rows": w.n_rows, "candidates": r.n_candidates,
-                       "max_new_tokens": args.transform, "like": like, "chunks": r.n_chunks},
+                       "max_new_tokens": args.transform, "like": like, "chunks": r.n_chunks,
+                       "decode_rows": args.decode_rows or 4096},
             "input_rows_per_s": w.n_rows / (ms / 1000.0), "p50_latency_ms": ms, "decode_ms_p50": dec_ms,
             "prefill_ms_p50": statistics.median([x.ms_prefill - x.ms_decode for x in res]),
             "decode_tflops": r.decode_flops / (dec_ms / 1000.0) / 1e12 if dec_ms else None,

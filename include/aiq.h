@@ -230,8 +230,8 @@ const char* aiq_last_error(void);
  * N % 256 == 0 and M >= 512; also selects them for aiq_op_gemm with bn = 256),
  * "attention_tc" (0/1, default 1: tcgen05 attention where the head shape
  * allows), "decode_rows" (aiq_run_transform: rows per prefill chunk, which
- * decode together, default 2048; the chunk's token budget grows to fit them,
- * up to 2^20 tokens). */
+ * decode together, default 4096; the chunk's token budget grows to fit them,
+ * up to 2^20 tokens and 32 GB of cached prompt keys/values). */
 aiq_status aiq_set_option(aiq_ctx* ctx, const char* name, int64_t value);
 
 /* The context's CUDA stream (a cudaStream_t), for callers that time the

@@ -154,7 +154,7 @@ struct aiq_ctx {
   bool profile = false;
   bool gemm_pair = true;  // CTA-pair (cta_group::2) GEMM tiles where the shape allows
   bool attention_tc = true;  // tcgen05 attention where the head shape allows
-  int64_t decode_rows = 2048;  // generation: target rows per prefill chunk (= decode batch)
+  int64_t decode_rows = 4096;  // generation: target rows per prefill chunk (= decode batch)
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
   std::map<std::string, StatAcc> stats;
@@ -759,9 +759,11 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
   int64_t budget = c->token_budget;
   if (gp) {
     // a chunk's rows decode together, one token each per step: size the chunks
-    // for about decode_rows rows so that the decode GEMMs have M of that order
+    // for about decode_rows rows so that the decode GEMMs have M of that order,
+    // within 2^20 tokens and 32 GB of cached prompt keys/values per chunk
     const int64_t per_row = T / S + 1;
-    budget = std::max(budget, std::min<int64_t>(c->decode_rows * per_row, int64_t(1) << 20));
+    const int64_t kv_cap = (int64_t(32) << 30) / (2 * int64_t(m.cfg.n_layers) * 2 * m.cfg.n_kv_heads * m.cfg.head_dim);
+    budget = std::max(budget, std::min<int64_t>({c->decode_rows * per_row, int64_t(1) << 20, kv_cap}));
   }
   const int64_t B = std::max<int64_t>(std::max<int64_t>(budget, max_len), P);
   const int64_t step = B - max_len + 1;

@@ -66,3 +66,34 @@ def compare_logits(gpu_logits, ref_logits, what=""):
         clear = others.max(axis=1) < -DECISION_MARGIN
     assert np.array_equal(gdec[clear], ref_dec[clear]), f"{what} decision mismatch on clear rows"
     return worst
+
+
+def check_greedy(model, prompts, toks, text_len, eos, pad, what=""):
+    """Teacher-forced validity of GPU greedy outputs; returns (worst gap
+    ratio, number of steps where the oracle's own argmax differs)."""
+    worst, flips = 0.0, 0
+    n_new = toks.shape[1]
+    for i, p in enumerate(prompts):
+        y = [int(v) for v in toks[i]]
+        L = int(text_len[i])
+        steps = min(L + 1, n_new)                  # decisions taken: the text, then the eos
+        if L < n_new:
+            assert y[L] == eos, f"{what} row {i}: text_len {L} but token {y[L]} is not the eos"
+            assert all(v == pad for v in y[L + 1:]), f"{what} row {i}: no pad after the eos"
+        assert eos not in y[:L], f"{what} row {i}: eos before text_len"
+        seq = np.concatenate([p, np.asarray(y[:steps - 1], np.int64)])
+        z = _tf().vocab_logits(model, [seq])[len(p) - 1:]
+        for t in range(steps):
+            zt = z[t]
+            top = float(zt.max())
+            gap = top - float(zt[y[t]])
+            ratio = gap / (MARGIN_RTOL * max(1.0, abs(top)))
+            worst = max(worst, ratio)
+            flips += int(_tf().first_argmax(zt) != y[t])
+            assert ratio <= 1.0, f"{what} row {i} step {t}: token {y[t]} is {gap:.4g} below the max"
+    return worst, flips
+
+
+def _tf():
+    from oracle import transformer as tf
+    return tf

@@ -8,7 +8,7 @@ import numpy as np
 import pytest
 
 import synth
-from helpers import compare_logits, gpu_ctx, oracle_preds, weights_list
+from helpers import check_greedy, compare_logits, gpu_ctx, oracle_preds, weights_list
 from oracle import query as oq
 from oracle import relational as rel
 from oracle import transformer as tf
@@ -112,3 +112,27 @@ def test_c5_sweep_1pct_full_query(ctx):
     w = synth.sweep_workload("1%", "lognormal")
     r, agg = _run_select_full(ctx, w, 6)
     assert np.array_equal(r.row_ids, agg["row_ids"])
+
+
+def test_transform_c2_select_1b_full_size(ctx):
+    """AI_TRANSFORM over the select workload's 13,050 candidates (1B shape) in
+    the benchmark's launch configuration (decode batches of ~4096 rows): row
+    ids exact, a seeded sample of rows checked by teacher forcing."""
+    w = synth.C2_SELECT
+    q = synth.make_inputs(w)
+    W = synth.make_weights(w.model, w.weight_seed)
+    m = ctx.load_model(w.model, weights_list(w.model, W))
+    t = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+    preds = oracle_preds(w.preds)
+    r = ctx.run_transform(t, m, preds, q.prefix, 16)
+    ctx.free_table(t)
+    ctx.free_model(m)
+    cand = rel.compact(rel.predicate_mask(q.table.cols, preds, q.table.n_rows))
+    assert np.array_equal(r.gen_row_ids, cand)
+    assert r.gen_tokens.shape == (len(cand), 16) and r.n_chunks >= 3
+    lens = np.diff(q.table.offsets)[cand]
+    sample = _sample(len(cand), 2, w.data_seed, lens)
+    prompts = oq.prompts(q.prefix, q.table.offsets, q.table.tokens, cand[sample])
+    worst, flips = check_greedy(tf.Model(w.model, W), prompts, r.gen_tokens[sample], r.gen_text_len[sample], -1, 0,
+                                "c2 transform")
+    print(f"c2 transform: worst gap ratio {worst:.3f}, near-tie flips {flips}")

@@ -16,7 +16,7 @@ import numpy as np
 import pytest
 
 import synth
-from helpers import MARGIN_RTOL, gpu_ctx, oracle_preds, weights_list
+from helpers import check_greedy, gpu_ctx, weights_list
 from oracle import query as oq
 from oracle import relational as rel
 from oracle import transformer as tf
@@ -30,32 +30,6 @@ def ctx():
     c = gpu_ctx()
     yield c
     c.close()
-
-
-def check_greedy(model, prompts, toks, text_len, eos, pad, what=""):
-    """Teacher-forced validity of GPU greedy outputs; returns (worst gap
-    ratio, number of steps where the oracle's own argmax differs)."""
-    worst, flips = 0.0, 0
-    n_new = toks.shape[1]
-    for i, p in enumerate(prompts):
-        y = [int(v) for v in toks[i]]
-        L = int(text_len[i])
-        steps = min(L + 1, n_new)                  # decisions taken: the text, then the eos
-        if L < n_new:
-            assert y[L] == eos, f"{what} row {i}: text_len {L} but token {y[L]} is not the eos"
-            assert all(v == pad for v in y[L + 1:]), f"{what} row {i}: no pad after the eos"
-        assert eos not in y[:L], f"{what} row {i}: eos before text_len"
-        seq = np.concatenate([p, np.asarray(y[:steps - 1], np.int64)])
-        z = tf.vocab_logits(model, [seq])[len(p) - 1:]
-        for t in range(steps):
-            zt = z[t]
-            top = float(zt.max())
-            gap = top - float(zt[y[t]])
-            ratio = gap / (MARGIN_RTOL * max(1.0, abs(top)))
-            worst = max(worst, ratio)
-            flips += int(tf.first_argmax(zt) != y[t])
-            assert ratio <= 1.0, f"{what} row {i} step {t}: token {y[t]} is {gap:.4g} below the max"
-    return worst, flips
 
 
 def _tiny_inputs(shape=synth.TINY, n_rows=96, seed=5, empty_every=0):
@@ -74,13 +48,15 @@ def _tiny_inputs(shape=synth.TINY, n_rows=96, seed=5, empty_every=0):
 def _run(ctx, shape, W, table, prefix, preds, max_new, eos=-1, pad=0, like=None, match_tokens=False, budget=None):
     m = ctx.load_model(shape, weights_list(shape, W))
     t = ctx.load_table(table.cols, (table.offsets, table.tokens))
-    if budget:
+    if budget:   # small chunks, so that several decode batches run
         ctx.set_option("token_budget", budget)
+        ctx.set_option("decode_rows", 8)
     try:
         return ctx.run_transform(t, m, preds, prefix, max_new, eos=eos, pad=pad, like=like,
                                  match_tokens=match_tokens)
     finally:
         ctx.set_option("token_budget", 131072)
+        ctx.set_option("decode_rows", 4096)
         ctx.free_table(t)
         ctx.free_model(m)
 
