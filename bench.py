@@ -59,6 +59,7 @@ def parse():
                    help="AI_TRANSFORM: greedy tokens per candidate row (0: the AI_IF query)")
     p.add_argument("--like", default="", help="AI_TRANSFORM ... LIKE pattern, comma-separated token ids")
     p.add_argument("--decode-rows", type=int, default=0, help="AI_TRANSFORM rows per decode batch (0: library default)")
+    p.add_argument("--pairs", action="store_true", help="Table 2 Q4: AI_IF over the reviews self-joined on movie id")
     return p.parse_args()
 
 
@@ -498,6 +499,68 @@ def transform_bench(args):
     ctx.close()
 
 
+def pairs_bench(args):
+    """Table 2 Q4 on the q4_pairs_1b workload: the self-join's pairs formed on
+    the device, AI_IF on each pair's prompt.  One JSON line (pairs/s, the
+    prefill GEMM roofline, and the host->device bytes against the bytes the
+    pair prompts would take if they were formed on the host)."""
+    import torch
+    from paper_2608_10139_gb300 import aiq
+    from paper_2608_10139_gb300 import build as _build
+    _build.build()
+    w = synth.Q4_PAIRS
+    q = synth.make_pair_inputs(w)
+    W = synth.make_weights(w.model, w.weight_seed)
+    ctx = aiq.Context(0)
+    model = ctx.load_model(w.model, [W[n] for n, _, _ in synth.weight_specs(w.model)])
+    table = ctx.load_table(q.table.cols, (q.table.offsets, q.table.tokens))
+    preds = [("score", 0, w.score_below)]   # LT
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+
+    def run():
+        return ctx.run_pair_select(table, "movie_id", model, preds, q.prefix, w.label_ids, agg=aiq.AGG_ROW_IDS)
+
+    for _ in range(args.warmup):
+        run()
+    clocks = ClockSampler(0)
+    ctx.reset_kernel_stats()
+    ctx.set_option("profile", 1)
+    clocks.start()
+    res = []
+    for _ in range(args.steps):
+        flush.add_(1.0)
+        torch.cuda.synchronize()
+        res.append(run())
+    clk = clocks.stop()
+    ctx.set_option("profile", 0)
+    stats = ctx.kernel_stats()
+    r = res[-1]
+    ms = statistics.median([x.ms_total for x in res])
+    g = [v for k, v in stats.items() if k.startswith("gemm_")]
+    g_ms = sum(v["total_ms"] for v in g)
+    g_tf = sum(v["flops"] for v in g) / (g_ms / 1000.0) / 1e12 if g_ms else None
+    pk, src = peaks()
+    peak = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+    line = {"metric": "Q4 pairs/s", "value": r.n_candidates / (ms / 1000.0), "unit": "pairs/s",
+            "higher_is_better": True, "steps": args.steps, "warmup": args.warmup, "dtype": "f16xf16->f32",
+            "data": "synthetic",
+            "config": {"workload": w.name, "rows": w.n_rows, "movies": w.n_movies, "pairs": r.n_candidates,
+                       "yes_pairs": r.count},
+            "input_rows_per_s": w.n_rows / (ms / 1000.0), "p50_latency_ms": ms,
+            "relational_ms_p50": statistics.median([x.ms_relational for x in res]),
+            "prefill_tflops": r.prefill_flops / (r.ms_prefill / 1000.0) / 1e12 if r.ms_prefill else None,
+            "h2d_table_bytes": int(q.table.nbytes()),
+            "host_pair_prompt_bytes": int(4 * r.n_tokens),
+            "kernel_ms_per_step": {k: round(v["total_ms"] / args.steps, 3) for k, v in sorted(stats.items())},
+            "roofline": {"kernel": "gemm_tcgen05", "bound": "tensor", "achieved": g_tf, "peak": peak,
+                         "unit": "TFLOP/s", "frac": g_tf / peak if g_tf else None,
+                         "peak_source": f"{src} bf16_tflops_sustained"},
+            "clocks": clk}
+    print(json.dumps(line), flush=True)
+    ctx.free_table(table)
+    ctx.close()
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -508,6 +571,8 @@ def main():
         sweep(args)
     elif args.transform:
         transform_bench(args)
+    elif args.pairs:
+        pairs_bench(args)
     else:
         ours(args)
 

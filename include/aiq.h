@@ -128,6 +128,8 @@ typedef struct {
   double prefill_flops; /* executed: 2*params per token + 4*Hq*hd*L per causal pair + head */
   int64_t n_launches;   /* CUDA kernels this query launched */
   int64_t n_prefill_tokens; /* tokens run through the decoder: the shared prefix once + every row's text */
+  /* aiq_run_pair_select with AIQ_AGG_ROW_IDS: the B row of each yes pair (row_ids holds its A row) */
+  const int32_t* row_ids_b;
   /* aiq_run_transform only (zero / NULL otherwise) */
   int32_t gen_max_new;        /* columns of gen_tokens: the generate spec's max_new_tokens */
   int64_t n_gen_rows;         /* rows of gen_tokens */
@@ -217,6 +219,21 @@ enum {
  * cross PCIe. */
 aiq_status aiq_run_transform(aiq_ctx* ctx, aiq_table table, aiq_model model, const aiq_select* q,
                              const aiq_generate* gen, aiq_result_h* out);
+
+/* Table 2 Q4: SELECT A.text, B.text, AI_IF([A.text, B.text]) FROM table A
+ * CROSS JOIN table B WHERE <preds> AND A.key = B.key AND A.row < B.row.
+ * The terms filter the table before it is joined with itself (both sides);
+ * key_column is an INT64 column; each pair (a, b) of selected rows with equal
+ * keys and a < b (the row index is the review id) is one candidate, in
+ * ascending (a, b) order, and its prompt is prefix ++ text(a) ++ text(b).
+ * The pairs are formed on the device: only the table crosses PCIe (§4.3).
+ * Candidates are pairs: n_candidates = number of pairs; with AIQ_FLAG_LOGITS
+ * cand_row_ids / cand_build_rows hold every pair's A / B row with its logits
+ * and decision; AIQ_AGG_COUNT gives the yes pairs' count, AIQ_AGG_ROW_IDS also
+ * their A rows (row_ids) and B rows (row_ids_b).  2 labels.  More than
+ * 2^31 - 1 pairs gives AIQ_ERR_CAPACITY. */
+aiq_status aiq_run_pair_select(aiq_ctx* ctx, aiq_table table, int32_t key_column, aiq_model model,
+                               const aiq_select* q, aiq_result_h* out);
 
 aiq_status aiq_result(aiq_ctx* ctx, aiq_result_h result, aiq_result_view* out);
 aiq_status aiq_result_free(aiq_ctx* ctx, aiq_result_h result);

@@ -64,7 +64,7 @@ class _View(C.Structure):
                 ("label_logits", C.POINTER(C.c_float)), ("decisions", C.POINTER(C.c_int32)),
                 ("ms_relational", C.c_float), ("ms_prefill", C.c_float), ("ms_aggregate", C.c_float),
                 ("ms_total", C.c_float), ("prefill_flops", C.c_double), ("n_launches", C.c_int64),
-                ("n_prefill_tokens", C.c_int64),
+                ("n_prefill_tokens", C.c_int64), ("row_ids_b", C.POINTER(C.c_int32)),
                 ("gen_max_new", C.c_int32), ("n_gen_rows", C.c_int64), ("gen_row_ids", C.POINTER(C.c_int32)),
                 ("gen_tokens", C.POINTER(C.c_int32)), ("gen_text_len", C.POINTER(C.c_int32)),
                 ("ms_decode", C.c_float), ("decode_flops", C.c_double), ("n_decode_steps", C.c_int64)]
@@ -98,6 +98,7 @@ _SIGS = {
     "aiq_run_select": [C.c_void_p, C.c_int64, C.c_int64, C.POINTER(_Select), C.POINTER(C.c_int64)],
     "aiq_run_join_select": [C.c_void_p, C.c_int64, C.c_int32, C.POINTER(_Pred), C.c_int32, C.c_int64, C.c_int32,
                             C.c_int64, C.POINTER(_Select), C.POINTER(C.c_int64)],
+    "aiq_run_pair_select": [C.c_void_p, C.c_int64, C.c_int32, C.c_int64, C.POINTER(_Select), C.POINTER(C.c_int64)],
     "aiq_run_transform": [C.c_void_p, C.c_int64, C.c_int64, C.POINTER(_Select), C.POINTER(_Generate),
                           C.POINTER(C.c_int64)],
     "aiq_result": [C.c_void_p, C.c_int64, C.POINTER(_View)],
@@ -195,6 +196,7 @@ class Result:
     prefill_flops: float
     n_launches: int
     n_prefill_tokens: int
+    row_ids_b: np.ndarray = None   # pair queries: B row of each yes pair
 
 
 @dataclass
@@ -334,7 +336,7 @@ class Context:
                      (s, k) if v.label_logits else (0, k)),
                 _arr(v.decisions, s if v.decisions else 0, np.int32),
                 v.ms_relational, v.ms_prefill, v.ms_aggregate, v.ms_total, v.prefill_flops, v.n_launches,
-                v.n_prefill_tokens)
+                v.n_prefill_tokens, _arr(v.row_ids_b, v.n_row_ids if v.row_ids_b else 0, np.int32))
         finally:
             self.lib.aiq_result_free(self.h, h)
 
@@ -354,6 +356,15 @@ class Context:
         h = C.c_int64()
         _check(self.lib.aiq_run_join_select(self.h, build.handle, build.col(build_key), bparr, nbp, probe.handle,
                                             probe.col(probe_key), model, C.byref(sel), C.byref(h)))
+        return self._fetch(h, len(labels))
+
+    def run_pair_select(self, table: TableRef, key: str, model: int, preds, prefix, labels,
+                        agg: int = AGG_ROW_IDS, flags: int = 0, text_name: str = "text") -> Result:
+        """Table 2 Q4: AI_IF over every (a < b) pair of selected rows with equal ``key``;
+        candidates are the pairs (cand_row_ids / cand_build_rows = A / B rows)."""
+        sel, keep = self._select(table, preds, prefix, labels, agg, flags, text_name)
+        h = C.c_int64()
+        _check(self.lib.aiq_run_pair_select(self.h, table.handle, table.col(key), model, C.byref(sel), C.byref(h)))
         return self._fetch(h, len(labels))
 
     def run_transform(self, table: TableRef, model: int, preds, prefix, max_new: int, eos: int = -1,

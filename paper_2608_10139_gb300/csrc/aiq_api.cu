@@ -99,7 +99,7 @@ struct ResultH {
   std::vector<int32_t> row_ids, group_rows, cand_ids, cand_build, decisions;
   std::vector<int64_t> group_keys, group_counts, label_counts;
   std::vector<float> logits;
-  std::vector<int32_t> gen_ids, gen_tok, gen_len;
+  std::vector<int32_t> gen_ids, gen_tok, gen_len, row_ids_b;
   int32_t gen_max_new = 0;
 };
 
@@ -550,7 +550,8 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
 
 struct QueryState {
   int64_t S = 0;
-  int32_t* ids = nullptr;        // candidate (probe) rows
+  int32_t* ids = nullptr;        // candidate (probe) rows; Q4 pairs: the A rows
+  int32_t* ids2 = nullptr;       // Q4 pairs: the B rows (their text follows A's)
   int32_t* build_rows = nullptr; // joins
   float* logits = nullptr;       // [S, K]
   int64_t T = 0, n_chunks = 0, pairs = 0;  // T: row tokens (prefix excluded)
@@ -745,7 +746,7 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
   CUDA_TRY(cudaMemsetAsync(pairs_d, 0, sizeof(unsigned long long), c->stream));
   {
     ProfScope p(c, "pack_plan", 0, 0);
-    launch_row_lengths(col.offsets, st->ids, S, P, lens, pairs_d, c->stream);
+    launch_row_lengths(col.offsets, st->ids, S, P, lens, pairs_d, c->stream, st->ids2);
     launch_scan_lengths(lens, S, cu, scan_scratch, c->stream);
     counted(c, 4);
   }
@@ -755,7 +756,7 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
   st->T = T;
   st->pairs = c->h_pin[1];
   st->P = P;
-  const int64_t max_len = col.max_len;  // longest row text; the prefix runs on its own
+  const int64_t max_len = col.max_len * (st->ids2 ? 2 : 1);  // longest row text; the prefix runs on its own
   int64_t budget = c->token_budget;
   if (gp) {
     // a chunk's rows decode together, one token each per step: size the chunks
@@ -817,7 +818,7 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
     {
       ProfScope p(c, "pack_chunk", 0, 0);
       launch_pack_chunk(cu, st->ids, col.offsets, static_cast<const int32_t*>(col.data), P, r0, r1, pb.tok, pb.pos,
-                        pb.seq_start, pb.last_idx, c->stream);
+                        pb.seq_start, pb.last_idx, c->stream, st->ids2);
       counted(c, 1);
     }
     // generation keeps every layer's prompt keys/values of the chunk for the decode steps
@@ -873,6 +874,15 @@ aiq_status aggregate_phase(aiq_ctx* c, const aiq_select* q, QueryState* st, cons
     counted(c, 2);
     R.row_ids.resize(Y);
     if (Y) CUDA_TRY(cudaMemcpyAsync(R.row_ids.data(), rows, Y * sizeof(int32_t), cudaMemcpyDeviceToHost, c->stream));
+    if (st->ids2) {  // Q4: the B row of every yes pair as well
+      int32_t* rows_b;
+      AIQ_TRY(ws(c, "a.rows_b", std::max<int64_t>(Y, 1), &rows_b));
+      launch_gather_rows_i32(st->ids2, 1, pos, Y, rows_b, c->stream);
+      counted(c, Y > 0);
+      R.row_ids_b.resize(Y);
+      if (Y)
+        CUDA_TRY(cudaMemcpyAsync(R.row_ids_b.data(), rows_b, Y * sizeof(int32_t), cudaMemcpyDeviceToHost, c->stream));
+    }
   }
   if (q->agg == AIQ_AGG_GROUP_BUILD_KEY) {
     const int64_t nbr = build->n_rows;
@@ -944,6 +954,7 @@ void finish_view(ResultH& R, const QueryState& st, int64_t n_input, int K, int a
   v.cand_build_rows = R.cand_build.empty() ? nullptr : R.cand_build.data();
   v.label_logits = R.logits.empty() ? nullptr : R.logits.data();
   v.decisions = R.decisions.empty() ? nullptr : R.decisions.data();
+  v.row_ids_b = R.row_ids_b.empty() ? nullptr : R.row_ids_b.data();
   v.gen_max_new = R.gen_max_new;
   v.n_gen_rows = static_cast<int64_t>(R.gen_ids.size());
   v.gen_row_ids = R.gen_ids.empty() ? nullptr : R.gen_ids.data();
@@ -1214,6 +1225,106 @@ aiq_status run_transform(aiq_ctx* c, const TableD& t, ModelD* m, const aiq_selec
                           2.0 * d * (qd + 2 * kd) * static_cast<double>(st.T) + tail * static_cast<double>(S) +
                           per_layer * pre +
                           4.0 * g.n_heads * g.head_dim * g.n_layers * (static_cast<double>(st.pairs) + pre * (pre + 1) / 2);
+  }
+  dst.v.n_launches = c->launches;
+  return AIQ_OK;
+}
+
+// Table 2 Q4: WHERE on the table, the key self-join into (a, b) pairs on the
+// device, then AI_IF on every pair's prompt and the aggregate over pairs.
+aiq_status run_pair_select(aiq_ctx* c, const TableD& t, int32_t key_col, ModelD* m, const aiq_select* q,
+                           aiq_result_h* out) {
+  if (q->flags & AIQ_FLAG_RELATIONAL_ONLY) return fail(AIQ_ERR_INVALID_ARG, "pair queries need the language model");
+  AIQ_TRY(validate_select(c, t, m, q));
+  AIQ_TRY(validate_prompt(t, m, q, t.cols[q->text_column].max_len));  // two texts per prompt
+  if (q->n_labels != 2) return fail(AIQ_ERR_INVALID_ARG, "pair queries need exactly 2 labels (yes, no)");
+  if (q->agg != AIQ_AGG_COUNT && q->agg != AIQ_AGG_ROW_IDS)
+    return fail(AIQ_ERR_INVALID_ARG, "pair queries aggregate with COUNT or ROW_IDS");
+  PredSet ps{};
+  AIQ_TRY(make_pred_set(t, q->preds, q->n_preds, &ps));
+
+  c->launches = 0;
+  cudaEvent_t ev[4];
+  for (auto& e : ev) e = take_event(c);
+  CUDA_TRY(cudaEventRecord(ev[0], c->stream));
+  int64_t S = 0;
+  int32_t* ids;
+  AIQ_TRY(filter_compact(c, t, ps, ProbeSpec{}, "sel", &S, &ids, nullptr));
+  // self-join on the key: stable radix sort of the candidates' keys, pair offsets, pairs
+  const int64_t tiles = (S + kRowsPerBlock - 1) / kRowsPerBlock;
+  const int64_t n1 = std::max<int64_t>(S, 1);
+  SelfJoinScratch w{};
+  AIQ_TRY(ws(c, "p.keys", n1, &w.keys));
+  AIQ_TRY(ws(c, "p.keys_tmp", n1, &w.keys_tmp));
+  AIQ_TRY(ws(c, "p.vals", n1, &w.vals));
+  AIQ_TRY(ws(c, "p.vals_tmp", n1, &w.vals_tmp));
+  AIQ_TRY(ws(c, "p.heads", n1, &w.heads));
+  AIQ_TRY(ws(c, "p.counts", n1, &w.counts));
+  AIQ_TRY(ws(c, "p.head_excl", S + 1, &w.head_excl));
+  AIQ_TRY(ws(c, "p.pair_off", S + 1, &w.pair_off));
+  AIQ_TRY(ws(c, "p.group_start", S + 1, &w.group_start));
+  AIQ_TRY(ws(c, "p.hist", 256 * std::max<int64_t>(tiles, 1), &w.hist));
+  AIQ_TRY(ws(c, "p.hist_off", 256 * std::max<int64_t>(tiles, 1) + 1, &w.hist_off));
+  const int64_t scan_n = std::max<int64_t>(S, 256 * tiles);
+  AIQ_TRY(ws(c, "p.scan", 2 * ((scan_n + kRowsPerBlock - 1) / kRowsPerBlock + 1), &w.scan_tmp));
+  {
+    ProfScope p(c, "self_join", 0, 0);
+    launch_self_join_pairs_plan(static_cast<const int64_t*>(t.cols[key_col].data), ids, S, w, c->stream);
+    counted(c, S > 0 ? 1 + 8 * 5 + 3 + 3 + 3 : 0);
+  }
+  int64_t n_pairs = 0;
+  if (S > 0) {
+    AIQ_TRY(read_i64(c, w.pair_off + S, 1, c->h_pin));
+    n_pairs = c->h_pin[0];
+  }
+  if (n_pairs > INT32_MAX) return fail(AIQ_ERR_CAPACITY, "more than 2^31 - 1 pairs");
+  QueryState st;
+  st.S = n_pairs;
+  AIQ_TRY(ws(c, "p.a", std::max<int64_t>(n_pairs, 1), &st.ids));
+  AIQ_TRY(ws(c, "p.b", std::max<int64_t>(n_pairs, 1), &st.ids2));
+  launch_self_join_pairs_emit(ids, S, w, st.ids, st.ids2, c->stream);
+  counted(c, S > 0);
+  CUDA_TRY(cudaEventRecord(ev[1], c->stream));
+
+  ResultH R;
+  if (q->flags & AIQ_FLAG_LOGITS) {
+    R.cand_ids.resize(n_pairs);
+    R.cand_build.resize(n_pairs);
+    if (n_pairs) {
+      CUDA_TRY(cudaMemcpyAsync(R.cand_ids.data(), st.ids, n_pairs * 4, cudaMemcpyDeviceToHost, c->stream));
+      CUDA_TRY(cudaMemcpyAsync(R.cand_build.data(), st.ids2, n_pairs * 4, cudaMemcpyDeviceToHost, c->stream));
+    }
+  }
+  AIQ_TRY(prefill_phase(c, t, *m, q, &st));
+  CUDA_TRY(cudaEventRecord(ev[2], c->stream));
+  AIQ_TRY(aggregate_phase(c, q, &st, nullptr, -1, R));
+  CUDA_TRY(cudaEventRecord(ev[3], c->stream));
+  AIQ_TRY(sync_and_check(c));
+  float t01 = 0, t12 = 0, t23 = 0, t03 = 0;
+  cudaEventElapsedTime(&t01, ev[0], ev[1]);
+  cudaEventElapsedTime(&t12, ev[1], ev[2]);
+  cudaEventElapsedTime(&t23, ev[2], ev[3]);
+  cudaEventElapsedTime(&t03, ev[0], ev[3]);
+  for (auto& e : ev) c->ev_pool.push_back(e);
+  collect_profile(c);
+  ResultH& dst = new_result(c, out);
+  dst = std::move(R);
+  finish_view(dst, st, t.n_rows, 2, q->agg);
+  dst.v.ms_relational = t01;
+  dst.v.ms_prefill = t12;
+  dst.v.ms_aggregate = t23;
+  dst.v.ms_total = t03;
+  {
+    const aiq_model_config& g = m->cfg;
+    const double pre = st.S > 0 ? static_cast<double>(st.P) : 0.0;
+    const double d = g.d_model, qd = double(g.n_heads) * g.head_dim, kd = double(g.n_kv_heads) * g.head_dim;
+    const double per_layer = m->linear_flops_per_token / g.n_layers;
+    const double tail = 2.0 * (qd * d + 3.0 * d * g.d_ffn);
+    dst.v.prefill_flops = per_layer * (g.n_layers - 1) * (static_cast<double>(st.T) + pre) +
+                          2.0 * d * (qd + 2 * kd) * static_cast<double>(st.T) + tail * static_cast<double>(st.S) +
+                          per_layer * pre +
+                          4.0 * g.n_heads * g.head_dim * g.n_layers * (static_cast<double>(st.pairs) + pre * (pre + 1) / 2) +
+                          2.0 * g.d_model * 2 * static_cast<double>(st.S);
   }
   dst.v.n_launches = c->launches;
   return AIQ_OK;
@@ -1539,6 +1650,20 @@ aiq_status aiq_run_transform(aiq_ctx* c, aiq_table table, aiq_model model, const
   if (mi == c->models.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown model handle");
   CUDA_TRY(cudaSetDevice(c->device));
   return run_transform(c, t->second, &mi->second, q, gen, out);
+}
+
+aiq_status aiq_run_pair_select(aiq_ctx* c, aiq_table table, int32_t key_column, aiq_model model,
+                               const aiq_select* q, aiq_result_h* out) {
+  if (!c || !q || !out) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
+  auto t = c->tables.find(table);
+  if (t == c->tables.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown table handle");
+  if (key_column < 0 || key_column >= static_cast<int32_t>(t->second.cols.size()) ||
+      t->second.cols[key_column].type != AIQ_INT64)
+    return fail(AIQ_ERR_INVALID_ARG, "key_column must be an INT64 column");
+  auto mi = c->models.find(model);
+  if (mi == c->models.end()) return fail(AIQ_ERR_NOT_FOUND, "unknown model handle");
+  CUDA_TRY(cudaSetDevice(c->device));
+  return run_pair_select(c, t->second, key_column, &mi->second, q, out);
 }
 
 aiq_status aiq_result(aiq_ctx* c, aiq_result_h h, aiq_result_view* out) {

@@ -72,9 +72,9 @@ struct DecCfg {
 // One block per (row, KV head): the G <= 8 query heads of the group against
 // all of the row's keys, on m16n8k16 tensor-core MMAs (the heads are the
 // rows of the A tile, the rest of its 16 rows are zero).  Warp w takes key
-// blocks w, w + 8, ... of 32 keys (16 at head_dim 128): it stages the block's
-// K and V rows in its own shared-memory slice with cp.async (all rows of both
-// at once), then
+// blocks w, w + 8, ... of 32 keys (16 at head_dim 128): it stages a block's K
+// and V rows in its own shared-memory slice with cp.async (all rows of both at
+// once), then
 // S = Q K^T, the online softmax on the accumulator fragments and O += P V
 // with V read through ldmatrix.trans.  The eight warps' partial (max, sum,
 // output) are merged at the end.

@@ -93,8 +93,9 @@ void launch_fill_u64(unsigned long long* p, int64_t n, unsigned long long v, cud
 // ------------------------------------------------------------------ pack ---
 // lens[i] = text length of row ids[i]; *pairs += causal (q, k) pairs of its tokens
 // (prefix keys included).
+// ids2 (optional): a second row per sequence whose text follows the first's (Q4 pairs).
 void launch_row_lengths(const int64_t* offsets, const int32_t* ids, int64_t S, int32_t prefix_len, int32_t* lens,
-                        unsigned long long* pairs, cudaStream_t s);
+                        unsigned long long* pairs, cudaStream_t s, const int32_t* ids2 = nullptr);
 // Exclusive scan of int32 lengths into int64 cu[S+1] (multi-block).
 void launch_scan_lengths(const int32_t* lens, int64_t S, int64_t* cu, int64_t* scratch_blocks, cudaStream_t s);
 // chunk_rows[c] = first row whose start offset >= c * budget_step, c = 0..n_chunks.
@@ -104,7 +105,7 @@ void launch_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64_t n_c
 // chunk-local sequence starts and last-token index (-1 for a row without tokens).
 void launch_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,
                        int32_t prefix_len, int64_t r0, int64_t r1, int32_t* tok, int32_t* pos, int32_t* seq_start,
-                       int32_t* last_idx, cudaStream_t s);
+                       int32_t* last_idx, cudaStream_t s, const int32_t* ids2 = nullptr);
 // The shared prefix as a single sequence at positions 0..P-1.
 void launch_pack_prefix(const int32_t* prefix, int32_t P, int32_t* tok, int32_t* pos, int32_t* seq_start,
                         cudaStream_t s);
@@ -183,6 +184,26 @@ void launch_like_match(const int32_t* gen_tok, const int32_t* gen_len, int64_t S
                        int plen, int32_t* match, cudaStream_t s);
 void launch_gather_rows_i32(const int32_t* src, int width, const int32_t* pos, int64_t n, int32_t* out,
                             cudaStream_t s);
+// ---------------------------------------------------------------- pairs ---
+// Device scratch of the Q4 self-join over S candidates (sizes in elements):
+// keys, keys_tmp [S] u64; vals, vals_tmp, heads, counts [S] i32; head_excl,
+// pair_off [S + 1] i64; group_start [S + 1] i64; hist [256 * tiles] i32,
+// hist_off [256 * tiles + 1] i64 (tiles = ceil(S / 2048)); scan_tmp
+// [2 * (ceil(max(S, 256 * tiles) / 2048) + 1)] i64.
+struct SelfJoinScratch {
+  uint64_t *keys, *keys_tmp;
+  int32_t *vals, *vals_tmp, *heads, *counts, *hist;
+  int64_t *head_excl, *pair_off, *group_start, *hist_off, *scan_tmp;
+};
+// Sort the candidates by key (stable), group them, and write pair_off: the
+// exclusive scan, in candidate order, of each candidate's pair count (its
+// group members after it); pair_off[S] is the number of pairs.
+void launch_self_join_pairs_plan(const int64_t* key_col, const int32_t* ids, int64_t S, const SelfJoinScratch& w,
+                                 cudaStream_t s);
+// (pa[k], pb[k]) = the k-th pair (a < b, equal keys), ascending (a, b).
+void launch_self_join_pairs_emit(const int32_t* ids, int64_t S, const SelfJoinScratch& w, int32_t* pa, int32_t* pb,
+                                 cudaStream_t s);
+
 // bits / per-block counts of the non-zero entries of an int32 flag array.
 void launch_flag_mask(const int32_t* flags, int64_t n, uint32_t* bits, int32_t* block_counts, cudaStream_t s);
 

@@ -2,8 +2,10 @@
 //
 // Every candidate row's prompt is the shared prefix followed by the row's
 // tokens (Table 1, AI_IF row: the text column feeds the causal LM; the prompt
-// prefix is the instruction shared by all rows).  The prefix is run through
-// the decoder once per query and its keys/values are reused by every row
+// prefix is the instruction shared by all rows); a Q4 pair's prompt is the
+// prefix followed by both rows' tokens (Table 2 Q4: AI_IF([A.text, B.text])).
+// The prefix is run through the decoder once per query and its keys/values
+// are reused by every row
 // (causal attention makes the prefix's states independent of what follows),
 // so the packed batch holds only each row's own tokens, at positions
 // P, P+1, ...  Rows are concatenated with no padding; cu (int64 [S+1]) holds
@@ -17,15 +19,17 @@
 namespace aiq {
 namespace {
 
-// lens[i] = text length of row ids[i]; pairs += len * P + len * (len + 1) / 2
-// (the causal query-key pairs its tokens attend, for the executed-FLOP count).
-__global__ void k_row_lengths(const int64_t* offsets, const int32_t* ids, int64_t S, int32_t P, int32_t* lens,
-                              unsigned long long* pairs) {
+// lens[i] = text length of row ids[i] (plus row ids2[i]'s for a pair prompt);
+// pairs += len * P + len * (len + 1) / 2 (the causal query-key pairs its tokens
+// attend, for the executed-FLOP count).
+__global__ void k_row_lengths(const int64_t* offsets, const int32_t* ids, const int32_t* ids2, int64_t S, int32_t P,
+                              int32_t* lens, unsigned long long* pairs) {
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   unsigned long long pr = 0;
   if (i < S) {
     const int32_t r = ids[i];
-    const int64_t len = offsets[r + 1] - offsets[r];
+    int64_t len = offsets[r + 1] - offsets[r];
+    if (ids2) len += offsets[ids2[i] + 1] - offsets[ids2[i]];
     lens[i] = static_cast<int32_t>(len);
     pr = static_cast<unsigned long long>(len * P + len * (len + 1) / 2);
   }
@@ -53,10 +57,11 @@ __global__ void k_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64
   out[2 * c + 1] = cu[lo];
 }
 
-// One warp per row: the row's tokens at positions P + j; a row with no tokens
-// of its own gets last_idx = -1 (its last position is the prefix's last).
-__global__ void k_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,
-                             int32_t P, int64_t r0, int64_t r1, int32_t* tok, int32_t* pos,
+// One warp per row: the row's tokens at positions P + j (for a pair prompt the
+// first row's text, then the second's); a row with no tokens of its own gets
+// last_idx = -1 (its last position is the prefix's last).
+__global__ void k_pack_chunk(const int64_t* cu, const int32_t* ids, const int32_t* ids2, const int64_t* offsets,
+                             const int32_t* text, int32_t P, int64_t r0, int64_t r1, int32_t* tok, int32_t* pos,
                              int32_t* seq_start, int32_t* last_idx) {
   const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
@@ -67,8 +72,10 @@ __global__ void k_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_
   const int64_t len = cu[i + 1] - cu[i];
   const int32_t r = ids[i];
   const int32_t* src = text + offsets[r];
+  const int64_t len_a = ids2 ? offsets[r + 1] - offsets[r] : len;
+  const int64_t off_b = ids2 ? offsets[ids2[i]] : 0;
   for (int64_t j = lane; j < len; j += 32) {
-    tok[dst + j] = src[j];
+    tok[dst + j] = j < len_a ? src[j] : text[off_b + (j - len_a)];
     pos[dst + j] = static_cast<int32_t>(P + j);
   }
   if (lane == 0) {
@@ -125,9 +132,9 @@ void launch_pack_prefix(const int32_t* prefix, int32_t P, int32_t* tok, int32_t*
 }
 
 void launch_row_lengths(const int64_t* offsets, const int32_t* ids, int64_t S, int32_t prefix_len, int32_t* lens,
-                        unsigned long long* pairs, cudaStream_t s) {
+                        unsigned long long* pairs, cudaStream_t s, const int32_t* ids2) {
   if (S <= 0) return;
-  k_row_lengths<<<static_cast<unsigned>((S + 255) / 256), 256, 0, s>>>(offsets, ids, S, prefix_len, lens, pairs);
+  k_row_lengths<<<static_cast<unsigned>((S + 255) / 256), 256, 0, s>>>(offsets, ids, ids2, S, prefix_len, lens, pairs);
 }
 
 void launch_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64_t n_chunks, int64_t* chunk_rows,
@@ -137,11 +144,11 @@ void launch_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64_t n_c
 
 void launch_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,
                        int32_t prefix_len, int64_t r0, int64_t r1, int32_t* tok, int32_t* pos, int32_t* seq_start,
-                       int32_t* last_idx, cudaStream_t s) {
+                       int32_t* last_idx, cudaStream_t s, const int32_t* ids2) {
   if (r1 <= r0) return;
   const int64_t threads = (r1 - r0) * 32;
-  k_pack_chunk<<<static_cast<unsigned>((threads + 255) / 256), 256, 0, s>>>(cu, ids, offsets, text, prefix_len, r0, r1,
-                                                                            tok, pos, seq_start, last_idx);
+  k_pack_chunk<<<static_cast<unsigned>((threads + 255) / 256), 256, 0, s>>>(cu, ids, ids2, offsets, text, prefix_len,
+                                                                            r0, r1, tok, pos, seq_start, last_idx);
 }
 
 void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t tile_tokens, int32_t* tile_seq,

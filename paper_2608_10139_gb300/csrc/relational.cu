@@ -15,6 +15,8 @@
 //    yes-row ids, GROUP BY build row with warp-aggregated atomics.
 #include <cstdio>
 
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -217,41 +219,57 @@ constexpr int kCompactWarps = 4;  // warps (= 2048-row tiles) per compaction blo
 // in the warp's own shared-memory slice in order and then written out as one
 // coalesced run.  No block-wide barrier is involved.  A payload (the join's
 // build row per probe row) is gathered straight to its output position.
+// Warps are persistent over the tiles (grid-stride) and load the next tile's
+// bitmask words and output offset before they work on the current one, so
+// two tiles' loads are in flight per warp.
 __global__ void __launch_bounds__(kCompactWarps * 32) k_compact(const uint32_t* bits, const int64_t* block_offsets,
                                                                 int64_t n, int32_t* ids, const int32_t* payload,
                                                                 int32_t* payload_out) {
   __shared__ int32_t s_ids[kCompactWarps][kRowsPerBlock];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t tile = static_cast<int64_t>(blockIdx.x) * kCompactWarps + warp;
   const int64_t n_tiles = (n + kRowsPerBlock - 1) / kRowsPerBlock;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kCompactWarps;
+  int64_t tile = static_cast<int64_t>(blockIdx.x) * kCompactWarps + warp;
   if (tile >= n_tiles) return;
-  const uint2 w2 = reinterpret_cast<const uint2*>(bits + tile * (kRowsPerBlock / 32))[lane];
-  const int c = __popc(w2.x) + __popc(w2.y);
-  int incl = c;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += y;
-  }
-  const int total = __shfl_sync(0xffffffffu, incl, 31);
-  int at = incl - c;
-  const int64_t out = block_offsets[tile];
-  const int64_t r0 = tile * kRowsPerBlock + lane * 64;
-  uint32_t wd[2] = {w2.x, w2.y};
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    uint32_t b = wd[h];
-    while (b) {
-      const int j = __ffs(b) - 1;
-      b &= b - 1;
-      const int64_t r = r0 + 32 * h + j;
-      s_ids[warp][at] = static_cast<int32_t>(r);
-      if (payload_out) payload_out[out + at] = payload[r];  // joins: a gather, written in place
-      ++at;
+  uint2 w2 = reinterpret_cast<const uint2*>(bits + tile * (kRowsPerBlock / 32))[lane];
+  int64_t out = block_offsets[tile];
+  for (; tile < n_tiles; tile += stride) {
+    const int64_t next = tile + stride;
+    uint2 w2n = make_uint2(0u, 0u);
+    int64_t out_n = 0;
+    if (next < n_tiles) {
+      w2n = reinterpret_cast<const uint2*>(bits + next * (kRowsPerBlock / 32))[lane];
+      out_n = block_offsets[next];
     }
+    const int c = __popc(w2.x) + __popc(w2.y);
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    const int total = __shfl_sync(0xffffffffu, incl, 31);
+    int at = incl - c;
+    const int64_t r0 = tile * kRowsPerBlock + lane * 64;
+    uint32_t wd[2] = {w2.x, w2.y};
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      uint32_t b = wd[h];
+      while (b) {
+        const int j = __ffs(b) - 1;
+        b &= b - 1;
+        const int64_t r = r0 + 32 * h + j;
+        s_ids[warp][at] = static_cast<int32_t>(r);
+        if (payload_out) payload_out[out + at] = payload[r];  // joins: a gather, written in place
+        ++at;
+      }
+    }
+    __syncwarp();
+    for (int i = lane; i < total; i += 32) ids[out + i] = s_ids[warp][i];
+    __syncwarp();  // the slice is rewritten by the next tile
+    w2 = w2n;
+    out = out_n;
   }
-  __syncwarp();
-  for (int i = lane; i < total; i += 32) ids[out + i] = s_ids[warp][i];
 }
 
 // ---------------------------------------------------------------- scans ---
@@ -460,8 +478,15 @@ void launch_scan_counts(const int32_t* counts, int64_t n, int64_t* offsets, cuda
 void launch_compact(const uint32_t* bits, const int64_t* block_offsets, int64_t n_rows, int32_t* ids_out,
                     const int32_t* payload, int32_t* payload_out, cudaStream_t s) {
   if (n_rows <= 0) return;
-  k_compact<<<blocks_for(n_rows, int64_t(kRowsPerBlock) * kCompactWarps), kCompactWarps * 32, 0, s>>>(
-      bits, block_offsets, n_rows, ids_out, payload, payload_out);
+  // persistent warps: as many blocks as fit on the device at once, at most one warp per tile
+  int dev = 0, sms = 0, per_sm = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_compact, kCompactWarps * 32, 0);
+  const int64_t need = blocks_for(n_rows, int64_t(kRowsPerBlock) * kCompactWarps);
+  const int64_t resident = std::max<int64_t>(1, static_cast<int64_t>(sms) * std::max(per_sm, 1));
+  const unsigned grid = static_cast<unsigned>(std::min<int64_t>(need, resident));
+  k_compact<<<grid, kCompactWarps * 32, 0, s>>>(bits, block_offsets, n_rows, ids_out, payload, payload_out);
 }
 
 void launch_hash_build(const int64_t* keys, const int32_t* rows, int64_t n, unsigned long long* table_keys,

@@ -136,6 +136,30 @@ C4_MULTILABEL = Workload(
     label_ids=(100, 101, 102, 103, 104), agg=AGG_GROUP_LABEL,
     data_seed=1004, weight_seed=2004)
 
+# Table 2 Q4 (pairwise AI_IF over the reviews self-joined on movie id): 20,000
+# reviews spread uniformly over 2,000 movies (about 10 per movie; a skewed key
+# would make the pair count quadratic in the head movie), score uniform 0..99,
+# the filter score < 40 on both sides, the select workload's text recipe.
+@dataclass(frozen=True)
+class PairWorkload:
+    name: str
+    n_rows: int
+    n_movies: int
+    text: TextRecipe
+    score_below: int
+    prefix_len: int
+    model: ModelShape
+    label_ids: Tuple[int, ...]
+    data_seed: int
+    weight_seed: int
+
+
+Q4_PAIRS = PairWorkload(
+    name="q4_pairs_1b", n_rows=20_000, n_movies=2_000,
+    text=TextRecipe("lognormal", 16, 512, median=120.0), score_below=40, prefix_len=64,
+    model=SHAPE_1B, label_ids=(YES_ID, NO_ID), data_seed=1006, weight_seed=2002)
+
+
 # Selectivity sweep thresholds ``rating >= R AND year >= Y`` on the c2 schema:
 # P(rating>=R) * P(year>=Y) with rating uniform 1..5 and year uniform 1950..2024.
 SWEEP_POINTS = {

@@ -22,7 +22,7 @@ from typing import Dict, List, Optional, Tuple
 
 import numpy as np
 
-from .configs import COLUMN_RANGES, ModelShape, TextRecipe, Workload
+from .configs import COLUMN_RANGES, ModelShape, PairWorkload, TextRecipe, Workload
 
 
 # ---------------------------------------------------------------- tables ---
@@ -122,6 +122,19 @@ def make_join_inputs(w: Workload) -> QueryInputs:
     movies = Table(m, {"movie_id": movie_id, "year": year})
     reviews = Table(w.n_rows, {"movie_id": fk}, offsets, tokens)
     return QueryInputs(reviews, prefix, build=movies)
+
+
+def make_pair_inputs(w: PairWorkload) -> QueryInputs:
+    """reviews(movie_id int64 uniform over n_movies distinct 63-bit ids,
+    score int32 uniform 0..99, text) for the Q4 self-join.  Draw order:
+    movie ids, the movie of each review, scores, text lengths, tokens, prefix."""
+    rng = np.random.Generator(np.random.PCG64(w.data_seed))
+    movie_ids = distinct_int63(rng, w.n_movies)
+    movie = movie_ids[rng.integers(0, w.n_movies, w.n_rows)]
+    score = rng.integers(0, 100, w.n_rows).astype(np.int32)
+    offsets, tokens = _text_column(rng, w.n_rows, w.text, w.model.vocab)
+    prefix = rng.integers(0, w.model.vocab, w.prefix_len).astype(np.int32)
+    return QueryInputs(Table(w.n_rows, {"movie_id": movie, "score": score}, offsets, tokens), prefix)
 
 
 def make_inputs(w: Workload) -> QueryInputs:
