@@ -50,7 +50,7 @@ def parse():
     p.add_argument("--rows", type=int, default=0, help="override the table size (testing)")
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--cpu-sample-rows", type=int, default=12)
+    p.add_argument("--cpu-sample-rows", type=int, default=64)
     p.add_argument("--micro", default="", choices=["", "relational"],
                    help="relational: predicate + compaction alone on a 2^28-row table, against HBM bandwidth")
     p.add_argument("--micro-rows", type=int, default=1 << 28)
