@@ -6,7 +6,8 @@ CUDA library and its Python binding) never imports this package, and this
 package never imports the product.  Inputs come from the ``synth`` generator.
 
 Parity status per function:
-  relational.*            pinned (brute force, invariants, hand-worked cases)
+  relational.*            pinned (brute force, invariants, hand-worked cases;
+                          masked_sum: hand cases, exact integers, fsum vs sorted sums)
   transformer.rmsnorm     pinned (closed form on constant rows, torch rms_norm)
   transformer.rope        pinned (rotation closed form, relative invariance)
   transformer.causal_attention  pinned (torch SDPA, identical-key prefix mean)

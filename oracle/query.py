@@ -28,7 +28,7 @@ import numpy as np
 from . import relational as rel
 from . import transformer as tf
 
-AGG_COUNT, AGG_ROW_IDS, AGG_GROUP_LABEL, AGG_GROUP_BUILD_KEY = 0, 1, 2, 3
+AGG_COUNT, AGG_ROW_IDS, AGG_GROUP_LABEL, AGG_GROUP_BUILD_KEY, AGG_SUM = 0, 1, 2, 3, 4
 
 
 @dataclass
@@ -50,12 +50,15 @@ def prompts(prefix: np.ndarray, offsets: np.ndarray, tokens: np.ndarray,
 
 def aggregate(agg: int, decision: np.ndarray, cand_rows: np.ndarray, k: int,
               cand_build_rows: Optional[np.ndarray] = None,
-              build_keys: Optional[np.ndarray] = None) -> dict:
+              build_keys: Optional[np.ndarray] = None,
+              sum_values: Optional[np.ndarray] = None) -> dict:
     """Masked aggregate over a full decision vector (Table 1, SELECT row)."""
     out = {}
     if k == 2:
         out["count"] = rel.count_yes(decision)
-    if agg == AGG_ROW_IDS:
+    if agg == AGG_SUM:
+        out["sum"] = rel.masked_sum(decision, cand_rows, sum_values)
+    elif agg == AGG_ROW_IDS:
         out["row_ids"] = rel.yes_row_ids(decision, cand_rows)
     elif agg == AGG_GROUP_LABEL:
         out["label_counts"] = rel.group_label_counts(decision, k)

@@ -150,6 +150,18 @@ def yes_row_ids(decision: np.ndarray, cand_rows: np.ndarray) -> np.ndarray:
     return np.array([int(r) for r, d in zip(cand_rows, decision) if d == 1], dtype=np.int32)
 
 
+def masked_sum(decision: np.ndarray, cand_rows: np.ndarray, values: np.ndarray):
+    """Fig. 2 / Table 1 SELECT row: SUM(values) over the rows decided yes (the
+    masked reduction ``where(filter, values, 0).sum()``).  Integer columns sum
+    exactly (Python integers); float columns are summed with correct rounding
+    (math.fsum of the exact float64 values)."""
+    import math
+    picked = [values[int(r)] for r, d in zip(cand_rows, decision) if d == 1]
+    if np.issubdtype(np.asarray(values).dtype, np.integer):
+        return sum(int(v) for v in picked)
+    return math.fsum(float(v) for v in picked)
+
+
 def group_label_counts(decision: np.ndarray, k: int) -> np.ndarray:
     """GROUP BY label COUNT(*), all K labels including empty ones."""
     counts = np.zeros(k, dtype=np.int64)

@@ -122,3 +122,20 @@ def test_aggregate_invariants():
     dec5 = rng.integers(0, 5, s).astype(np.int32)
     lc = oq.aggregate(oq.AGG_GROUP_LABEL, dec5, cand, 5)["label_counts"]
     assert lc.sum() == s and lc.tolist() == [int(np.sum(dec5 == k)) for k in range(5)]
+
+
+def test_masked_sum_hand_cases_and_exactness():
+    dec = np.array([1, 0, 1, 1], np.int32)
+    cand = np.array([0, 2, 3, 5], np.int32)
+    vals = np.array([10, 20, 30, 40, 50, 60], np.int32)
+    assert rel.masked_sum(dec, cand, vals) == 10 + 40 + 60
+    assert rel.masked_sum(np.zeros(4, np.int32), cand, vals) == 0
+    big = np.array([2 ** 62, 2 ** 62, -5], np.int64)                       # exact beyond float64
+    assert rel.masked_sum(np.ones(3, np.int32), np.arange(3), big) == 2 ** 63 - 5
+    f = np.array([1e16, 1.0, -1e16, 1.0], np.float32)                       # cancellation: exact sum 2
+    assert rel.masked_sum(np.ones(4, np.int32), np.arange(4), f) == 2.0
+    r = np.random.default_rng(5).standard_normal(1000).astype(np.float32)
+    exact = rel.masked_sum(np.ones(1000, np.int32), np.arange(1000), r)
+    assert abs(exact - float(np.sum(np.sort(r.astype(np.float64))))) < 1e-9
+    agg = oq.aggregate(oq.AGG_SUM, dec, cand, 2, sum_values=vals)
+    assert agg == {"count": 3, "sum": 110}
