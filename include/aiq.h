@@ -77,7 +77,10 @@ typedef enum {
   AIQ_AGG_COUNT = 0,          /* COUNT(*) of rows decided "yes" (2 labels) */
   AIQ_AGG_ROW_IDS = 1,        /* ids of the "yes" rows, ascending, and their count */
   AIQ_AGG_GROUP_LABEL = 2,    /* GROUP BY predicted label COUNT(*), all labels */
-  AIQ_AGG_GROUP_BUILD_KEY = 3 /* joins: GROUP BY build-side key COUNT(*) of "yes" rows */
+  AIQ_AGG_GROUP_BUILD_KEY = 3, /* joins: GROUP BY build-side key COUNT(*) of "yes" rows */
+  AIQ_AGG_SUM = 4              /* SUM(sum_column) over the "yes" rows, and their count (Fig. 2's
+                                  masked reduction); integer columns sum exactly in int64 (wrapping
+                                  on overflow), FLOAT32 columns in fp64 in a fixed order */
 } aiq_agg;
 
 enum {
@@ -100,6 +103,7 @@ typedef struct {
   int32_t n_labels;
   int32_t agg;   /* aiq_agg */
   int32_t flags; /* AIQ_FLAG_* */
+  int32_t sum_column; /* AIQ_AGG_SUM: index of an INT32, INT64 or FLOAT32 column (else ignored) */
 } aiq_select;
 
 /* Result view.  Pointers are host memory owned by the result; valid until
@@ -139,6 +143,10 @@ typedef struct {
   float ms_decode;            /* device time of the decode steps (inside ms_prefill) */
   double decode_flops;        /* 2*params per decoded token + attention over cached keys + full LM head */
   int64_t n_decode_steps;     /* sum over prefill chunks of max_new_tokens */
+  /* AIQ_AGG_SUM: the sum (sum_int for INT32 / INT64 columns, sum_float for FLOAT32); with
+   * count == 0 it is 0 (SQL's NULL) */
+  int64_t sum_int;
+  double sum_float;
 } aiq_result_view;
 
 typedef struct aiq_ctx aiq_ctx;

@@ -20,7 +20,7 @@ OK, ERR_INVALID_ARG, ERR_NOT_FOUND, ERR_OOM, ERR_CUDA, ERR_CAPACITY, ERR_DEVICE_
     0, -1, -2, -3, -4, -5, -6, -7
 INT32, INT64, FLOAT32, TOKENS = 0, 1, 2, 3
 LT, LE, GT, GE, EQ, NE = 0, 1, 2, 3, 4, 5
-AGG_COUNT, AGG_ROW_IDS, AGG_GROUP_LABEL, AGG_GROUP_BUILD_KEY = 0, 1, 2, 3
+AGG_COUNT, AGG_ROW_IDS, AGG_GROUP_LABEL, AGG_GROUP_BUILD_KEY, AGG_SUM = 0, 1, 2, 3, 4
 FLAG_LOGITS, FLAG_RELATIONAL_ONLY = 1, 2
 GEN_MATCH_TOKENS = 1
 EPI_F16, EPI_ROPE_F16, EPI_RESID_F32, EPI_SWIGLU_F16 = 0, 1, 2, 3
@@ -50,7 +50,7 @@ class _Select(C.Structure):
     _fields_ = [("preds", C.POINTER(_Pred)), ("n_preds", C.c_int32), ("text_column", C.c_int32),
                 ("prefix", C.POINTER(C.c_int32)), ("prefix_len", C.c_int32),
                 ("label_ids", C.POINTER(C.c_int32)), ("n_labels", C.c_int32), ("agg", C.c_int32),
-                ("flags", C.c_int32)]
+                ("flags", C.c_int32), ("sum_column", C.c_int32)]
 
 
 class _View(C.Structure):
@@ -67,7 +67,8 @@ class _View(C.Structure):
                 ("n_prefill_tokens", C.c_int64), ("row_ids_b", C.POINTER(C.c_int32)),
                 ("gen_max_new", C.c_int32), ("n_gen_rows", C.c_int64), ("gen_row_ids", C.POINTER(C.c_int32)),
                 ("gen_tokens", C.POINTER(C.c_int32)), ("gen_text_len", C.POINTER(C.c_int32)),
-                ("ms_decode", C.c_float), ("decode_flops", C.c_double), ("n_decode_steps", C.c_int64)]
+                ("ms_decode", C.c_float), ("decode_flops", C.c_double), ("n_decode_steps", C.c_int64),
+                ("sum_int", C.c_int64), ("sum_float", C.c_double)]
 
 
 class _Generate(C.Structure):
@@ -168,6 +169,7 @@ class TableRef:
     handle: int
     n_rows: int
     names: List[str]
+    types: List[int] = None
 
     def col(self, name: str) -> int:
         return self.names.index(name)
@@ -197,6 +199,7 @@ class Result:
     n_launches: int
     n_prefill_tokens: int
     row_ids_b: np.ndarray = None   # pair queries: B row of each yes pair
+    sum: object = None             # AGG_SUM: int (integer column) or float
 
 
 @dataclass
@@ -231,6 +234,8 @@ class Context:
     """One library context on one CUDA device (its own stream and buffers)."""
 
     def __init__(self, device: int = 0):
+        self._sum_float = False
+        self._sum = None
         self.lib = load_library()
         h = C.c_void_p()
         _check(self.lib.aiq_init(device, C.byref(h)))
@@ -260,6 +265,7 @@ class Context:
         keep = []
         specs = []
         names = []
+        types = []
         n = n_rows
         for name, a in cols.items():
             a = np.ascontiguousarray(a)
@@ -270,6 +276,7 @@ class Context:
             keep.append(a)
             specs.append(_Column(name.encode(), t, a.ctypes.data, None))
             names.append(name)
+            types.append(t)
         if text is not None:
             off = np.ascontiguousarray(text[0], dtype=np.int64)
             ids = _i32(text[1])
@@ -278,10 +285,11 @@ class Context:
             specs.append(_Column(text_name.encode(), TOKENS, ids.ctypes.data if ids.size else off.ctypes.data,
                                  off.ctypes.data))
             names.append(text_name)
+            types.append(TOKENS)
         arr = (_Column * len(specs))(*specs)
         h = C.c_int64()
         _check(self.lib.aiq_load_table(self.h, arr, len(specs), n or 0, C.byref(h)))
-        return TableRef(h.value, n or 0, names)
+        return TableRef(h.value, n or 0, names, types)
 
     def free_table(self, t: TableRef):
         _check(self.lib.aiq_free_table(self.h, t.handle))
@@ -309,13 +317,14 @@ class Context:
         arr = (_Pred * max(len(ps), 1))(*ps)
         return arr, len(ps)
 
-    def _select(self, t: TableRef, preds, prefix, labels, agg, flags, text_name):
+    def _select(self, t: TableRef, preds, prefix, labels, agg, flags, text_name, sum_column=None):
         parr, np_ = self._preds(t, preds)
         prefix = _i32(prefix)
         labels = _i32(labels)
         sel = _Select(parr, np_, t.col(text_name) if text_name in t.names else -1,
                       prefix.ctypes.data_as(C.POINTER(C.c_int32)), len(prefix),
-                      labels.ctypes.data_as(C.POINTER(C.c_int32)), len(labels), agg, flags)
+                      labels.ctypes.data_as(C.POINTER(C.c_int32)), len(labels), agg, flags,
+                      t.col(sum_column) if sum_column is not None else -1)
         return sel, (parr, prefix, labels)
 
     def _fetch(self, h: C.c_int64, k: int) -> Result:
@@ -323,6 +332,7 @@ class Context:
         try:
             _check(self.lib.aiq_result(self.h, h, C.byref(v)))
             s = v.n_candidates
+            self._sum = v.sum_float if self._sum_float else v.sum_int
             return Result(
                 v.n_input_rows, v.n_candidates, v.n_tokens, v.n_chunks, v.count,
                 _arr(v.row_ids, v.n_row_ids, np.int32),
@@ -336,14 +346,17 @@ class Context:
                      (s, k) if v.label_logits else (0, k)),
                 _arr(v.decisions, s if v.decisions else 0, np.int32),
                 v.ms_relational, v.ms_prefill, v.ms_aggregate, v.ms_total, v.prefill_flops, v.n_launches,
-                v.n_prefill_tokens, _arr(v.row_ids_b, v.n_row_ids if v.row_ids_b else 0, np.int32))
+                v.n_prefill_tokens, _arr(v.row_ids_b, v.n_row_ids if v.row_ids_b else 0, np.int32),
+                self._sum)
         finally:
             self.lib.aiq_result_free(self.h, h)
 
     def run_select(self, table: TableRef, model: int, preds, prefix, labels, agg: int = AGG_COUNT,
-                   flags: int = 0, text_name: str = "text") -> Result:
-        """preds: (column name, op, constant) triples, conjoined."""
-        sel, keep = self._select(table, preds, prefix, labels, agg, flags, text_name)
+                   flags: int = 0, text_name: str = "text", sum_column: Optional[str] = None) -> Result:
+        """preds: (column name, op, constant) triples, conjoined.  AGG_SUM sums
+        ``sum_column`` over the yes rows (Result.sum: int, or float for a FLOAT32 column)."""
+        self._sum_float = sum_column is not None and table.types[table.col(sum_column)] == FLOAT32
+        sel, keep = self._select(table, preds, prefix, labels, agg, flags, text_name, sum_column)
         h = C.c_int64()
         _check(self.lib.aiq_run_select(self.h, table.handle, model, C.byref(sel), C.byref(h)))
         return self._fetch(h, len(labels))
@@ -352,6 +365,7 @@ class Context:
                         model: int, preds, prefix, labels, agg: int = AGG_GROUP_BUILD_KEY, flags: int = 0,
                         text_name: str = "text") -> Result:
         bparr, nbp = self._preds(build, build_preds)
+        self._sum_float = False
         sel, keep = self._select(probe, preds, prefix, labels, agg, flags, text_name)
         h = C.c_int64()
         _check(self.lib.aiq_run_join_select(self.h, build.handle, build.col(build_key), bparr, nbp, probe.handle,
@@ -362,6 +376,7 @@ class Context:
                         agg: int = AGG_ROW_IDS, flags: int = 0, text_name: str = "text") -> Result:
         """Table 2 Q4: AI_IF over every (a < b) pair of selected rows with equal ``key``;
         candidates are the pairs (cand_row_ids / cand_build_rows = A / B rows)."""
+        self._sum_float = False
         sel, keep = self._select(table, preds, prefix, labels, agg, flags, text_name)
         h = C.c_int64()
         _check(self.lib.aiq_run_pair_select(self.h, table.handle, table.col(key), model, C.byref(sel), C.byref(h)))

@@ -100,6 +100,8 @@ struct ResultH {
   std::vector<int64_t> group_keys, group_counts, label_counts;
   std::vector<float> logits;
   std::vector<int32_t> gen_ids, gen_tok, gen_len, row_ids_b;
+  uint64_t sum_bits = 0;  // AIQ_AGG_SUM: int64 or double bits
+  bool sum_is_float = false;
   int32_t gen_max_new = 0;
 };
 
@@ -842,7 +844,7 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
 // ------------------------------------------------------- aggregate phase ---
 
 aiq_status aggregate_phase(aiq_ctx* c, const aiq_select* q, QueryState* st, const TableD* build, int32_t build_key,
-                           ResultH& R) {
+                           ResultH& R, const TableD* probe = nullptr) {
   const int K = q->n_labels;
   const int64_t S = st->S;
   const int64_t nb = (S + kRowsPerBlock - 1) / kRowsPerBlock;
@@ -883,6 +885,20 @@ aiq_status aggregate_phase(aiq_ctx* c, const aiq_select* q, QueryState* st, cons
       if (Y)
         CUDA_TRY(cudaMemcpyAsync(R.row_ids_b.data(), rows_b, Y * sizeof(int32_t), cudaMemcpyDeviceToHost, c->stream));
     }
+  }
+  if (q->agg == AIQ_AGG_SUM && probe) {
+    // Fig. 2: where(filter, values, 0).sum() over the candidates decided yes
+    const ColD& col = probe->cols[q->sum_column];
+    void *partial, *total;
+    AIQ_TRY(ws(c, "a.sum_part", std::max<int64_t>(nb, 1) * 8, reinterpret_cast<uint8_t**>(&partial)));
+    AIQ_TRY(ws(c, "a.sum", 8, reinterpret_cast<uint8_t**>(&total)));
+    {
+      ProfScope p(c, "masked_sum", 0, 0);
+      launch_masked_sum(dec, st->ids, col.data, col.type, S, partial, total, c->stream);
+      counted(c, 1 + (nb > 0));
+    }
+    R.sum_is_float = col.type == AIQ_FLOAT32;
+    CUDA_TRY(cudaMemcpyAsync(&R.sum_bits, total, 8, cudaMemcpyDeviceToHost, c->stream));
   }
   if (q->agg == AIQ_AGG_GROUP_BUILD_KEY) {
     const int64_t nbr = build->n_rows;
@@ -955,6 +971,9 @@ void finish_view(ResultH& R, const QueryState& st, int64_t n_input, int K, int a
   v.label_logits = R.logits.empty() ? nullptr : R.logits.data();
   v.decisions = R.decisions.empty() ? nullptr : R.decisions.data();
   v.row_ids_b = R.row_ids_b.empty() ? nullptr : R.row_ids_b.data();
+  v.sum_int = R.sum_is_float ? 0 : static_cast<int64_t>(R.sum_bits);
+  v.sum_float = 0.0;
+  if (R.sum_is_float) std::memcpy(&v.sum_float, &R.sum_bits, 8);
   v.gen_max_new = R.gen_max_new;
   v.n_gen_rows = static_cast<int64_t>(R.gen_ids.size());
   v.gen_row_ids = R.gen_ids.empty() ? nullptr : R.gen_ids.data();
@@ -990,7 +1009,13 @@ aiq_status validate_select(aiq_ctx* c, const TableD& t, const ModelD* m, const a
   if (q->n_labels < 2 || q->n_labels > 16 || !q->label_ids) return fail(AIQ_ERR_INVALID_ARG, "n_labels must be 2..16");
   for (int i = 0; i < q->n_labels; ++i)
     if (q->label_ids[i] < 0 || q->label_ids[i] >= V) return fail(AIQ_ERR_INVALID_ARG, "label id out of range");
-  if (q->agg < AIQ_AGG_COUNT || q->agg > AIQ_AGG_GROUP_BUILD_KEY) return fail(AIQ_ERR_INVALID_ARG, "unknown agg");
+  if (q->agg < AIQ_AGG_COUNT || q->agg > AIQ_AGG_SUM) return fail(AIQ_ERR_INVALID_ARG, "unknown agg");
+  if (q->agg == AIQ_AGG_SUM) {
+    if (q->n_labels != 2) return fail(AIQ_ERR_INVALID_ARG, "SUM needs exactly 2 labels (yes, no)");
+    if (q->sum_column < 0 || q->sum_column >= static_cast<int32_t>(t.cols.size()) ||
+        t.cols[q->sum_column].type == AIQ_TOKENS)
+      return fail(AIQ_ERR_INVALID_ARG, "sum_column must name an INT32, INT64 or FLOAT32 column");
+  }
   if ((q->agg == AIQ_AGG_COUNT || q->agg == AIQ_AGG_ROW_IDS) && q->n_labels != 2)
     return fail(AIQ_ERR_INVALID_ARG, "COUNT / ROW_IDS need exactly 2 labels (yes, no)");
   if (q->agg == AIQ_AGG_GROUP_BUILD_KEY && q->n_labels != 2)
@@ -1054,7 +1079,7 @@ aiq_status run_query(aiq_ctx* c, const TableD* build, int32_t build_key, const a
   if (!rel_only) {
     AIQ_TRY(prefill_phase(c, probe, *m, q, &st));
     CUDA_TRY(cudaEventRecord(ev[2], c->stream));
-    AIQ_TRY(aggregate_phase(c, q, &st, build, build_key, R));
+    AIQ_TRY(aggregate_phase(c, q, &st, build, build_key, R, &probe));
   } else {
     CUDA_TRY(cudaEventRecord(ev[2], c->stream));
   }

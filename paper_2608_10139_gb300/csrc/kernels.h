@@ -153,6 +153,12 @@ void launch_label_head(const float* resid, const int32_t* last_idx, const float*
 // yes-bitmask (K == 2), per-block yes counts, label counts [K] (int64, atomics).
 void launch_decide(const float* logits, int64_t S, int K, int32_t* decision, uint32_t* yes_bits,
                    int32_t* block_counts, unsigned long long* label_counts, cudaStream_t s);
+// Fig. 2's masked reduction: SUM(col[ids[i]]) over rows with decision[i] == 1,
+// deterministic (fixed-order block and final reductions).  type: 0 int32,
+// 1 int64 (exact int64 sum), 2 float32 (fp64 sum).  partial: >= ceil(S / 2048)
+// 8-byte slots; out: one 8-byte slot (int64 or double by type).
+void launch_masked_sum(const int32_t* decision, const int32_t* ids, const void* col, int type, int64_t S,
+                       void* partial, void* out, cudaStream_t s);
 // group counts[build_row] += 1 for yes rows.
 void launch_group_build(const int32_t* decision, const int32_t* cand_build_rows, int64_t S,
                         unsigned long long* group_counts, cudaStream_t s);

@@ -422,6 +422,44 @@ __global__ void __launch_bounds__(kThreads) k_flag_mask(const int32_t* flags, in
   if (threadIdx.x == 0) block_counts[blockIdx.x] = total;
 }
 
+// Fixed-order reductions (warp shuffle tree, then the warps in order) so that
+// the float sum is the same on every run.
+template <typename T>
+__device__ __forceinline__ T block_sum_fixed(T v, T* sh) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) sh[warp] = v;
+  __syncthreads();
+  T t = 0;
+  if (threadIdx.x == 0)
+    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) t += sh[w];
+  return t;
+}
+
+template <typename T, typename C>
+__global__ void __launch_bounds__(kThreads) k_masked_sum(const int32_t* decision, const int32_t* ids, const C* col,
+                                                         int64_t S, T* partial) {
+  __shared__ T sh[kThreads / 32];
+  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock + threadIdx.x * 8;
+  T acc = 0;
+  for (int j = 0; j < 8; ++j) {
+    const int64_t i = r0 + j;
+    if (i < S && decision[i] == 1) acc += static_cast<T>(col[ids[i]]);
+  }
+  const T t = block_sum_fixed<T>(acc, sh);
+  if (threadIdx.x == 0) partial[blockIdx.x] = t;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(1024) k_sum_final(const T* partial, int64_t n, T* out) {
+  __shared__ T sh[32];
+  T acc = 0;
+  for (int64_t i = threadIdx.x; i < n; i += 1024) acc += partial[i];
+  const T t = block_sum_fixed<T>(acc, sh);
+  if (threadIdx.x == 0) *out = t;
+}
+
 __global__ void k_group_build(const int32_t* decision, const int32_t* build_rows, int64_t S,
                               unsigned long long* counts) {
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
@@ -525,6 +563,26 @@ void launch_decide(const float* logits, int64_t S, int K, int32_t* decision, uin
 void launch_flag_mask(const int32_t* flags, int64_t n, uint32_t* bits, int32_t* block_counts, cudaStream_t s) {
   if (n <= 0) return;
   k_flag_mask<<<blocks_for(n, kRowsPerBlock), kThreads, 0, s>>>(flags, n, bits, block_counts);
+}
+
+void launch_masked_sum(const int32_t* decision, const int32_t* ids, const void* col, int type, int64_t S,
+                       void* partial, void* out, cudaStream_t s) {
+  const unsigned nb = S > 0 ? blocks_for(S, kRowsPerBlock) : 0;
+  if (type == 2) {
+    if (nb) k_masked_sum<double, float><<<nb, kThreads, 0, s>>>(decision, ids, static_cast<const float*>(col), S,
+                                                                 static_cast<double*>(partial));
+    k_sum_final<double><<<1, 1024, 0, s>>>(static_cast<const double*>(partial), nb, static_cast<double*>(out));
+  } else {
+    // integers sum modulo 2^64 (unsigned arithmetic: a wrap is defined), read back as int64
+    unsigned long long* pp = static_cast<unsigned long long*>(partial);
+    if (nb && type == 0)
+      k_masked_sum<unsigned long long, int32_t><<<nb, kThreads, 0, s>>>(decision, ids,
+                                                                         static_cast<const int32_t*>(col), S, pp);
+    if (nb && type == 1)
+      k_masked_sum<unsigned long long, long long><<<nb, kThreads, 0, s>>>(decision, ids,
+                                                                           static_cast<const long long*>(col), S, pp);
+    k_sum_final<unsigned long long><<<1, 1024, 0, s>>>(pp, nb, static_cast<unsigned long long*>(out));
+  }
 }
 
 void launch_group_build(const int32_t* decision, const int32_t* cand_build_rows, int64_t S,

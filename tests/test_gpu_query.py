@@ -232,3 +232,36 @@ def test_degenerate_queries(ctx):
     assert e.value.status == aiq.ERR_NOT_FOUND
     ctx.free_table(t)
     ctx.free_model(mh)
+
+
+def test_sum_aggregate_matches_oracle_on_gpu_decisions(ctx):
+    """Fig. 2's SELECT SUM(values) ... WHERE AI_IF(...) = 1: integer sums exact,
+    the float sum within fp64 rounding of the correctly rounded sum."""
+    w = synth.C1_TINY
+    q = synth.make_inputs(w)
+    W = synth.make_weights(w.model, w.weight_seed)
+    rng = np.random.default_rng(17)
+    n = q.table.n_rows
+    cols = dict(q.table.cols)
+    cols["v32"] = rng.integers(-2 ** 31, 2 ** 31 - 1, n).astype(np.int32)
+    cols["v64"] = rng.integers(-2 ** 50, 2 ** 50, n).astype(np.int64)
+    cols["vf"] = (rng.standard_normal(n) * 1e3).astype(np.float32)
+    m = ctx.load_model(w.model, weights_list(w.model, W))
+    t = ctx.load_table(cols, (q.table.offsets, q.table.tokens))
+    preds = oracle_preds(w.preds)
+    for name in ("v32", "v64", "vf"):
+        r = ctx.run_select(t, m, preds, q.prefix, w.label_ids, agg=aiq.AGG_SUM, flags=aiq.FLAG_LOGITS,
+                           sum_column=name)
+        want = rel.masked_sum(r.decisions, r.cand_row_ids, cols[name])
+        assert r.count == rel.count_yes(r.decisions)
+        if name == "vf":
+            bound = 1e-12 * float(np.abs(cols[name]).astype(np.float64).sum())
+            assert abs(r.sum - want) <= bound, (r.sum, want)
+        else:
+            assert r.sum == want
+    e = ctx.run_select(t, m, [("rating", rel.GT, 100)], q.prefix, w.label_ids, agg=aiq.AGG_SUM, sum_column="v64")
+    assert e.count == 0 and e.sum == 0
+    with pytest.raises(aiq.AiqError):
+        ctx.run_select(t, m, preds, q.prefix, w.label_ids, agg=aiq.AGG_SUM, sum_column="text")
+    ctx.free_table(t)
+    ctx.free_model(m)
