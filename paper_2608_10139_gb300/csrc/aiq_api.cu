@@ -764,9 +764,14 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
     // a chunk's rows decode together, one token each per step: size the chunks
     // for about decode_rows rows so that the decode GEMMs have M of that order,
     // within 2^20 tokens and 32 GB of cached prompt keys/values per chunk
+    // (and at most ~32 GB of generated-token keys/values per chunk: long
+    // generations decode fewer rows at a time)
     const int64_t per_row = T / S + 1;
-    const int64_t kv_cap = (int64_t(32) << 30) / (2 * int64_t(m.cfg.n_layers) * 2 * m.cfg.n_kv_heads * m.cfg.head_dim);
+    const int64_t kv_row = 2 * int64_t(m.cfg.n_layers) * 2 * m.cfg.n_kv_heads * m.cfg.head_dim;  // bytes/token
+    const int64_t kv_cap = (int64_t(32) << 30) / kv_row;
+    const int64_t gen_rows_cap = std::max<int64_t>(1, (int64_t(32) << 30) / (kv_row * std::max(gp->max_new - 1, 1)));
     budget = std::max(budget, std::min<int64_t>({c->decode_rows * per_row, int64_t(1) << 20, kv_cap}));
+    budget = std::min(budget, gen_rows_cap * per_row);
   }
   const int64_t B = std::max<int64_t>(std::max<int64_t>(budget, max_len), P);
   const int64_t step = B - max_len + 1;
