@@ -212,11 +212,15 @@ def ours(args):
     from paper_2608_10139_gb300 import build as _build
 
     rank, world, local = dist_env()
+    torch.cuda.set_device(local)
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
-    torch.cuda.set_device(local)
-    _build.build()
+    # one process compiles (an up-to-date library is left alone); the others wait for it
+    if local == 0:
+        _build.build()
+    if world > 1:
+        torch.distributed.barrier()
     w = workload(args)
     if world > 1:   # weak scaling: every rank owns its own shard of the job's table
         w = dataclasses.replace(w, data_seed=w.data_seed + 1000 * rank)
