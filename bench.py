@@ -172,6 +172,45 @@ def cpu_oracle_sample(w, q, W, n_rows: int, start: int = 0):
     return time.perf_counter() - t0, n_rows, len(o.cand_rows)
 
 
+def attention_flops_host(w, q) -> float:
+    """Algorithmic FLOPs of the prefill attention of one select query:
+    4 Hq hd per causal (query, key) pair per layer, every row attending the
+    shared prefix and its own earlier tokens, plus the prefix pass itself.
+    (Host arithmetic for the report only; 0 for the join workloads.)"""
+    if w.join_build_rows:
+        return 0.0
+    mask = np.ones(w.n_rows, dtype=bool)
+    ops = {0: np.less, 1: np.less_equal, 2: np.greater, 3: np.greater_equal, 4: np.equal, 5: np.not_equal}
+    for p in w.preds:
+        mask &= ops[p.op](q.table.cols[p.column].astype(np.int64), p.value)
+    lens = np.diff(q.table.offsets)[mask].astype(np.float64)
+    P = float(w.prefix_len)
+    pairs = float(np.sum(lens * P + lens * (lens + 1) / 2)) + (P * (P + 1) / 2 if mask.any() else 0.0)
+    s = w.model
+    return 4.0 * s.n_heads * s.head_dim * s.n_layers * pairs
+
+
+def kernel_rooflines(stats, steps, pk, attn_flops) -> dict:
+    """Per kernel class: device ms per step and the achieved rate against its
+    bound (tensor: TFLOP/s vs the sustained dense peak; HBM: GB/s vs the copy peak)."""
+    out = {}
+    tens = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+    for name, v in sorted(stats.items()):
+        ms = v["total_ms"]
+        if ms <= 0:
+            continue
+        e = {"ms_per_step": round(ms / steps, 3)}
+        flops = v["flops"] if v["flops"] else (attn_flops if name == "attention" else 0.0)
+        if flops:
+            a = flops / (ms / 1000.0) / 1e12
+            e.update(bound="tensor", achieved=round(a, 1), unit="TFLOP/s", frac=round(a / tens, 3))
+        elif v["bytes"]:
+            a = v["bytes"] / (ms / 1000.0) / 1e9
+            e.update(bound="hbm", achieved=round(a, 1), unit="GB/s", frac=round(a / pk["hbm_gbs"], 3))
+        out[name] = e
+    return out
+
+
 def reference_arm(args):
     """The CPU oracle as it stands, timed on this host's cores, on a bounded
     sample of the workload per step (rank 0 only)."""
@@ -281,6 +320,7 @@ def ours(args):
     achieved = gemm_flops / (gemm_ms / 1000.0) / 1e12 if gemm_ms else 0.0
     traffic = GEMM_TRAFFIC["bytes_per_launch"] if GEMM_TRAFFIC["source_sha"] == gemm_source_sha() else None
     step_ms = {k: round(v["total_ms"] / args.steps, 3) for k, v in sorted(stats.items())}
+    kernels = kernel_rooflines(stats, args.steps, pk, attention_flops_host(w, q) * args.steps)
 
     # end to end through the C-ABI with host buffers: upload table(s), query, download results
     e2e_ms, h2d, d2h = [], q.table.nbytes() + (q.build.nbytes() if q.build else 0), 0
@@ -329,6 +369,7 @@ def ours(args):
             "phase_ms": {"relational": res.ms_relational, "prefill": res.ms_prefill,
                          "aggregate": res.ms_aggregate},
             "kernel_ms_per_step": step_ms,
+            "kernels": kernels,
             "roofline": {"kernel": "gemm_tcgen05 (QKV+RoPE, O+residual, gate/up+SwiGLU, down+residual)",
                          "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                          "frac": achieved / peak if peak else None, "traffic": traffic,

@@ -474,7 +474,8 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
   // there than the kernel it removed.
   const int parts = d / 128;
   {
-    ProfScope p(c, "embed", 0, 0);
+    // bf16 row in; fp32 residual, fp16 copy and the partial sums of squares out
+    ProfScope p(c, "embed", 0, double(T) * d * 8.0 + double(T) * parts * 4.0);
     launch_embed(b.tok, T, m.embed, d, b.resid, b.xn, b.ss_attn, c->d_err, c->stream);
     counted(c, T > 0);
   }
@@ -515,7 +516,7 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
       e2.out = b.resid;
       AIQ_TRY(gemm(c, "gemm_o_resid", b.att, Hq * hd, L.wo, Hq * hd, M, d, Hq * hd, m.bn_o, e2));
       {
-        ProfScope p(c, "rmsnorm", 0, 0);
+        ProfScope p(c, "rmsnorm", 0, 6.0 * double(T) * d);  // fp32 in, fp16 out
         launch_rmsnorm(b.resid, T, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
         counted(c, T > 0);
       }
@@ -539,7 +540,7 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
       e2.out = b.resid_last;
       AIQ_TRY(gemm(c, "gemm_o_resid", b.qkv, Hq * hd, L.wo, Hq * hd, Mo, d, Hq * hd, m.bn_o, e2));
       {
-        ProfScope p(c, "rmsnorm", 0, 0);
+        ProfScope p(c, "rmsnorm", 0, 6.0 * double(Mo) * d);
         launch_rmsnorm(b.resid_last, Mo, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
         counted(c, Mo > 0);
       }
@@ -629,7 +630,7 @@ aiq_status decode_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const Deco
   const int64_t ldkv = 2 * static_cast<int64_t>(Hkv) * hd;
   const int parts = dm / 128;
   {
-    ProfScope p(c, "embed", 0, 0);
+    ProfScope p(c, "embed", 0, double(R) * dm * 8.0 + double(R) * parts * 4.0);
     launch_embed(d.next, R, m.embed, dm, b.resid, b.xn, b.ss_attn, c->d_err, c->stream);
     counted(c, 1);
   }
@@ -672,7 +673,7 @@ aiq_status decode_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const Deco
     e2.ss_parts = parts;
     AIQ_TRY(gemm(c, "dec_gemm_o_resid", b.att, Hq * hd, L.wo, Hq * hd, R, dm, Hq * hd, m.bn_o, e2));
     {
-      ProfScope p(c, "rmsnorm", 0, 0);
+      ProfScope p(c, "rmsnorm", 0, 6.0 * double(R) * dm);
       launch_rmsnorm(b.resid, R, dm, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
       counted(c, 1);
     }
@@ -696,7 +697,7 @@ aiq_status decode_chunk(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const Decod
   const aiq_model_config& g = m.cfg;
   launch_patch_empty_rows(b.resid_last, b.last_compact, prefix_last, R, g.d_model, c->stream);
   {
-    ProfScope p(c, "rmsnorm", 0, 0);
+    ProfScope p(c, "rmsnorm", 0, 6.0 * double(R) * g.d_model);
     launch_rmsnorm(b.resid_last, R, g.d_model, m.final_norm, g.rms_eps, b.xn, c->d_err, c->stream);
     counted(c, 2);
   }
@@ -704,7 +705,7 @@ aiq_status decode_chunk(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const Decod
   for (int t = 1; t < gp->max_new; ++t) {
     AIQ_TRY(decode_layers(c, m, b, d, R, Tc, pkv, P, t - 1));
     {
-      ProfScope p(c, "rmsnorm", 0, 0);
+      ProfScope p(c, "rmsnorm", 0, 6.0 * double(R) * g.d_model);
       launch_rmsnorm(b.resid, R, g.d_model, m.final_norm, g.rms_eps, b.xn, c->d_err, c->stream);
       counted(c, 1);
     }
