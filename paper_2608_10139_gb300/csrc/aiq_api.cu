@@ -760,27 +760,33 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
   st->pairs = c->h_pin[1];
   st->P = P;
   const int64_t max_len = col.max_len * (st->ids2 ? 2 : 1);  // longest row text; the prefix runs on its own
-  int64_t budget = c->token_budget;
+  int64_t n_chunks = 1, step = 0, rows_per_chunk = 0;
   if (gp) {
-    // a chunk's rows decode together, one token each per step: size the chunks
-    // for about decode_rows rows so that the decode GEMMs have M of that order,
-    // within 2^20 tokens and 32 GB of cached prompt keys/values per chunk
-    // (and at most ~32 GB of generated-token keys/values per chunk: long
-    // generations decode fewer rows at a time)
+    // a chunk's rows decode together, one token each per step: as few chunks
+    // of equal row counts as fit at most decode_rows rows, 2^20 tokens and
+    // ~32 GB of prompt keys/values each (and of generated-token keys/values:
+    // long generations decode fewer rows at a time).  (Splitting further to
+    // fill the decode GEMMs' last tile wave measured slower: more launches.)
     const int64_t per_row = T / S + 1;
     const int64_t kv_row = 2 * int64_t(m.cfg.n_layers) * 2 * m.cfg.n_kv_heads * m.cfg.head_dim;  // bytes/token
     const int64_t kv_cap = (int64_t(32) << 30) / kv_row;
     const int64_t gen_rows_cap = std::max<int64_t>(1, (int64_t(32) << 30) / (kv_row * std::max(gp->max_new - 1, 1)));
-    budget = std::max(budget, std::min<int64_t>({c->decode_rows * per_row, int64_t(1) << 20, kv_cap}));
-    budget = std::min(budget, gen_rows_cap * per_row);
+    const int64_t row_cap = std::max<int64_t>(
+        1, std::min<int64_t>({c->decode_rows, (int64_t(1) << 20) / per_row, kv_cap / per_row, gen_rows_cap}));
+    n_chunks = (S + row_cap - 1) / row_cap;
+    rows_per_chunk = (S + n_chunks - 1) / n_chunks;
+  } else {
+    const int64_t B = std::max<int64_t>(std::max<int64_t>(c->token_budget, max_len), P);
+    step = B - max_len + 1;
+    n_chunks = std::max<int64_t>(1, (T + step - 1) / step);
   }
-  const int64_t B = std::max<int64_t>(std::max<int64_t>(budget, max_len), P);
-  const int64_t step = B - max_len + 1;
-  const int64_t n_chunks = std::max<int64_t>(1, (T + step - 1) / step);
   st->n_chunks = n_chunks;
   int64_t* chunk_d;
   AIQ_TRY(ws(c, "q.chunks", 2 * (n_chunks + 1), &chunk_d));
-  launch_chunk_bounds(cu, S, step, n_chunks, chunk_d, c->stream);
+  if (gp)
+    launch_chunk_bounds_rows(cu, S, rows_per_chunk, n_chunks, chunk_d, c->stream);
+  else
+    launch_chunk_bounds(cu, S, step, n_chunks, chunk_d, c->stream);
   counted(c, 1);
   std::vector<int64_t> chunks(2 * (n_chunks + 1));
   CUDA_TRY(cudaMemcpyAsync(chunks.data(), chunk_d, chunks.size() * sizeof(int64_t), cudaMemcpyDeviceToHost, c->stream));

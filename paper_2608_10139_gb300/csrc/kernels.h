@@ -101,6 +101,9 @@ void launch_scan_lengths(const int32_t* lens, int64_t S, int64_t* cu, int64_t* s
 // chunk_rows[c] = first row whose start offset >= c * budget_step, c = 0..n_chunks.
 void launch_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64_t n_chunks, int64_t* chunk_rows,
                          cudaStream_t s);
+// Chunks of equal row counts: chunk_rows[2c] = min(c * rows_per_chunk, S), [2c+1] = cu[that row].
+void launch_chunk_bounds_rows(const int64_t* cu, int64_t S, int64_t rows_per_chunk, int64_t n_chunks,
+                              int64_t* chunk_rows, cudaStream_t s);
 // Pack rows [r0, r1) of a chunk: their own tokens at positions prefix_len + j,
 // chunk-local sequence starts and last-token index (-1 for a row without tokens).
 void launch_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,

@@ -57,6 +57,16 @@ __global__ void k_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64
   out[2 * c + 1] = cu[lo];
 }
 
+// chunk_rows[2c] = min(c * rows_per_chunk, S), chunk_rows[2c+1] = cu[that row].
+__global__ void k_chunk_bounds_rows(const int64_t* cu, int64_t S, int64_t rows_per_chunk, int64_t n_chunks,
+                                    int64_t* out) {
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (c > n_chunks) return;
+  const int64_t row = c * rows_per_chunk < S ? c * rows_per_chunk : S;
+  out[2 * c] = row;
+  out[2 * c + 1] = cu[row];
+}
+
 // One warp per row: the row's tokens at positions P + j (for a pair prompt the
 // first row's text, then the second's); a row with no tokens of its own gets
 // last_idx = -1 (its last position is the prefix's last).
@@ -140,6 +150,12 @@ void launch_row_lengths(const int64_t* offsets, const int32_t* ids, int64_t S, i
 void launch_chunk_bounds(const int64_t* cu, int64_t S, int64_t step, int64_t n_chunks, int64_t* chunk_rows,
                          cudaStream_t s) {
   k_chunk_bounds<<<static_cast<unsigned>((n_chunks + 1 + 127) / 128), 128, 0, s>>>(cu, S, step, n_chunks, chunk_rows);
+}
+
+void launch_chunk_bounds_rows(const int64_t* cu, int64_t S, int64_t rows_per_chunk, int64_t n_chunks,
+                              int64_t* chunk_rows, cudaStream_t s) {
+  k_chunk_bounds_rows<<<static_cast<unsigned>((n_chunks + 1 + 127) / 128), 128, 0, s>>>(cu, S, rows_per_chunk, n_chunks,
+                                                                                       chunk_rows);
 }
 
 void launch_pack_chunk(const int64_t* cu, const int32_t* ids, const int64_t* offsets, const int32_t* text,
