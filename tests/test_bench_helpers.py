@@ -1,0 +1,49 @@
+"""The benchmark's reporting arithmetic (CPU): the algorithmic attention FLOPs
+of a select query and the per-kernel roofline classification."""
+import importlib.util
+import os
+
+import numpy as np
+
+import synth
+from helpers import ROOT
+from oracle import relational as rel
+
+
+def _bench():
+    spec = importlib.util.spec_from_file_location("bench_mod", os.path.join(ROOT, "bench.py"))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    return mod
+
+
+def test_attention_flops_counts_causal_pairs_with_the_prefix():
+    b = _bench()
+    w = synth.C1_TINY
+    q = synth.make_inputs(w)
+    preds = [(p.column, p.op, p.value) for p in w.preds]
+    cand = rel.compact(rel.predicate_mask(q.table.cols, preds, q.table.n_rows))
+    P = w.prefix_len
+    # brute force: every row token attends the P prefix keys and its own earlier tokens
+    pairs = 0
+    for r in cand:
+        n = int(q.table.offsets[r + 1] - q.table.offsets[r])
+        pairs += sum(P + j + 1 for j in range(n))
+    pairs += P * (P + 1) // 2                      # the prefix pass, once per query
+    s = w.model
+    assert b.attention_flops_host(w, q) == 4.0 * s.n_heads * s.head_dim * s.n_layers * pairs
+
+
+def test_kernel_rooflines_bounds_and_fractions():
+    b = _bench()
+    pk = {"hbm_gbs": 6000.0, "bf16_tflops": 2000.0, "bf16_tflops_sustained": 1500.0}
+    stats = {"gemm_a": {"total_ms": 2.0, "flops": 3.0e12, "bytes": 0.0},
+             "rmsnorm": {"total_ms": 1.0, "flops": 0.0, "bytes": 3.0e9},
+             "attention": {"total_ms": 4.0, "flops": 0.0, "bytes": 0.0},
+             "pack_chunk": {"total_ms": 0.5, "flops": 0.0, "bytes": 0.0}}
+    k = b.kernel_rooflines(stats, 2, pk, attn_flops=1.2e12)
+    assert k["gemm_a"]["bound"] == "tensor" and np.isclose(k["gemm_a"]["achieved"], 1500.0)
+    assert np.isclose(k["gemm_a"]["frac"], 1.0)
+    assert k["rmsnorm"]["bound"] == "hbm" and np.isclose(k["rmsnorm"]["frac"], 0.5)
+    assert k["attention"]["bound"] == "tensor" and np.isclose(k["attention"]["achieved"], 300.0)
+    assert k["pack_chunk"] == {"ms_per_step": 0.25}
