@@ -23,7 +23,9 @@ typedef enum {
   AIQ_EPI_F16 = 0,       /* out fp16 [M, N] = A B^T */
   AIQ_EPI_ROPE_F16 = 1,  /* as F16, then rotary embedding on columns < rope_cols */
   AIQ_EPI_RESID_F32 = 2, /* out fp32 [M, N] += A B^T (residual stream update) */
-  AIQ_EPI_SWIGLU_F16 = 3 /* B rows interleave gate/up blocks of bn/2: out fp16 [M, N/2] = silu(g) * u */
+  AIQ_EPI_SWIGLU_F16 = 3, /* B rows interleave gate/up blocks of bn/2: out fp16 [M, N/2] = silu(g) * u */
+  AIQ_EPI_RESID_ADD_F32 = 5 /* as RESID_F32, the add done by TMA reduce-add tiles (out 16-byte aligned,
+                               ldo a multiple of 4) */
 } aiq_epilogue;
 
 /* A decoder linear layer on the tensor cores: A fp16 [M, K] (row pitch lda

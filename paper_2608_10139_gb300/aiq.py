@@ -23,7 +23,7 @@ LT, LE, GT, GE, EQ, NE = 0, 1, 2, 3, 4, 5
 AGG_COUNT, AGG_ROW_IDS, AGG_GROUP_LABEL, AGG_GROUP_BUILD_KEY, AGG_SUM = 0, 1, 2, 3, 4
 FLAG_LOGITS, FLAG_RELATIONAL_ONLY = 1, 2
 GEN_MATCH_TOKENS = 1
-EPI_F16, EPI_ROPE_F16, EPI_RESID_F32, EPI_SWIGLU_F16 = 0, 1, 2, 3
+EPI_F16, EPI_ROPE_F16, EPI_RESID_F32, EPI_SWIGLU_F16, EPI_RESID_ADD_F32 = 0, 1, 2, 3, 5
 
 
 class AiqError(RuntimeError):

@@ -294,7 +294,8 @@ inline void counted(aiq_ctx* c, int n) { c->launches += n; }
 
 aiq_status gemm(aiq_ctx* c, const char* name, const __half* A, int64_t lda, const __half* B, int64_t ldb, int M, int N,
                 int K, int bn, const GemmEpilogue& ep) {
-  const double out_bytes = (ep.kind == EPI_RESID_F32 ? 8.0 : (ep.kind == EPI_SWIGLU_F16 ? 1.0 : 2.0)) * M * N;
+  const double out_bytes =
+      (ep.kind == EPI_RESID_F32 || ep.kind == EPI_RESID_ADD ? 8.0 : (ep.kind == EPI_SWIGLU_F16 ? 1.0 : 2.0)) * M * N;
   ProfScope ps(c, name, 2.0 * M * N * K, 2.0 * (double(M) * K + double(N) * K) + out_bytes);
   const bool pair = c->gemm_pair && bn == 256 && M >= 512;
   int e = gemm_f16_tcgen05(A, lda, B, ldb, M, N, K, bn, pair, ep, c->num_sms, c->stream);
@@ -514,7 +515,9 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
     e3.err = c->d_err;
     if (!prune) {
       e2.out = b.resid;
+      e2.kind = EPI_RESID_ADD;  // the residual add is done by the TMA unit (no fp16 copy wanted here)
       AIQ_TRY(gemm(c, "gemm_o_resid", b.att, Hq * hd, L.wo, Hq * hd, M, d, Hq * hd, m.bn_o, e2));
+      e2.kind = EPI_RESID_F32;
       {
         ProfScope p(c, "rmsnorm", 0, 6.0 * double(T) * d);  // fp32 in, fp16 out
         launch_rmsnorm(b.resid, T, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
@@ -538,6 +541,7 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
       }
       const int Mo = static_cast<int>(n_seqs);
       e2.out = b.resid_last;
+      e2.kind = EPI_RESID_ADD;
       AIQ_TRY(gemm(c, "gemm_o_resid", b.qkv, Hq * hd, L.wo, Hq * hd, Mo, d, Hq * hd, m.bn_o, e2));
       {
         ProfScope p(c, "rmsnorm", 0, 6.0 * double(Mo) * d);
@@ -666,12 +670,13 @@ aiq_status decode_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const Deco
                                       cudaGetErrorString(static_cast<cudaError_t>(e)));
     }
     GemmEpilogue e2;
-    e2.kind = EPI_RESID_F32;
+    e2.kind = EPI_RESID_ADD;
     e2.out = b.resid;
     e2.ldo = dm;
     e2.err = c->d_err;
     e2.ss_parts = parts;
     AIQ_TRY(gemm(c, "dec_gemm_o_resid", b.att, Hq * hd, L.wo, Hq * hd, R, dm, Hq * hd, m.bn_o, e2));
+    e2.kind = EPI_RESID_F32;
     {
       ProfScope p(c, "rmsnorm", 0, 6.0 * double(R) * dm);
       launch_rmsnorm(b.resid, R, dm, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
@@ -1777,7 +1782,8 @@ aiq_status aiq_op_gemm(aiq_ctx* c, const void* A, int64_t lda, const void* B, in
                        int32_t K, int32_t bn, int32_t epilogue, void* out, int64_t ldo, const int32_t* positions,
                        const float* rope_cos, const float* rope_sin, int32_t rope_cols, int32_t head_dim) {
   if (!c || !A || !B || !out) return fail(AIQ_ERR_INVALID_ARG, "NULL argument");
-  if (epilogue < AIQ_EPI_F16 || epilogue > AIQ_EPI_SWIGLU_F16) return fail(AIQ_ERR_INVALID_ARG, "unknown epilogue");
+  if ((epilogue < AIQ_EPI_F16 || epilogue > AIQ_EPI_SWIGLU_F16) && epilogue != AIQ_EPI_RESID_ADD_F32)
+    return fail(AIQ_ERR_INVALID_ARG, "unknown epilogue");
   if (M < 0 || N <= 0 || K <= 0 || K % 64 || !(bn == 128 || bn == 256) || N % bn)
     return fail(AIQ_ERR_INVALID_ARG, "need M >= 0, K % 64 == 0, bn in {128, 256}, N % bn == 0");
   if (lda < K || ldb < K) return fail(AIQ_ERR_INVALID_ARG, "lda/ldb smaller than K");

@@ -47,6 +47,15 @@ struct KArgs {
   GemmEpilogue ep;
 };
 
+// EPI_RESID_ADD stages the accumulator in shared memory for TMA reduce-add:
+// per epilogue warp two 32 x 32 fp32 buffers (4 KB each, 128-byte swizzle),
+// after the operand ring and the barriers, 1024-byte aligned.
+template <int EPI>
+constexpr int epi_stage_bytes() {
+  return EPI == EPI_RESID_ADD ? 4 * 2 * 4096 : 0;
+}
+constexpr int round_up_1k(int x) { return (x + 1023) & ~1023; }
+
 // Tile order: bands of at most kBandTiles output-tile columns, all row tiles
 // of a band before the next band, columns fastest within a band.  Running
 // CTAs then share one band of the weight matrix (<= 32 MB for 2048-deep K)
@@ -350,9 +359,46 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
   if (bad) set_dev_error(ep.err, DEVERR_FP16_RANGE);
 }
 
+__device__ __forceinline__ void st_shared_v4(uint32_t saddr, uint4 v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(saddr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+
+// out[rows m0q .. m0q + 31][n0 .. n0 + BN) += acc, one 32 x 32 tile at a time:
+// each lane writes its row (TMEM lane) into a swizzled staging buffer, lane 0
+// hands the tile to the TMA unit as a reduce-add (rows past M are clipped by
+// the tensor map).  Two buffers alternate; a buffer is rewritten only after
+// the reduce issued from it two tiles earlier has read it.
+template <int BN>
+__device__ __forceinline__ void epilogue_tma_add(const CUtensorMap* tma_c, uint32_t trow, int m0q, int n0,
+                                                 uint8_t* stage, int lane, uint32_t& nbuf) {
+#pragma unroll 1
+  for (int c = 0; c < BN; c += 32) {
+    float v[32];
+    load32(trow + c, v);
+    uint8_t* buf = stage + (nbuf & 1) * 4096;
+    if (lane == 0) bulk_wait_group_read<1>();
+    __syncwarp();
+    const uint32_t row = smem_u32(buf) + lane * 128;
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      st_shared_v4(row + ((j ^ (lane & 7)) << 4), make_uint4(__float_as_uint(v[4 * j]), __float_as_uint(v[4 * j + 1]),
+                                                             __float_as_uint(v[4 * j + 2]),
+                                                             __float_as_uint(v[4 * j + 3])));
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_reduce_add_2d(tma_c, buf, n0 + c, m0q);
+      bulk_commit_group();
+    }
+    ++nbuf;
+  }
+}
+
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_gemm_tcgen05(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b, KArgs args) {
+    k_gemm_tcgen05(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
+                   const __grid_constant__ CUtensorMap tma_c, KArgs args) {
   using C = Cfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -475,6 +521,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ------------------------------------------------------------ epilogue
     const int quarter = warp & 3;  // TMEM lanes this warp may access
+    uint8_t* stage = smem + round_up_1k(C::STAGES * C::STAGE_BYTES + C::BAR_BYTES) + quarter * 8192;
+    uint32_t nbuf = 0;
     int acc = 0;
     uint32_t acc_ph = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
@@ -489,12 +537,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
       tc_fence_after();
       const uint32_t trow = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-      epilogue_tile<BN, EPI>(args, trow, m0 + quarter * 32 + lane, n0, inv);
+      if constexpr (EPI == EPI_RESID_ADD)
+        epilogue_tma_add<BN>(&tma_c, trow, m0 + quarter * 32, n0, stage, lane, nbuf);
+      else
+        epilogue_tile<BN, EPI>(args, trow, m0 + quarter * 32 + lane, n0, inv);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
       acc ^= 1;
       if (acc == 0) acc_ph ^= 1;
+    }
+    if constexpr (EPI == EPI_RESID_ADD) {
+      if (lane == 0) bulk_wait_group_all();  // the reduces have completed before the CTA leaves
     }
   }
 
@@ -525,7 +579,7 @@ struct CfgPair {
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     k_gemm_tcgen05_pair(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
-                        KArgs args) {
+                        const __grid_constant__ CUtensorMap tma_c, KArgs args) {
   using C = CfgPair;
   constexpr int BN = 256;
   extern __shared__ uint8_t smem_raw[];
@@ -653,6 +707,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------ epilogue (both CTAs)
     const int quarter = warp & 3;
     const uint32_t tempty_leader = map_to_cta(smem_u32(tempty), 0);
+    uint8_t* stage = smem + round_up_1k(C::STAGES * C::STAGE_BYTES + 256) + quarter * 8192;
+    uint32_t nbuf = 0;
     int acc = 0;
     uint32_t acc_ph = 0;
     for (int tile = pair; tile < num_tiles; tile += n_pairs) {
@@ -667,12 +723,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
       tc_fence_after();
       const uint32_t trow = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
-      epilogue_tile<BN, EPI>(args, trow, m0 + quarter * 32 + lane, n0, inv);
+      if constexpr (EPI == EPI_RESID_ADD)
+        epilogue_tma_add<BN>(&tma_c, trow, m0 + quarter * 32, n0, stage, lane, nbuf);
+      else
+        epilogue_tile<BN, EPI>(args, trow, m0 + quarter * 32 + lane, n0, inv);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(tempty_leader + acc * 8);
       acc ^= 1;
       if (acc == 0) acc_ph ^= 1;
+    }
+    if constexpr (EPI == EPI_RESID_ADD) {
+      if (lane == 0) bulk_wait_group_all();  // the reduces have completed before the CTA leaves
     }
   }
 
@@ -710,28 +772,60 @@ bool make_map(CUtensorMap* m, const __half* base, int64_t rows, int64_t cols, in
   return r == CUDA_SUCCESS;
 }
 
+// 2-D fp32 tensor [rows, cols] (row pitch ld elements), box 32 x 32, 128B swizzle:
+// the target of EPI_RESID_ADD's reduce-add tiles.
+bool make_map_out_f32(CUtensorMap* m, float* base, int64_t rows, int64_t cols, int64_t ld) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld * 4)};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 template <int BN, int EPI>
-int launch(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, int num_sms, cudaStream_t stream) {
+constexpr int smem_single() {
   using C = Cfg<BN>;
-  cudaError_t e = cudaFuncSetAttribute(k_gemm_tcgen05<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  return EPI == EPI_RESID_ADD ? 1024 + round_up_1k(C::STAGES * C::STAGE_BYTES + C::BAR_BYTES) + epi_stage_bytes<EPI>()
+                              : C::SMEM;
+}
+template <int EPI>
+constexpr int smem_pair() {
+  using C = CfgPair;
+  return EPI == EPI_RESID_ADD ? 1024 + round_up_1k(C::STAGES * C::STAGE_BYTES + 256) + epi_stage_bytes<EPI>()
+                              : C::SMEM;
+}
+static_assert(smem_single<256, EPI_RESID_ADD>() <= 232448 && smem_single<128, EPI_RESID_ADD>() <= 232448 &&
+                  smem_pair<EPI_RESID_ADD>() <= 232448,
+              "shared memory per block");
+
+template <int BN, int EPI>
+int launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mc, const KArgs& a, int num_sms,
+           cudaStream_t stream) {
+  constexpr int SM = smem_single<BN, EPI>();
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tcgen05<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM);
   if (e != cudaSuccess) return e;
   const int tiles = ((a.M + BM - 1) / BM) * (a.N / BN);
   const int grid = tiles < num_sms ? tiles : num_sms;
-  k_gemm_tcgen05<BN, EPI><<<grid, kThreads, C::SMEM, stream>>>(ma, mb, a);
+  k_gemm_tcgen05<BN, EPI><<<grid, kThreads, SM, stream>>>(ma, mb, mc, a);
   return cudaGetLastError();
 }
 
 template <int EPI>
-int launch_pair(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, int num_sms, cudaStream_t stream) {
-  using C = CfgPair;
-  cudaError_t e = cudaFuncSetAttribute(k_gemm_tcgen05_pair<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+int launch_pair(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mc, const KArgs& a, int num_sms,
+                cudaStream_t stream) {
+  constexpr int SM = smem_pair<EPI>();
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tcgen05_pair<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, SM);
   if (e != cudaSuccess) return e;
   const int tiles = ((a.M + 2 * BM - 1) / (2 * BM)) * (a.N / 256);
   const int pairs = tiles < num_sms / 2 ? tiles : num_sms / 2;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * pairs, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.dynamicSmemBytes = SM;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -740,30 +834,34 @@ int launch_pair(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, in
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, k_gemm_tcgen05_pair<EPI>, ma, mb, a);
+  e = cudaLaunchKernelEx(&cfg, k_gemm_tcgen05_pair<EPI>, ma, mb, mc, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
-int dispatch_pair(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, int num_sms, cudaStream_t s) {
+int dispatch_pair(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mc, const KArgs& a, int num_sms,
+                  cudaStream_t s) {
   switch (a.ep.kind) {
-    case EPI_F16: return launch_pair<EPI_F16>(ma, mb, a, num_sms, s);
-    case EPI_ROPE_F16: return launch_pair<EPI_ROPE_F16>(ma, mb, a, num_sms, s);
-    case EPI_RESID_F32: return launch_pair<EPI_RESID_F32>(ma, mb, a, num_sms, s);
-    case EPI_SWIGLU_F16: return launch_pair<EPI_SWIGLU_F16>(ma, mb, a, num_sms, s);
-    case EPI_ARGMAX: return launch_pair<EPI_ARGMAX>(ma, mb, a, num_sms, s);
+    case EPI_F16: return launch_pair<EPI_F16>(ma, mb, mc, a, num_sms, s);
+    case EPI_ROPE_F16: return launch_pair<EPI_ROPE_F16>(ma, mb, mc, a, num_sms, s);
+    case EPI_RESID_F32: return launch_pair<EPI_RESID_F32>(ma, mb, mc, a, num_sms, s);
+    case EPI_SWIGLU_F16: return launch_pair<EPI_SWIGLU_F16>(ma, mb, mc, a, num_sms, s);
+    case EPI_ARGMAX: return launch_pair<EPI_ARGMAX>(ma, mb, mc, a, num_sms, s);
+    case EPI_RESID_ADD: return launch_pair<EPI_RESID_ADD>(ma, mb, mc, a, num_sms, s);
   }
   return cudaErrorInvalidValue;
 }
 
 template <int BN>
-int dispatch_epi(const CUtensorMap& ma, const CUtensorMap& mb, const KArgs& a, int num_sms, cudaStream_t s) {
+int dispatch_epi(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& mc, const KArgs& a, int num_sms,
+                 cudaStream_t s) {
   switch (a.ep.kind) {
-    case EPI_F16: return launch<BN, EPI_F16>(ma, mb, a, num_sms, s);
-    case EPI_ROPE_F16: return launch<BN, EPI_ROPE_F16>(ma, mb, a, num_sms, s);
-    case EPI_RESID_F32: return launch<BN, EPI_RESID_F32>(ma, mb, a, num_sms, s);
-    case EPI_SWIGLU_F16: return launch<BN, EPI_SWIGLU_F16>(ma, mb, a, num_sms, s);
-    case EPI_ARGMAX: return launch<BN, EPI_ARGMAX>(ma, mb, a, num_sms, s);
+    case EPI_F16: return launch<BN, EPI_F16>(ma, mb, mc, a, num_sms, s);
+    case EPI_ROPE_F16: return launch<BN, EPI_ROPE_F16>(ma, mb, mc, a, num_sms, s);
+    case EPI_RESID_F32: return launch<BN, EPI_RESID_F32>(ma, mb, mc, a, num_sms, s);
+    case EPI_SWIGLU_F16: return launch<BN, EPI_SWIGLU_F16>(ma, mb, mc, a, num_sms, s);
+    case EPI_ARGMAX: return launch<BN, EPI_ARGMAX>(ma, mb, mc, a, num_sms, s);
+    case EPI_RESID_ADD: return launch<BN, EPI_RESID_ADD>(ma, mb, mc, a, num_sms, s);
   }
   return cudaErrorInvalidValue;
 }
@@ -782,11 +880,20 @@ int gemm_f16_tcgen05(const __half* A, int64_t lda, const __half* B, int64_t ldb,
     if (!(hd == 32 || hd == 64 || hd == 128) || bn % hd != 0 || !ep.positions || !ep.rope_cos) return cudaErrorInvalidValue;
   }
   if (ep.kind == EPI_ARGMAX && (!ep.bias || !ep.best)) return cudaErrorInvalidValue;
-  CUtensorMap ma, mb;
+  if (ep.kind == EPI_RESID_ADD &&
+      (!ep.out || (reinterpret_cast<uintptr_t>(ep.out) & 15) || (ep.ldo * 4) % 16 != 0 || ep.xh_out))
+    return cudaErrorInvalidValue;
+  CUtensorMap ma, mb, mc;
   if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, B, N, K, ldb, pair ? 128 : bn)) return cudaErrorInvalidValue;
+  if (ep.kind == EPI_RESID_ADD) {
+    if (!make_map_out_f32(&mc, static_cast<float*>(ep.out), M, N, ep.ldo)) return cudaErrorInvalidValue;
+  } else {
+    mc = ma;  // unused by the other epilogues
+  }
   KArgs a{M, N, K, ep};
-  if (pair) return dispatch_pair(ma, mb, a, num_sms, stream);
-  return bn == 256 ? dispatch_epi<256>(ma, mb, a, num_sms, stream) : dispatch_epi<128>(ma, mb, a, num_sms, stream);
+  if (pair) return dispatch_pair(ma, mb, mc, a, num_sms, stream);
+  return bn == 256 ? dispatch_epi<256>(ma, mb, mc, a, num_sms, stream)
+                   : dispatch_epi<128>(ma, mb, mc, a, num_sms, stream);
 }
 
 }  // namespace aiq

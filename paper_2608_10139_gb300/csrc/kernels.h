@@ -16,6 +16,7 @@ enum GemmEpi : int {
   EPI_SWIGLU_F16 = 3, // B interleaves gate/up blocks of BN/2 rows: out fp16 [M, N/2] = silu(g) * u
   EPI_ARGMAX = 4,     // per row: max over columns of acc + bias[col] and its first column, folded into
                       // best[row] with a 64-bit atomicMax of (order-preserving value bits, ~col)
+  EPI_RESID_ADD = 5,  // out fp32 [M, N] += acc by TMA reduce-add tiles (no xh_out / ss_out)
 };
 
 struct GemmEpilogue {

@@ -58,16 +58,21 @@ def test_gemm_f16_store(ctx, M, N, K, bn):
     _close(_np64(out), ref, 2e-3, 2e-3 * np.sqrt(K) * 0.05, f"f16 M{M} N{N} K{K}")
 
 
-@pytest.mark.parametrize("M,N,K,bn", GEMM_CASES[:4])
-def test_gemm_residual_add(ctx, M, N, K, bn):
+@pytest.mark.parametrize("epi", [2, 5])   # residual add in the epilogue threads / by TMA reduce-add tiles
+@pytest.mark.parametrize("M,N,K,bn", GEMM_CASES[:4] + [GEMM_CASES[5]])
+def test_gemm_residual_add(ctx, M, N, K, bn, epi):
     rng = np.random.default_rng(7 * M + N)
     A = rng.standard_normal((M, K)).astype(np.float16)
     B = (rng.standard_normal((N, K)) * 0.05).astype(np.float16)
     R = rng.standard_normal((M, N)).astype(np.float32)
-    dA, dB, dR = _h(A), _h(B), _h(R)
-    ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, bn, 2, dR.data_ptr(), N)
+    guard = rng.standard_normal((M + 40, N)).astype(np.float32)     # rows past M must stay untouched
+    guard[:M] = R
+    dA, dB, dR = _h(A), _h(B), _h(guard)
+    ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, bn, epi, dR.data_ptr(), N)
     ref = R.astype(np.float64) + A.astype(np.float64) @ B.astype(np.float64).T
-    _close(_np64(dR), ref, 1e-5, 2e-6 * np.sqrt(K), f"resid M{M} N{N} K{K}")
+    got = _np64(dR)
+    _close(got[:M], ref, 1e-5, 2e-6 * np.sqrt(K), f"resid{epi} M{M} N{N} K{K}")
+    assert np.array_equal(got[M:], guard[M:].astype(np.float64))
 
 
 @pytest.mark.parametrize("M,f,K,bn", [(130, 256, 128, 256), (700, 512, 256, 128), (2049, 1024, 512, 256)])
@@ -187,7 +192,7 @@ def test_attention_with_shared_prefix(ctx, hd, Hq, Hkv, P):
 
 @pytest.mark.parametrize("pair", [0, 1])
 @pytest.mark.parametrize("M,N,K,epi", [(512, 256, 128, 0), (1000, 512, 2048, 0), (4099, 1536, 512, 2),
-                                       (3000, 2048, 256, 3), (70000, 1024, 256, 0)])
+                                       (4099, 1536, 512, 5), (3000, 2048, 256, 3), (70000, 1024, 256, 0)])
 def test_gemm_cta_pair_vs_single(ctx, pair, M, N, K, epi):
     """256 x 256 tiles on CTA pairs (tcgen05 cta_group::2) and 128 x 256 tiles on
     single CTAs give the oracle's product, ragged M included."""
@@ -202,10 +207,10 @@ def test_gemm_cta_pair_vs_single(ctx, pair, M, N, K, epi):
             out = torch.zeros((M, N), dtype=torch.float16, device="cuda")
             ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, 256, 0, out.data_ptr(), N)
             _close(_np64(out), a @ b.T, 2e-3, 2e-3 * np.sqrt(K) * 0.05, f"pair{pair} f16 M{M}")
-        elif epi == 2:
+        elif epi in (2, 5):
             R = rng.standard_normal((M, N)).astype(np.float32)
             dR = _h(R)
-            ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, 256, 2, dR.data_ptr(), N)
+            ctx.op_gemm(dA.data_ptr(), K, dB.data_ptr(), K, M, N, K, 256, epi, dR.data_ptr(), N)
             _close(_np64(dR), R.astype(np.float64) + a @ b.T, 1e-5, 2e-6 * np.sqrt(K), f"pair{pair} resid M{M}")
         else:
             f = N // 2
