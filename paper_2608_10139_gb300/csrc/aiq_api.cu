@@ -229,6 +229,8 @@ aiq_status sync_and_check(aiq_ctx* c) {
     if (err & DEVERR_HASH_FULL) return fail(AIQ_ERR_CAPACITY, "hash table probe sequence exhausted");
     if (err & DEVERR_TIMEOUT) return fail(AIQ_ERR_DEVICE_CHECK, "a kernel's bounded wait expired");
     if (err & DEVERR_FP16_RANGE) return fail(AIQ_ERR_DEVICE_CHECK, "an activation left the fp16 range (or was NaN)");
+    if (err & DEVERR_BOUNDS)
+      return fail(AIQ_ERR_DEVICE_CHECK, "an index failed its bounds check (e.g. no finite logit for a greedy step)");
     return fail(AIQ_ERR_DEVICE_CHECK, "device check failed (code " + std::to_string(err) + ")");
   }
   return AIQ_OK;
