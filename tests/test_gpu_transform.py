@@ -176,7 +176,7 @@ def test_transform_rejects_bad_specs(ctx):
         assert ei.value.status == aiq.ERR_INVALID_ARG
 
 
-@pytest.mark.parametrize("hd,hq,hkv", [(32, 4, 4), (64, 8, 2), (128, 8, 1), (64, 32, 8)])
+@pytest.mark.parametrize("hd,hq,hkv", [(32, 4, 4), (64, 8, 2), (128, 8, 1), (64, 32, 8), (128, 32, 8), (64, 16, 8)])
 def test_op_decode_attention_matches_fp32_reference(ctx, hd, hq, hkv):
     torch = pytest.importorskip("torch")
     dev = "cuda"
