@@ -79,6 +79,25 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
+// Packed fp32 pairs (Blackwell f32x2): two IEEE fma / add per instruction,
+// each lane's result identical to the scalar operation.
+__device__ __forceinline__ unsigned long long f2_bits(float2 v) {
+  return (static_cast<unsigned long long>(__float_as_uint(v.y)) << 32) | __float_as_uint(v.x);
+}
+__device__ __forceinline__ float2 bits_f2(unsigned long long b) {
+  return make_float2(__uint_as_float(static_cast<uint32_t>(b)), __uint_as_float(static_cast<uint32_t>(b >> 32)));
+}
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  unsigned long long r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(f2_bits(a)), "l"(f2_bits(b)), "l"(f2_bits(c)));
+  return bits_f2(r);
+}
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  unsigned long long r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(f2_bits(a)), "l"(f2_bits(b)));
+  return bits_f2(r);
+}
+
 __device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t saddr) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
@@ -359,24 +378,23 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
             tmem_st_wait();
           }
         }
-        float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        float2 ps[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
         const uint32_t prow = smem_u32(sP(b)) + r * 128;
-        const float sc = a.scale_log2, neg_m = -m_used;
+        const float2 sc2 = make_float2(a.scale_log2, a.scale_log2), nm2 = make_float2(-m_used, -m_used);
 #pragma unroll
         for (int ch = 0; ch < 8; ++ch) {
           uint32_t pk[4];
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
-            const float p0 = ex2_approx(fmaf(v[ch * 8 + 2 * i], sc, neg_m));
-            const float p1 = ex2_approx(fmaf(v[ch * 8 + 2 * i + 1], sc, neg_m));
-            ps[2 * i] += p0;
-            ps[2 * i + 1] += p1;
-            __half2 h = __floats2half2_rn(p0, p1);
+            const float2 x = ffma2(make_float2(v[ch * 8 + 2 * i], v[ch * 8 + 2 * i + 1]), sc2, nm2);
+            const float2 p = make_float2(ex2_approx(x.x), ex2_approx(x.y));
+            ps[i] = fadd2(ps[i], p);
+            __half2 h = __floats2half2_rn(p.x, p.y);
             pk[i] = *reinterpret_cast<uint32_t*>(&h);
           }
           st_shared_v4(prow + ((ch ^ (r & 7)) << 4), make_uint4(pk[0], pk[1], pk[2], pk[3]));
         }
-        l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+        l += ((ps[0].x + ps[0].y) + (ps[1].x + ps[1].y)) + ((ps[2].x + ps[2].y) + (ps[3].x + ps[3].y));
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&p_full[b]);
