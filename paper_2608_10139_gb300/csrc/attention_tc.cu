@@ -44,7 +44,9 @@ struct ACfg {
   static constexpr int OFF_P = OFF_VT + 2 * VT_BYTES;
   static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
   static constexpr int SMEM = 1024 + OFF_BAR + 256;
-  static constexpr int TMEM_COLS = 256;  // two 64-column score buffers + the output
+  // two 64-column score buffers, then two HD-column output accumulators (one
+  // per alternating work item), rounded up to a power of two
+  static constexpr int TMEM_COLS = HD == 64 ? 256 : 512;
   static constexpr int O_COL = 128;
 };
 
@@ -128,9 +130,9 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
   uint64_t* s_full = bars + 6;    // [2]
   uint64_t* p_full = bars + 8;    // [2]
   uint64_t* o_done = bars + 10;   // [2]: PV of block g commits o_done[g & 1]
-  uint64_t* o_free = bars + 12;
-  uint64_t* mma_done = bars + 13;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 14);
+  uint64_t* o_free = bars + 12;   // [2]: output accumulator it & 1 read out
+  uint64_t* mma_done = bars + 14;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 15);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   auto sK = [&](int b) { return smem + C::OFF_K + b * C::K_BYTES; };
   auto sV = [&](int b) { return smem + C::OFF_V + b * C::K_BYTES; };
@@ -149,7 +151,8 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       mbar_init(&p_full[b], 4);
       mbar_init(&o_done[b], 1);
     }
-    mbar_init(o_free, 4);
+    mbar_init(&o_free[0], 4);
+    mbar_init(&o_free[1], 4);
     mbar_init(mma_done, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -240,9 +243,8 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         const int n_kv = n_pre + (q_end + kKeys - 1) / kKeys;
         if (!mbar_wait_bounded(q_full, it & 1, abort_flag, err)) break;
         tc_fence_after();
-        // the softmax warps have read out the previous item's output
-        if (!mbar_wait_bounded(o_free, (it & 1) ^ 1, abort_flag, err)) break;
-        tc_fence_after();
+        // the first scores only need Q and the key block: they are computed
+        // while the softmax warps still read out the previous item's output
         if (!issue_s(g)) break;
         for (int j = 0; j < n_kv; ++j, ++g) {
           if (j + 1 < n_kv && !issue_s(g + 1)) {
@@ -255,10 +257,16 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
             ok = false;
             break;
           }
+          // the first PV overwrites this item's accumulator: the softmax warps
+          // must have read out the output of the item two back
+          if (j == 0 && !mbar_wait_bounded(&o_free[it & 1], ((it >> 1) & 1) ^ 1, abort_flag, err)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            umma_f16_ss(tmem_base + C::O_COL, smem_desc_k_sw128(smem_u32(sP(b)) + k * 32),
+            umma_f16_ss(tmem_base + C::O_COL + (it & 1) * HD, smem_desc_k_sw128(smem_u32(sP(b)) + k * 32),
                         smem_desc_k_sw128(smem_u32(sVt(b)) + k * 32), idesc_o, (j | k) != 0);
           umma_commit(&kv_empty[b]);
           umma_commit(&o_done[b]);
@@ -277,6 +285,46 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
     uint32_t g = 0;
     int it = 0;
     bool ok = true;
+    // The output of an item is read out after the next item's first block
+    // (its last PV may still be running meanwhile): O / l, stored for the
+    // tile's real tokens, then the accumulator is handed back to the MMA warp.
+    struct Pending {
+      bool on, live;
+      int buf;
+      uint32_t g_last;
+      float inv;
+      __half* dst;
+    } pend{false, false, 0, 0, 0.f, nullptr};
+    auto flush = [&]() -> bool {
+      if (!mbar_wait_bounded(&o_done[pend.g_last & 1], (pend.g_last >> 1) & 1, abort_flag, err)) return false;
+      tc_fence_after();
+      const uint32_t ocol = trow + C::O_COL + pend.buf * HD;
+#pragma unroll 1
+      for (int c = 0; c < HD; c += 32) {
+        uint32_t o[32];
+        tmem_ld_32x32b_x32(ocol + c, o);
+        tmem_ld_wait();
+        if (pend.live) {
+          uint4* d4 = reinterpret_cast<uint4*>(pend.dst + c);
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4) {
+            uint32_t pk[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              __half2 h = __floats2half2_rn(__uint_as_float(o[q4 * 8 + 2 * i]) * pend.inv,
+                                            __uint_as_float(o[q4 * 8 + 2 * i + 1]) * pend.inv);
+              pk[i] = *reinterpret_cast<uint32_t*>(&h);
+            }
+            d4[q4] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&o_free[pend.buf]);
+      pend.on = false;
+      return true;
+    };
     for (int w = blockIdx.x; w < n_work && ok; w += gridDim.x, ++it) {
       const int tidx = w / a.Hkv, kvh = w % a.Hkv;
       const int s = a.tile_seq[tidx], q0 = a.tile_q0[tidx];
@@ -284,6 +332,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       const int q_end = min(q0 + a.TQ, len);
       const int n_kv = n_pre + (q_end + kKeys - 1) / kKeys;
       const int qpos = q0 + t;
+      const uint32_t ocol = trow + C::O_COL + (it & 1) * HD;
       float m_used = 0.f, l = 0.f;
       for (int j = 0; j < n_kv; ++j, ++g) {
         const int b = g & 1;
@@ -369,11 +418,11 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
 #pragma unroll 1
             for (int c = 0; c < HD; c += 32) {
               uint32_t o[32];
-              tmem_ld_32x32b_x32(trow + C::O_COL + c, o);
+              tmem_ld_32x32b_x32(ocol + c, o);
               tmem_ld_wait();
 #pragma unroll
               for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
-              tmem_st_32x32b_x32(trow + C::O_COL + c, o);
+              tmem_st_32x32b_x32(ocol + c, o);
             }
             tmem_st_wait();
           }
@@ -398,38 +447,20 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&p_full[b]);
-      }
-      if (!ok) break;
-      // output row: O / l, stored for the tile's real tokens
-      if (!mbar_wait_bounded(&o_done[(g - 1) & 1], ((g - 1) >> 1) & 1, abort_flag, err)) break;
-      tc_fence_after();
-      const float inv = l > 0.f ? 1.f / l : 0.f;
-      const bool live = qpos < len;
-      __half* dst = a.out + static_cast<int64_t>(st + qpos) * (a.Hq * HD) + (kvh * a.G + gq) * HD;
-#pragma unroll 1
-      for (int c = 0; c < HD; c += 32) {
-        uint32_t o[32];
-        tmem_ld_32x32b_x32(trow + C::O_COL + c, o);
-        tmem_ld_wait();
-        if (live) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + c);
-#pragma unroll
-          for (int q4 = 0; q4 < 4; ++q4) {
-            uint32_t pk[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              __half2 h = __floats2half2_rn(__uint_as_float(o[q4 * 8 + 2 * i]) * inv,
-                                            __uint_as_float(o[q4 * 8 + 2 * i + 1]) * inv);
-              pk[i] = *reinterpret_cast<uint32_t*>(&h);
-            }
-            d4[q4] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-          }
+        if (j == 0 && pend.on && !flush()) {
+          ok = false;
+          break;
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(o_free);
+      if (!ok) break;
+      pend.on = true;
+      pend.live = qpos < len;
+      pend.buf = it & 1;
+      pend.g_last = g - 1;
+      pend.inv = l > 0.f ? 1.f / l : 0.f;
+      pend.dst = a.out + static_cast<int64_t>(st + qpos) * (a.Hq * HD) + (kvh * a.G + gq) * HD;
     }
+    if (ok && pend.on) flush();
   }
 
   __syncthreads();
