@@ -111,6 +111,17 @@ typedef struct {
 aiq_status aiq_filter_compact_static(const aiq_term* terms, int32_t n_terms, int64_t n_rows, int32_t* ids_out,
                                      int64_t* count_out, void* stream);
 
+/* Self-test of the device-side failure detection that every pipelined kernel
+ * of the library uses.  One CTA of two warps waits on an mbarrier phase that
+ * nothing completes: warp 0 with a limit of limit_ns, warp 1 with four times
+ * that, both through the same bounded wait as the kernels.  Warp 0's wait runs
+ * out, records the timeout and raises the CTA's abort flag, on which warp 1
+ * returns without waiting out its own limit.  The call then returns
+ * AIQ_ERR_DEVICE_CHECK ("a kernel's bounded wait expired"), and the context
+ * stays usable: the device error word is cleared and no CUDA error is left.
+ * limit_ns in [1000, 1000000000]; anything else gives AIQ_ERR_INVALID_ARG. */
+aiq_status aiq_op_wait_expiry_selftest(aiq_ctx* ctx, uint64_t limit_ns);
+
 #ifdef __cplusplus
 }
 #endif

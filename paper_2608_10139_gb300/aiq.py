@@ -119,6 +119,7 @@ _SIGS = {
     "aiq_op_decode_attention": [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_void_p,
                                 C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p],
     "aiq_filter_compact_static": [C.POINTER(_Term), C.c_int32, C.c_int64, C.c_void_p, C.c_void_p, C.c_void_p],
+    "aiq_op_wait_expiry_selftest": [C.c_void_p, C.c_uint64],
 }
 
 
@@ -442,6 +443,11 @@ class Context:
     def op_attention(self, qkv: int, T: int, seq_start: int, n_seqs: int, Hq: int, Hkv: int, hd: int, out: int,
                      prefix_kv: int = 0, P: int = 0):
         _check(self.lib.aiq_op_attention(self.h, qkv, T, seq_start, n_seqs, Hq, Hkv, hd, prefix_kv or None, P, out))
+
+    def op_wait_expiry_selftest(self, limit_ns: int):
+        """Runs the bounded-wait self-test (see aiq_ops.h); raises AiqError
+        with AIQ_ERR_DEVICE_CHECK when the wait expired as it should."""
+        _check(self.lib.aiq_op_wait_expiry_selftest(self.h, limit_ns))
 
     def op_decode_attention(self, qkv: int, R: int, Hq: int, Hkv: int, hd: int, own_kv: int, seq_start: int,
                             gen_kv: int, gen_cap: int, slot: int, out: int, prefix_kv: int = 0, P: int = 0):

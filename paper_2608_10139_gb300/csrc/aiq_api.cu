@@ -1859,4 +1859,13 @@ aiq_status aiq_op_decode_attention(aiq_ctx* c, const void* qkv, int32_t R, int32
   return sync_and_check(c);
 }
 
+aiq_status aiq_op_wait_expiry_selftest(aiq_ctx* c, uint64_t limit_ns) {
+  if (!c || limit_ns < 1000 || limit_ns > 1000000000ull) return fail(AIQ_ERR_INVALID_ARG, "bad args");
+  CUDA_TRY(cudaSetDevice(c->device));
+  const int e = launch_wait_expiry(limit_ns, c->d_err, c->stream);
+  if (e != 0) return fail(AIQ_ERR_CUDA, std::string("wait self-test launch: ") +
+                                            cudaGetErrorString(static_cast<cudaError_t>(e)));
+  return sync_and_check(c);
+}
+
 }  // extern "C"

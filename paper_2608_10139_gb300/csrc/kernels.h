@@ -173,6 +173,11 @@ void launch_gather_groups(const int32_t* rows, int64_t g, const int64_t* build_k
                           const unsigned long long* counts, int64_t* keys_out, int64_t* counts_out,
                           cudaStream_t s);
 
+// ------------------------------------------------------------- self-test ---
+// One CTA of two warps waiting on an mbarrier phase that never completes (warp 0
+// with limit_ns, warp 1 with 4 x limit_ns; see aiq_op_wait_expiry_selftest).
+int launch_wait_expiry(uint64_t limit_ns, int* err, cudaStream_t s);
+
 // ---------------------------------------------------------------- decode ---
 // Decode attention of R single-token rows (row r's token: q/k/v in qkv row r).
 // Keys of row r: the P shared-prefix rows of pkv, its own prompt rows
