@@ -36,8 +36,9 @@ PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 L2_BYTES = 129 * 1024 * 1024
 
 # DRAM traffic of one tcgen05 GEMM launch from an ncu capture, valid only for the
-# GEMM source it was measured on (sha256 prefix of csrc/gemm_tcgen05.cu).
-GEMM_TRAFFIC = {"source_sha": "6164ad24e18a6f17", "bytes_per_launch": 4.146e9}
+# GEMM source it was measured on (sha256 prefix of csrc/gemm_tcgen05.cu followed
+# by csrc/common.cuh, the device helpers it includes).
+GEMM_TRAFFIC = {"source_sha": "102b5a926777bc70", "bytes_per_launch": 4.696e9}
 
 
 def parse():
@@ -151,8 +152,11 @@ class ClockSampler:
 
 
 def gemm_source_sha():
-    src = os.path.join(ROOT, "paper_2608_10139_gb300", "csrc", "gemm_tcgen05.cu")
-    return hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    h = hashlib.sha256()
+    for name in ("gemm_tcgen05.cu", "common.cuh"):
+        with open(os.path.join(ROOT, "paper_2608_10139_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 # ------------------------------------------------------------ CPU oracle ---
