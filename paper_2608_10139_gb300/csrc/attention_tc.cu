@@ -6,17 +6,23 @@
 // keys of the shared prompt prefix (computed once per query, in prefix_kv)
 // come first, then the sequence's own keys up to the tile's last token.
 //
-//   warp 0    TMA: the Q tile (3-D box hd x heads x tokens), then K and V
-//             blocks of 64 keys into a two-slot ring (128-byte swizzle).
+//   warp 0    TMA: the Q tile (3-D box hd x heads x tokens) into one of two
+//             slots, then K and V blocks of 64 keys into two separate rings of
+//             NKV slots (128-byte swizzle).  A K slot is free once the S MMA
+//             that read it has completed, a V slot once the softmax warps have
+//             transposed it, so a block's loads are issued NKV blocks before
+//             its scores are needed instead of one.
 //   warp 1    tcgen05.mma: S = Q K^T into one of two TMEM score buffers, and
-//             O += P V^T into the TMEM output accumulator.
+//             O += P V^T into the item's TMEM output accumulator.
 //   warps 2-5 one query row per thread: read its 64 scores with tcgen05.ld,
 //             apply the causal / prefix / length mask, keep the running max
 //             (the output is rescaled only when the max grows by more than
 //             2^8, so P never exceeds 256), write exp2(s - max) as fp16 into
-//             the swizzled P tile and transpose their quarter of the V block
-//             into the K-major V^T tile with ldmatrix.trans; at the end divide
-//             by the row sum and store the output row.
+//             the swizzled P tile, then transpose their quarter of the V block
+//             into the K-major V^T tile with ldmatrix.trans (P and V^T are
+//             rewritten once the previous block's PV has completed); an item's
+//             output is divided by the row sum and stored after the next
+//             item's first block.
 // Work items are persistent per CTA; every wait is bounded.
 #include <cudaTypedefs.h>
 
@@ -32,23 +38,28 @@ constexpr int kKeys = 64;  // keys per block
 template <int HD>
 struct ACfg {
   static constexpr int NC = HD / 64;             // 64-column sub-tiles of one head
+  static constexpr int NKV = 3;                  // slots of the K ring and of the V ring
   static constexpr int Q_BYTES = 128 * HD * 2;   // 128 rows
   static constexpr int SUB = 64 * 128;           // one [64 x 64] fp16 sub-tile
   static constexpr int K_BYTES = NC * SUB;
   static constexpr int VT_BYTES = HD * 128;      // HD rows x 64 keys
   static constexpr int P_BYTES = 128 * 128;      // 128 rows x 64 keys
-  static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K = OFF_Q + Q_BYTES;
-  static constexpr int OFF_V = OFF_K + 2 * K_BYTES;
-  static constexpr int OFF_VT = OFF_V + 2 * K_BYTES;
-  static constexpr int OFF_P = OFF_VT + 2 * VT_BYTES;
-  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
-  static constexpr int SMEM = 1024 + OFF_BAR + 256;
+  static constexpr int OFF_Q = 0;                // two slots
+  static constexpr int OFF_K = OFF_Q + 2 * Q_BYTES;
+  static constexpr int OFF_V = OFF_K + NKV * K_BYTES;
+  static constexpr int OFF_VT = OFF_V + NKV * K_BYTES;
+  static constexpr int OFF_P = OFF_VT + VT_BYTES;
+  static constexpr int OFF_BAR = OFF_P + P_BYTES;
+  static constexpr int N_BARS = 4 + 4 * NKV + 2 + 1 + 2 + 2 + 1;
+  static constexpr int SMEM = 1024 + OFF_BAR + N_BARS * 8 + 16;
   // two 64-column score buffers, then two HD-column output accumulators (one
   // per alternating work item), rounded up to a power of two
   static constexpr int TMEM_COLS = HD == 64 ? 256 : 512;
   static constexpr int O_COL = 128;
 };
+// two CTAs per SM at HD = 64 (each also keeps 1 KB of the SM's shared memory)
+static_assert(2 * (ACfg<64>::SMEM + 1024) <= 233472, "HD = 64 tiles must fit two CTAs per SM");
+static_assert(ACfg<128>::SMEM <= 232448, "HD = 128 tiles must fit one CTA");
 
 struct AttnArgs {
   const int32_t* seq_start;
@@ -119,40 +130,46 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
     k_attention_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
                    const __grid_constant__ CUtensorMap tm_pre, AttnArgs a) {
   using C = ACfg<HD>;
+  constexpr int NKV = C::NKV;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sQ = smem + C::OFF_Q;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
-  uint64_t* q_full = bars + 0;
-  uint64_t* q_empty = bars + 1;
-  uint64_t* kv_full = bars + 2;   // [2]
-  uint64_t* kv_empty = bars + 4;  // [2]
-  uint64_t* s_full = bars + 6;    // [2]
-  uint64_t* p_full = bars + 8;    // [2]
-  uint64_t* o_done = bars + 10;   // [2]: PV of block g commits o_done[g & 1]
-  uint64_t* o_free = bars + 12;   // [2]: output accumulator it & 1 read out
-  uint64_t* mma_done = bars + 14;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 15);
+  uint64_t* q_full = bars + 0;             // [2]
+  uint64_t* q_empty = bars + 2;            // [2]: the item's S MMAs have completed
+  uint64_t* k_full = bars + 4;             // [NKV]
+  uint64_t* k_empty = k_full + NKV;        // [NKV]: the S MMA of the block has completed
+  uint64_t* v_full = k_empty + NKV;        // [NKV]
+  uint64_t* v_empty = v_full + NKV;        // [NKV]: the softmax warps have transposed the block
+  uint64_t* s_full = v_empty + NKV;        // [2]
+  uint64_t* p_full = s_full + 2;           // P and V^T of the block written
+  uint64_t* o_done = p_full + 1;           // [2]: PV of block g commits o_done[g & 1]
+  uint64_t* o_free = o_done + 2;           // [2]: output accumulator it & 1 read out
+  uint64_t* mma_done = o_free + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  auto sQ = [&](int b) { return smem + C::OFF_Q + b * C::Q_BYTES; };
   auto sK = [&](int b) { return smem + C::OFF_K + b * C::K_BYTES; };
   auto sV = [&](int b) { return smem + C::OFF_V + b * C::K_BYTES; };
-  auto sVt = [&](int b) { return smem + C::OFF_VT + b * C::VT_BYTES; };
-  auto sP = [&](int b) { return smem + C::OFF_P + b * C::P_BYTES; };
+  uint8_t* sVt = smem + C::OFF_VT;
+  uint8_t* sP = smem + C::OFF_P;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   int* err = a.err;
   if (threadIdx.x == 0) {
-    mbar_init(q_full, 1);
-    mbar_init(q_empty, 1);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&kv_full[b], 1);
-      mbar_init(&kv_empty[b], 1);
+      mbar_init(&q_full[b], 1);
+      mbar_init(&q_empty[b], 1);
       mbar_init(&s_full[b], 1);
-      mbar_init(&p_full[b], 4);
       mbar_init(&o_done[b], 1);
+      mbar_init(&o_free[b], 4);
     }
-    mbar_init(&o_free[0], 4);
-    mbar_init(&o_free[1], 4);
+    for (int b = 0; b < NKV; ++b) {
+      mbar_init(&k_full[b], 1);
+      mbar_init(&k_empty[b], 1);
+      mbar_init(&v_full[b], 1);
+      mbar_init(&v_empty[b], 4);
+    }
+    mbar_init(p_full, 4);
     mbar_init(mma_done, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -175,42 +192,56 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------ TMA
-      uint32_t g = 0;  // key blocks issued so far (ring position)
-      int it = 0;
+      uint32_t g = 0;   // key blocks whose K load was issued (ring position)
+      uint32_t gv = 0;  // key blocks whose V load was issued
+      int it = 0;       // Q loads issued
       bool ok = true;
-      for (int w = blockIdx.x; w < n_work && ok; w += gridDim.x, ++it) {
+      for (int w = blockIdx.x; w < n_work && ok; w += gridDim.x) {
         const int tidx = w / a.Hkv, kvh = w % a.Hkv;
         const int s = a.tile_seq[tidx], q0 = a.tile_q0[tidx];
         const int st = a.seq_start[s], len = a.seq_start[s + 1] - st;
         const int q_end = min(q0 + a.TQ, len);
         const int n_kv = n_pre + (q_end + kKeys - 1) / kKeys;
-        if (!mbar_wait_bounded(q_empty, (it & 1) ^ 1, abort_flag, err)) break;
-        mbar_arrive_expect_tx(q_full, C::Q_BYTES);
-        for (int c = 0; c < C::NC; ++c) tma_load_3d(sQ + c * (128 * 128), &tm_q, q_full, c * 64, kvh * a.G, st + q0);
+        const int qb = it & 1;
+        if (!mbar_wait_bounded(&q_empty[qb], ((it >> 1) & 1) ^ 1, abort_flag, err)) break;
+        mbar_arrive_expect_tx(&q_full[qb], C::Q_BYTES);
+        ++it;
+        for (int c = 0; c < C::NC; ++c)
+          tma_load_3d(sQ(qb) + c * (128 * 128), &tm_q, &q_full[qb], c * 64, kvh * a.G, st + q0);
         for (int j = 0; j < n_kv; ++j, ++g) {
-          const int b = g & 1;
-          if (!mbar_wait_bounded(&kv_empty[b], ((g >> 1) & 1) ^ 1, abort_flag, err)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(&kv_full[b], 2 * C::K_BYTES);
+          const int b = g % NKV;
+          const uint32_t ph = ((g / NKV) & 1) ^ 1;
           const bool pre = j < n_pre;
           const CUtensorMap* map = pre ? &tm_pre : &tm_kv;
           const int kcol = pre ? kvh * HD : (a.Hq + kvh) * HD;
           const int vcol = pre ? (a.Hkv + kvh) * HD : (a.Hq + a.Hkv + kvh) * HD;
           const int row = pre ? j * kKeys : st + (j - n_pre) * kKeys;
-          for (int c = 0; c < C::NC; ++c) {
-            tma_load_2d(sK(b) + c * C::SUB, map, &kv_full[b], kcol + c * 64, row);
-            tma_load_2d(sV(b) + c * C::SUB, map, &kv_full[b], vcol + c * 64, row);
+          if (!mbar_wait_bounded(&k_empty[b], ph, abort_flag, err)) {
+            ok = false;
+            break;
           }
+          mbar_arrive_expect_tx(&k_full[b], C::K_BYTES);
+          for (int c = 0; c < C::NC; ++c) tma_load_2d(sK(b) + c * C::SUB, map, &k_full[b], kcol + c * 64, row);
+          if (!mbar_wait_bounded(&v_empty[b], ph, abort_flag, err)) {
+            ok = false;
+            ++g;  // this block's K load is in flight, its V load is not
+            break;
+          }
+          mbar_arrive_expect_tx(&v_full[b], C::K_BYTES);
+          for (int c = 0; c < C::NC; ++c) tma_load_2d(sV(b) + c * C::SUB, map, &v_full[b], vcol + c * 64, row);
+          ++gv;
         }
       }
       if (!ok || *abort_flag) {
         // let this thread's copies still in flight land before the CTA can exit
+        // (the last use of each slot is the only one that can be outstanding)
         volatile int never = 0;
-        for (uint32_t i = g > 2 ? g - 2 : 0; i < g; ++i)
-          mbar_wait_bounded(&kv_full[i & 1], (i >> 1) & 1, &never, nullptr, 200000000ull);
-        mbar_wait_bounded(q_full, (it & 1), &never, nullptr, 200000000ull);
+        for (uint32_t i = g > NKV ? g - NKV : 0; i < g; ++i)
+          mbar_wait_bounded(&k_full[i % NKV], (i / NKV) & 1, &never, nullptr, 200000000ull);
+        for (uint32_t i = gv > NKV ? gv - NKV : 0; i < gv; ++i)
+          mbar_wait_bounded(&v_full[i % NKV], (i / NKV) & 1, &never, nullptr, 200000000ull);
+        for (int i = it > 2 ? it - 2 : 0; i < it; ++i)
+          mbar_wait_bounded(&q_full[i & 1], (i >> 1) & 1, &never, nullptr, 200000000ull);
       }
     }
   } else if (warp == 1) {
@@ -221,18 +252,19 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       uint32_t g = 0;
       int it = 0;
       bool ok = true;
-      auto issue_s = [&](uint32_t gg) -> bool {
-        const int b = gg & 1;
-        if (!mbar_wait_bounded(&kv_full[b], (gg >> 1) & 1, abort_flag, err)) return false;
+      auto issue_s = [&](uint32_t gg, int qb) -> bool {
+        const int kb = gg % NKV;
+        if (!mbar_wait_bounded(&k_full[kb], (gg / NKV) & 1, abort_flag, err)) return false;
         tc_fence_after();
-        const uint32_t d = tmem_base + b * kKeys;
+        const uint32_t d = tmem_base + (gg & 1) * kKeys;
 #pragma unroll
         for (int c = 0; c < C::NC; ++c)
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            umma_f16_ss(d, smem_desc_k_sw128(smem_u32(sQ + c * (128 * 128)) + k * 32),
-                        smem_desc_k_sw128(smem_u32(sK(b) + c * C::SUB) + k * 32), idesc_s, (c | k) != 0);
-        umma_commit(&s_full[b]);
+            umma_f16_ss(d, smem_desc_k_sw128(smem_u32(sQ(qb) + c * (128 * 128)) + k * 32),
+                        smem_desc_k_sw128(smem_u32(sK(kb) + c * C::SUB) + k * 32), idesc_s, (c | k) != 0);
+        umma_commit(&k_empty[kb]);
+        umma_commit(&s_full[gg & 1]);
         return true;
       };
       for (int w = blockIdx.x; w < n_work && ok; w += gridDim.x, ++it) {
@@ -241,35 +273,34 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         const int len = a.seq_start[s + 1] - a.seq_start[s];
         const int q_end = min(q0 + a.TQ, len);
         const int n_kv = n_pre + (q_end + kKeys - 1) / kKeys;
-        if (!mbar_wait_bounded(q_full, it & 1, abort_flag, err)) break;
+        const int qb = it & 1;
+        if (!mbar_wait_bounded(&q_full[qb], (it >> 1) & 1, abort_flag, err)) break;
         tc_fence_after();
         // the first scores only need Q and the key block: they are computed
         // while the softmax warps still read out the previous item's output
-        if (!issue_s(g)) break;
+        if (!issue_s(g, qb)) break;
         for (int j = 0; j < n_kv; ++j, ++g) {
-          if (j + 1 < n_kv && !issue_s(g + 1)) {
+          if (j + 1 < n_kv && !issue_s(g + 1, qb)) {
             ok = false;
             break;
           }
-          if (j + 1 == n_kv) umma_commit(q_empty);  // all S MMAs of this item issued
-          const int b = g & 1;
-          if (!mbar_wait_bounded(&p_full[b], (g >> 1) & 1, abort_flag, err)) {
+          if (j + 1 == n_kv) umma_commit(&q_empty[qb]);  // all S MMAs of this item issued
+          if (!mbar_wait_bounded(p_full, g & 1, abort_flag, err)) {
             ok = false;
             break;
           }
           // the first PV overwrites this item's accumulator: the softmax warps
           // must have read out the output of the item two back
-          if (j == 0 && !mbar_wait_bounded(&o_free[it & 1], ((it >> 1) & 1) ^ 1, abort_flag, err)) {
+          if (j == 0 && !mbar_wait_bounded(&o_free[qb], ((it >> 1) & 1) ^ 1, abort_flag, err)) {
             ok = false;
             break;
           }
           tc_fence_after();
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            umma_f16_ss(tmem_base + C::O_COL + (it & 1) * HD, smem_desc_k_sw128(smem_u32(sP(b)) + k * 32),
-                        smem_desc_k_sw128(smem_u32(sVt(b)) + k * 32), idesc_o, (j | k) != 0);
-          umma_commit(&kv_empty[b]);
-          umma_commit(&o_done[b]);
+            umma_f16_ss(tmem_base + C::O_COL + qb * HD, smem_desc_k_sw128(smem_u32(sP) + k * 32),
+                        smem_desc_k_sw128(smem_u32(sVt) + k * 32), idesc_o, (j | k) != 0);
+          umma_commit(&o_done[g & 1]);
         }
       }
       umma_commit(mma_done);
@@ -285,6 +316,12 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
     uint32_t g = 0;
     int it = 0;
     bool ok = true;
+    // PV of block gg done (o_done completes once per block on slot gg & 1;
+    // this thread has already seen PV of block gg - 2 complete, and PV of
+    // block gg + 2 needs a P that it has not yet written, so parity is exact)
+    auto wait_pv = [&](uint32_t gg) -> bool {
+      return mbar_wait_bounded(&o_done[gg & 1], (gg >> 1) & 1, abort_flag, err);
+    };
     // The output of an item is read out after the next item's first block
     // (its last PV may still be running meanwhile): O / l, stored for the
     // tile's real tokens, then the accumulator is handed back to the MMA warp.
@@ -296,7 +333,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       __half* dst;
     } pend{false, false, 0, 0, 0.f, nullptr};
     auto flush = [&]() -> bool {
-      if (!mbar_wait_bounded(&o_done[pend.g_last & 1], (pend.g_last >> 1) & 1, abort_flag, err)) return false;
+      if (!wait_pv(pend.g_last)) return false;
       tc_fence_after();
       const uint32_t ocol = trow + C::O_COL + pend.buf * HD;
 #pragma unroll 1
@@ -336,39 +373,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       float m_used = 0.f, l = 0.f;
       for (int j = 0; j < n_kv; ++j, ++g) {
         const int b = g & 1;
-        const uint32_t ph = (g >> 1) & 1;
-        // the V block has landed and the V^T / P slot is free once the PV of
-        // two blocks ago has completed: transpose before the scores are ready
-        if (!mbar_wait_bounded(&kv_full[b], ph, abort_flag, err) ||
-            !mbar_wait_bounded(&kv_empty[b], ph ^ 1, abort_flag, err)) {
-          ok = false;
-          break;
-        }
-        // transpose this warp's 16 keys of the V block into the K-major V^T tile
-        {
-          const uint32_t vbase = smem_u32(sV(b));
-          const uint32_t tbase = smem_u32(sVt(b));
-          const int mi = lane >> 3, rr = lane & 7;
-#pragma unroll
-          for (int i = 0; i < HD / 16; ++i) {
-            const int q = 4 * i + mi;           // 8x8 block: key group (q / (HD/8)), dim group (q % (HD/8))
-            const int kg = q / (HD / 8), dg = q % (HD / 8);
-            const int key = quarter * 16 + kg * 8 + rr;
-            const int d = dg * 8;
-            const uint32_t src = vbase + (d / 64) * C::SUB + key * 128 + ((((d % 64) >> 3) ^ (key & 7)) << 4);
-            uint32_t x[4];
-            ldsm_x4_trans(x, src);
-#pragma unroll
-            for (int m = 0; m < 4; ++m) {
-              const int qm = 4 * i + m;
-              const int kgm = qm / (HD / 8), dgm = qm % (HD / 8);
-              const int dd = dgm * 8 + (lane >> 2);
-              const int kk = quarter * 16 + kgm * 8 + 2 * (lane & 3);
-              st_shared_u32(tbase + dd * 128 + ((((kk >> 3) ^ (dd & 7))) << 4) + (kk & 7) * 2, x[m]);
-            }
-          }
-        }
-        if (!mbar_wait_bounded(&s_full[b], ph, abort_flag, err)) {
+        if (!mbar_wait_bounded(&s_full[b], (g >> 1) & 1, abort_flag, err)) {
           ok = false;
           break;
         }
@@ -396,20 +401,19 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         const float mr = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
                                fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
         const float mx = mr * a.scale_log2;
+        // P and V^T are rewritten, and the output may be rescaled, only once
+        // the previous block's PV has completed
+        if (g > 0 && !wait_pv(g - 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
         if (j == 0) {
           m_used = mx == -INFINITY ? 0.f : mx;
         } else {
           const bool grow = mx > m_used + 8.f;
           if (__any_sync(0xffffffffu, grow)) {
-            // rescale this warp's output rows once the previous block's PV is done
-            // (per-slot barrier: PV of block g-3 is already known complete and
-            // PV of block g+1 cannot start before this block's P, so the
-            // parity test cannot alias)
-            if (!mbar_wait_bounded(&o_done[(g - 1) & 1], ((g - 1) >> 1) & 1, abort_flag, err)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
+            // rescale this warp's output rows
             const float f = grow ? ex2_approx(m_used - mx) : 1.f;
             if (grow) {
               l *= f;
@@ -428,7 +432,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
           }
         }
         float2 ps[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-        const uint32_t prow = smem_u32(sP(b)) + r * 128;
+        const uint32_t prow = smem_u32(sP) + r * 128;
         const float2 sc2 = make_float2(a.scale_log2, a.scale_log2), nm2 = make_float2(-m_used, -m_used);
 #pragma unroll
         for (int ch = 0; ch < 8; ++ch) {
@@ -444,9 +448,43 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
           st_shared_v4(prow + ((ch ^ (r & 7)) << 4), make_uint4(pk[0], pk[1], pk[2], pk[3]));
         }
         l += ((ps[0].x + ps[0].y) + (ps[1].x + ps[1].y)) + ((ps[2].x + ps[2].y) + (ps[3].x + ps[3].y));
+        // transpose this warp's 16 keys of the V block into the K-major V^T tile,
+        // then hand the V slot back to the producer
+        const int vb = g % NKV;
+        if (!mbar_wait_bounded(&v_full[vb], (g / NKV) & 1, abort_flag, err)) {
+          ok = false;
+          break;
+        }
+        {
+          const uint32_t vbase = smem_u32(sV(vb));
+          const uint32_t tbase = smem_u32(sVt);
+          const int mi = lane >> 3, rr = lane & 7;
+#pragma unroll
+          for (int i = 0; i < HD / 16; ++i) {
+            const int q = 4 * i + mi;           // 8x8 block: key group (q / (HD/8)), dim group (q % (HD/8))
+            const int kg = q / (HD / 8), dg = q % (HD / 8);
+            const int key = quarter * 16 + kg * 8 + rr;
+            const int d = dg * 8;
+            const uint32_t src = vbase + (d / 64) * C::SUB + key * 128 + ((((d % 64) >> 3) ^ (key & 7)) << 4);
+            uint32_t x[4];
+            ldsm_x4_trans(x, src);
+#pragma unroll
+            for (int m = 0; m < 4; ++m) {
+              const int qm = 4 * i + m;
+              const int kgm = qm / (HD / 8), dgm = qm % (HD / 8);
+              const int dd = dgm * 8 + (lane >> 2);
+              const int kk = quarter * 16 + kgm * 8 + 2 * (lane & 3);
+              st_shared_u32(tbase + dd * 128 + ((((kk >> 3) ^ (dd & 7))) << 4) + (kk & 7) * 2, x[m]);
+            }
+          }
+        }
         fence_proxy_async_smem();
+        tc_fence_before();  // this block's score reads are complete
         __syncwarp();
-        if (lane == 0) mbar_arrive(&p_full[b]);
+        if (lane == 0) {
+          mbar_arrive(&v_empty[vb]);
+          mbar_arrive(p_full);
+        }
         if (j == 0 && pend.on && !flush()) {
           ok = false;
           break;
