@@ -267,40 +267,67 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         umma_commit(&s_full[gg & 1]);
         return true;
       };
-      for (int w = blockIdx.x; w < n_work && ok; w += gridDim.x, ++it) {
+      // key blocks of an item (the shared prefix's, then the row's own up to
+      // the tile's last token)
+      auto blocks_of = [&](int w) -> int {
         const int tidx = w / a.Hkv;
         const int s = a.tile_seq[tidx], q0 = a.tile_q0[tidx];
         const int len = a.seq_start[s + 1] - a.seq_start[s];
-        const int q_end = min(q0 + a.TQ, len);
-        const int n_kv = n_pre + (q_end + kKeys - 1) / kKeys;
-        const int qb = it & 1;
-        if (!mbar_wait_bounded(&q_full[qb], (it >> 1) & 1, abort_flag, err)) break;
-        tc_fence_after();
-        // the first scores only need Q and the key block: they are computed
-        // while the softmax warps still read out the previous item's output
-        if (!issue_s(g, qb)) break;
-        for (int j = 0; j < n_kv; ++j, ++g) {
-          if (j + 1 < n_kv && !issue_s(g + 1, qb)) {
-            ok = false;
-            break;
-          }
-          if (j + 1 == n_kv) umma_commit(&q_empty[qb]);  // all S MMAs of this item issued
-          if (!mbar_wait_bounded(p_full, g & 1, abort_flag, err)) {
-            ok = false;
-            break;
-          }
-          // the first PV overwrites this item's accumulator: the softmax warps
-          // must have read out the output of the item two back
-          if (j == 0 && !mbar_wait_bounded(&o_free[qb], ((it >> 1) & 1) ^ 1, abort_flag, err)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
+        return n_pre + (min(q0 + a.TQ, len) + kKeys - 1) / kKeys;
+      };
+      // The blocks of all this CTA's items form one stream: the scores of the
+      // next block, also the first block of the next item, are issued before
+      // this block's PV, so an item boundary costs no extra hand-off.
+      int w = blockIdx.x;
+      if (w < n_work) {
+        int n_kv = blocks_of(w);
+        if (!mbar_wait_bounded(&q_full[0], 0, abort_flag, err) || (tc_fence_after(), !issue_s(g, 0))) ok = false;
+        while (ok) {
+          const int qb = it & 1;
+          const int w_next = w + gridDim.x;
+          const int n_next = w_next < n_work ? blocks_of(w_next) : 0;
+          for (int j = 0; j < n_kv; ++j, ++g) {
+            if (j + 1 < n_kv) {
+              if (!issue_s(g + 1, qb)) {
+                ok = false;
+                break;
+              }
+            } else {
+              umma_commit(&q_empty[qb]);  // all S MMAs of this item issued
+              if (n_next > 0) {
+                const int it1 = it + 1;
+                if (!mbar_wait_bounded(&q_full[it1 & 1], (it1 >> 1) & 1, abort_flag, err)) {
+                  ok = false;
+                  break;
+                }
+                tc_fence_after();
+                if (!issue_s(g + 1, it1 & 1)) {
+                  ok = false;
+                  break;
+                }
+              }
+            }
+            if (!mbar_wait_bounded(p_full, g & 1, abort_flag, err)) {
+              ok = false;
+              break;
+            }
+            // the first PV overwrites this item's accumulator: the softmax warps
+            // must have read out the output of the item two back
+            if (j == 0 && !mbar_wait_bounded(&o_free[qb], ((it >> 1) & 1) ^ 1, abort_flag, err)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
-            umma_f16_ss(tmem_base + C::O_COL + qb * HD, smem_desc_k_sw128(smem_u32(sP) + k * 32),
-                        smem_desc_k_sw128(smem_u32(sVt) + k * 32), idesc_o, (j | k) != 0);
-          umma_commit(&o_done[g & 1]);
+            for (int k = 0; k < 4; ++k)
+              umma_f16_ss(tmem_base + C::O_COL + qb * HD, smem_desc_k_sw128(smem_u32(sP) + k * 32),
+                          smem_desc_k_sw128(smem_u32(sVt) + k * 32), idesc_o, (j | k) != 0);
+            umma_commit(&o_done[g & 1]);
+          }
+          if (!ok || n_next == 0) break;
+          w = w_next;
+          n_kv = n_next;
+          ++it;
         }
       }
       umma_commit(mma_done);
