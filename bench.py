@@ -84,6 +84,11 @@ def make_step(ctx, w, q, model, aiq):
                                         w.label_ids, agg=w.agg)), [table, build]
 
 
+def model_desc(m) -> str:
+    return (f"decoder d{m.d_model} L{m.n_layers} {m.n_heads}/{m.n_kv_heads} heads hd{m.head_dim} "
+            f"ffn{m.d_ffn} V{m.vocab}, random init")
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -238,7 +243,7 @@ def reference_arm(args):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000 * total / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name, "rows": w.n_rows, "model": "1B-shape decoder, random init",
+            "config": {"workload": w.name, "rows": w.n_rows, "model": model_desc(w.model),
                        "sample_rows_per_step": n},
             "cpu_baseline": {"value": value, "unit": "rows/s", "cores": os.cpu_count(), "kind": "oracle",
                              "sample": f"{n} consecutive input rows per step ({cands} LM candidates over "
@@ -361,9 +366,7 @@ def ours(args):
             "dtype": "f16xf16->f32 (bf16 model values)", "data": "synthetic",
             "config": {"workload": w.name, "rows": w.n_rows, "candidates": res.n_candidates,
                        "tokens": res.n_tokens, "prefill_tokens": res.n_prefill_tokens, "chunks": res.n_chunks,
-                       "model": (f"decoder d{w.model.d_model} L{w.model.n_layers} {w.model.n_heads}/"
-                                 f"{w.model.n_kv_heads} heads hd{w.model.head_dim} ffn{w.model.d_ffn} "
-                                 f"V{w.model.vocab}, random init"),
+                       "model": model_desc(w.model),
                        "l2": "2x L2 written between timed steps; weights and activations exceed L2",
                        "parallelism": f"replicas x{world}"},
             "p50_latency_ms": statistics.median(ms),

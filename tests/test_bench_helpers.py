@@ -47,3 +47,25 @@ def test_kernel_rooflines_bounds_and_fractions():
     assert k["rmsnorm"]["bound"] == "hbm" and np.isclose(k["rmsnorm"]["frac"], 0.5)
     assert k["attention"]["bound"] == "tensor" and np.isclose(k["attention"]["achieved"], 300.0)
     assert k["pack_chunk"] == {"ms_per_step": 0.25}
+
+
+def test_reference_arm_json_line_on_the_tiny_workload():
+    """`bench.py --impl reference` (the oracle, on the host cores) prints one
+    JSON line with the contract's keys, describing the workload it ran."""
+    import json
+    import subprocess
+    import sys
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload",
+                        "c1_tiny_select", "--steps", "2", "--warmup", "1"], capture_output=True, text=True,
+                       timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == "AI-query input rows/s" and d["unit"] == "rows/s"
+    assert d["steps"] == 2 and d["warmup"] == 1 and d["higher_is_better"] is True and d["value"] > 0
+    assert d["config"]["workload"] == "c1_tiny_select" and d["config"]["rows"] == synth.C1_TINY.n_rows
+    assert d["config"]["model"].startswith(f"decoder d{synth.C1_TINY.model.d_model} L{synth.C1_TINY.model.n_layers} ")
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
