@@ -25,6 +25,13 @@ import sys
 import threading
 import time
 
+# The CPU oracle (the reference arm and the cpu_baseline leg) runs numpy BLAS on
+# every host core.  torchrun sets OMP_NUM_THREADS=1 for each rank, which would
+# pin the reference arm's rank 0 to one thread: give BLAS the host's cores
+# before numpy loads it.
+if "reference" in sys.argv and os.environ.get("OMP_NUM_THREADS") == "1" and "OPENBLAS_NUM_THREADS" not in os.environ:
+    os.environ["OPENBLAS_NUM_THREADS"] = str(os.cpu_count() or 1)
+
 import numpy as np
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -82,6 +89,23 @@ def make_step(ctx, w, q, model, aiq):
     bpreds = [(p.column, p.op, p.value) for p in w.join_build_preds]
     return (lambda: ctx.run_join_select(build, "movie_id", bpreds, table, "movie_id", model, preds, q.prefix,
                                         w.label_ids, agg=w.agg)), [table, build]
+
+
+def blas_threads() -> int:
+    """Threads the CPU oracle's BLAS runs on: threadpoolctl's report where it
+    is installed, else the thread count OpenBLAS takes from the environment."""
+    try:
+        from threadpoolctl import threadpool_info
+        n = [int(p["num_threads"]) for p in threadpool_info() if p.get("user_api") == "blas"]
+        if n:
+            return max(n)
+    except Exception:
+        pass
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        v = os.environ.get(k, "")
+        if v.isdigit() and int(v) > 0:
+            return int(v)
+    return os.cpu_count() or 1
 
 
 def model_desc(m) -> str:
@@ -245,7 +269,7 @@ def reference_arm(args):
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "rows": w.n_rows, "model": model_desc(w.model),
                        "sample_rows_per_step": n},
-            "cpu_baseline": {"value": value, "unit": "rows/s", "cores": os.cpu_count(), "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": "rows/s", "cores": blas_threads(), "kind": "oracle",
                              "sample": f"{n} consecutive input rows per step ({cands} LM candidates over "
                                        f"{args.steps} steps), fp64 numpy"},
             "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -355,7 +379,7 @@ def ours(args):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline and not w.join_build_rows:
         s, n, c = cpu_oracle_sample(w, q, W, args.cpu_sample_rows)
-        cpu = {"value": n / s, "unit": "rows/s", "cores": os.cpu_count(), "kind": "oracle",
+        cpu = {"value": n / s, "unit": "rows/s", "cores": blas_threads(), "kind": "oracle",
                "sample": f"first {n} input rows ({c} LM candidates), relational + fp64 transformer, numpy"}
 
     if rank == 0:
