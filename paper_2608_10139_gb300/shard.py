@@ -38,8 +38,10 @@ def local_result(res, row_offset: int) -> Dict[str, np.ndarray]:
 
 def merge(parts: Sequence[Dict[str, np.ndarray]]) -> Dict[str, np.ndarray]:
     """Merge rank results given in rank order (rank r covers rows below rank r+1)."""
+    counts = [int(p["count"]) for p in parts]
     out = {
-        "count": np.int64(sum(int(p["count"]) for p in parts)),
+        # a negative count means "not defined for this aggregate" (e.g. K > 2 labels)
+        "count": np.int64(-1 if any(c < 0 for c in counts) else sum(counts)),
         "n_candidates": np.int64(sum(int(p["n_candidates"]) for p in parts)),
         "row_ids": np.concatenate([p["row_ids"] for p in parts]) if parts else np.zeros(0, np.int64),
     }

@@ -78,3 +78,15 @@ def test_shard_ranges_partition():
             assert rs[0][0] == 0 and rs[-1][1] == n
             assert all(a[1] == b[0] for a, b in zip(rs, rs[1:]))
             assert max(h - l for l, h in rs) - min(h - l for l, h in rs) <= 1
+
+
+def test_merge_keeps_a_count_that_the_aggregate_does_not_define():
+    """K > 2 labels report count -1 (undefined); the merge keeps -1 instead of
+    summing it, and sums label counts element-wise."""
+    e = np.zeros(0, np.int64)
+    parts = [{"count": np.int64(-1), "n_candidates": np.int64(n), "row_ids": e,
+              "label_counts": np.array(lc, np.int64), "group_build_rows": e, "group_keys": e, "group_counts": e}
+             for n, lc in ((3, [1, 0, 2, 0, 0]), (4, [0, 1, 1, 1, 1]))]
+    m = shard.merge(parts)
+    assert int(m["count"]) == -1 and int(m["n_candidates"]) == 7
+    assert m["label_counts"].tolist() == [1, 1, 3, 1, 1]
