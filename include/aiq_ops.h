@@ -92,9 +92,10 @@ typedef struct {
  * of caller-owned device columns that satisfy every term, written to ids_out
  * (device, room for n_rows ids), and their number to *count_out (device int64).
  * The paper has no counterpart: this is for callers that must not allocate
- * device memory while they run (work recorded into a CUDA graph, a worker
- * confined to a fixed device arena, an operator inside another library's
- * allocation-free loop).  It runs the same kernels as aiq_run_select's
+ * device memory while they run (a worker confined to a fixed device arena, an
+ * operator inside another engine's allocation-free loop, a latency-bound path
+ * that cannot take cudaMalloc's implicit synchronisation or its failure under
+ * memory pressure).  It runs the same kernels as aiq_run_select's
  * relational phase, asynchronously on `stream` (a cudaStream_t; NULL = the
  * legacy default stream), with their scratch in one static device array of
  * about 2.1 MB that every GPU loading the library keeps until the process exits.
@@ -102,12 +103,17 @@ typedef struct {
  *   - No cudaMalloc, cudaFree or allocating library call is made.  The first
  *     call on a device looks up the array's device address once
  *     (cudaGetSymbolAddress) with that device current; make that first call
- *     before any stream capture.
+ *     before any stream capture.  The address is cached for the life of the
+ *     process: after a cudaDeviceReset of a device, do not call this entry
+ *     point on that device again.
  *   - All calls share the one array: two calls whose work overlaps on the GPU
  *     (different streams, or different host threads on one device) race and
  *     both results are undefined.  Calls ordered on one stream are safe; each
  *     call rewrites every scratch word it reads.
- *   - Errors are returned as aiq_status, described by aiq_last_error(). */
+ *   - n_rows == 0 writes 0 to *count_out and nothing to ids_out.
+ *   - Errors are returned as aiq_status, described by aiq_last_error(); a
+ *     failed kernel launch gives AIQ_ERR_CUDA and leaves ids_out and
+ *     *count_out undefined. */
 aiq_status aiq_filter_compact_static(const aiq_term* terms, int32_t n_terms, int64_t n_rows, int32_t* ids_out,
                                      int64_t* count_out, void* stream);
 

@@ -1,20 +1,24 @@
 // Allocation-free variant of the predicate + order-preserving compaction.
 //
 // Some callers cannot allocate device memory at the time they run a filter:
-// code recorded into a CUDA graph (cudaMalloc is not a capturable operation),
 // a database worker that is handed a fixed device arena and must not grow
-// the process's footprint, or an operator called from inside another
-// library's allocation-free execution loop.  aiq_filter_compact_static gives
-// them the same kernels as the query path (predicate bitmask, tile-count
-// scan, compaction), with their scratch (bitmask, tile counts, tile offsets)
-// held in one file-scope device array instead of a context's workspace.
+// the process's footprint, an operator called from inside another engine's
+// allocation-free execution loop, or a latency-bound path that cannot afford
+// cudaMalloc's implicit device-wide synchronisation or its failure under
+// memory pressure.  aiq_filter_compact_static gives them the same kernels as
+// the query path (predicate bitmask, tile-count scan, compaction), with their
+// scratch (bitmask, tile counts, tile offsets) held in one file-scope device
+// array instead of a context's workspace.
 //
 // The array is a global of this shared library: every GPU that loads the
 // library keeps kStaticScratchBytes reserved on it until the process exits.
 // Host code cannot pass `g_filter_scratch` itself to a kernel (in host code
 // that name is a host-side shadow, not a device address): the device address
 // is obtained once per device with cudaGetSymbolAddress, with that device
-// current, on the first call made on that device.
+// current, on the first call made on that device, and cached.  A
+// cudaDeviceReset in this process invalidates the cached address; the cache
+// is not refreshed, so a process that resets a device must not call this
+// entry point on it afterwards.
 #include <mutex>
 #include <string>
 
@@ -108,7 +112,13 @@ aiq_status aiq_filter_compact_static(const aiq_term* terms, int32_t n_terms, int
   launch_scan_counts(counts, tiles, offsets, s);
   launch_compact(bits, offsets, n_rows, ids_out, nullptr, nullptr, s);
   k_copy_count<<<1, 1, 0, s>>>(offsets + tiles, count_out);
-  cudaError_t e = cudaGetLastError();
+  // A failed predicate launch is recorded (and its CUDA error consumed) by its
+  // launcher; take that record here so that it is reported by this call and
+  // not left behind for the next call on this host thread.
+  const char* what = nullptr;
+  const cudaError_t le = take_launch_error(&what);
+  const cudaError_t e = cudaGetLastError();
+  if (le != cudaSuccess) return static_fail(AIQ_ERR_CUDA, what, le);
   if (e != cudaSuccess) return static_fail(AIQ_ERR_CUDA, "kernel launch", e);
   return AIQ_OK;
 }
