@@ -154,11 +154,19 @@ typedef int64_t aiq_table;
 typedef int64_t aiq_model;
 typedef int64_t aiq_result_h;
 
-/* Creates a context on CUDA device `device` with its own stream.  Options
- * come from the environment: AIQ_DEVICE_BYTES_MAX caps the bytes the context
- * may allocate (AIQ_ERR_OOM beyond it). */
+/* Section 3 (opening): the whole AI query, relational operators and LLM
+ * inference together, runs as one program on one accelerator.  A context is
+ * that accelerator: CUDA device `device`, one stream on which every step of a
+ * query is issued, and the device memory that holds the resident tables,
+ * models and the query workspace.  Options come from the environment:
+ * AIQ_DEVICE_BYTES_MAX caps the bytes the context may allocate (AIQ_ERR_OOM
+ * beyond it).  *out is owned by the caller until aiq_shutdown.  Errors:
+ * AIQ_ERR_INVALID_ARG (NULL out, no such device), AIQ_ERR_UNSUPPORTED (not an
+ * sm_103 GPU), AIQ_ERR_CUDA (the device cannot be initialised). */
 aiq_status aiq_init(int device, aiq_ctx** out);
-/* Frees every table, model, result and buffer of the context. */
+/* Section 3 (opening): ends the context of aiq_init.  Frees every table,
+ * model, result and buffer of the context; ctx is invalid afterwards.  NULL
+ * is ignored. */
 void aiq_shutdown(aiq_ctx* ctx);
 
 /* Table 1, FROM row: copy n_cols columns of n_rows rows to the device.
@@ -168,7 +176,11 @@ void aiq_shutdown(aiq_ctx* ctx);
 aiq_status aiq_load_table(aiq_ctx* ctx, const aiq_column* cols, int32_t n_cols, int64_t n_rows, aiq_table* out);
 aiq_status aiq_free_table(aiq_ctx* ctx, aiq_table table);
 
-/* Copy a model's weights (host bf16 bit patterns, uint16) to the device.
+/* Fig. 2: the semantic operator is a causal-LM forward pass whose weights
+ * live on the accelerator beside the table; Section 3.2: the model is the AI
+ * operator's template that the compiled program calls.  Copies a model's
+ * weights (host bf16 bit patterns, uint16; the caller keeps its buffers) to
+ * the device, where they stay resident until aiq_free_model.
  * Tensor order, linear weights in [out_features, in_features] layout:
  *   embed [V, d];
  *   per layer: attn_norm [d], wq [Hq*hd, d], wk [Hkv*hd, d], wv [Hkv*hd, d],
@@ -243,7 +255,15 @@ aiq_status aiq_run_transform(aiq_ctx* ctx, aiq_table table, aiq_model model, con
 aiq_status aiq_run_pair_select(aiq_ctx* ctx, aiq_table table, int32_t key_column, aiq_model model,
                                const aiq_select* q, aiq_result_h* out);
 
+/* Section 3.3 (H2D boundary consolidation): only a query's final results
+ * cross back to the host, never its masks, activations or logits (the
+ * per-candidate logits only on request, the paper's debug outputs of Table 2
+ * Q5).  Fills *out with host pointers to those results; they stay valid until
+ * aiq_result_free of the same handle.  Errors: AIQ_ERR_NOT_FOUND (unknown
+ * handle), AIQ_ERR_INVALID_ARG (NULL out). */
 aiq_status aiq_result(aiq_ctx* ctx, aiq_result_h result, aiq_result_view* out);
+/* Section 3.3: releases the host copy of a query's results; the view's
+ * pointers are invalid afterwards.  AIQ_ERR_NOT_FOUND for an unknown handle. */
 aiq_status aiq_result_free(aiq_ctx* ctx, aiq_result_h result);
 
 /* Thread-local description of the last failure on this thread ("" if none). */
@@ -256,7 +276,10 @@ const char* aiq_last_error(void);
  * "attention_tc" (0/1, default 1: tcgen05 attention where the head shape
  * allows), "decode_rows" (aiq_run_transform: rows per prefill chunk, which
  * decode together, default 4096; the chunk's token budget grows to fit them,
- * up to 2^20 tokens and 32 GB of cached prompt keys/values). */
+ * up to 2^20 tokens and 32 GB of cached prompt keys/values), "device_bytes_max"
+ * (the context's device byte cap, as AIQ_DEVICE_BYTES_MAX at aiq_init; <= 0
+ * lifts it; memory already held stays, only further growth is refused with
+ * AIQ_ERR_OOM). */
 aiq_status aiq_set_option(aiq_ctx* ctx, const char* name, int64_t value);
 
 /* The context's CUDA stream (a cudaStream_t), for callers that time the

@@ -14,6 +14,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "aiq.h"
 #include "aiq_ops.h"
 #include "common.cuh"
@@ -138,6 +140,30 @@ cudaError_t aiq::take_launch_error(const char** what) {
   if (what) *what = g_launch_what.c_str();
   return e;
 }
+
+namespace {
+// NVTX ranges (host issue time) that name a query's phases for profilers:
+// "relational", "prefill" (with one "prefix" and one "chunk" range per token
+// chunk inside it) and "aggregate".  begin() closes the previous phase.
+class NvtxPhase {
+ public:
+  NvtxPhase() = default;
+  explicit NvtxPhase(const char* name) { begin(name); }
+  ~NvtxPhase() { end(); }
+  void begin(const char* name) {
+    end();
+    nvtxRangePushA(name);
+    open_ = true;
+  }
+  void end() {
+    if (open_) nvtxRangePop();
+    open_ = false;
+  }
+
+ private:
+  bool open_ = false;
+};
+}  // namespace
 
 struct aiq_ctx {
   int device = 0;
@@ -826,6 +852,7 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
   if (P > 0) {
     // the shared prefix once: its per-layer keys/values and its last hidden state
     AIQ_TRY(ws(c, "pf.prefix_kv", static_cast<int64_t>(g.n_layers) * P * ldkv, &pkv));
+    NvtxPhase pr("prefix");
     launch_pack_prefix(prefix_d, P, pb.tok, pb.pos, pb.seq_start, c->stream);
     counted(c, 1);
     AIQ_TRY(run_layers(c, m, pb, P, 1, nullptr, 0, pkv, false));
@@ -836,6 +863,7 @@ aiq_status prefill_phase(aiq_ctx* c, const TableD& t, ModelD& m, const aiq_selec
     const int64_t r0 = chunks[2 * i], r1 = chunks[2 * (i + 1)];
     const int64_t Tc = chunks[2 * (i + 1) + 1] - chunks[2 * i + 1];
     if (r1 <= r0) continue;
+    NvtxPhase chunk_range("chunk");
     {
       ProfScope p(c, "pack_chunk", 0, 0);
       launch_pack_chunk(cu, st->ids, col.offsets, static_cast<const int32_t*>(col.data), P, r0, r1, pb.tok, pb.pos,
@@ -1055,6 +1083,8 @@ aiq_status run_query(aiq_ctx* c, const TableD* build, int32_t build_key, const a
   c->launches = 0;
   cudaEvent_t ev[4];
   for (auto& e : ev) e = take_event(c);
+  NvtxPhase whole(build ? "aiq_run_join_select" : "aiq_run_select");
+  NvtxPhase phase("relational");
   CUDA_TRY(cudaEventRecord(ev[0], c->stream));
   QueryState st;
   ProbeSpec pr;
@@ -1096,13 +1126,16 @@ aiq_status run_query(aiq_ctx* c, const TableD* build, int32_t build_key, const a
     }
   }
   if (!rel_only) {
+    phase.begin("prefill");
     AIQ_TRY(prefill_phase(c, probe, *m, q, &st));
     CUDA_TRY(cudaEventRecord(ev[2], c->stream));
+    phase.begin("aggregate");
     AIQ_TRY(aggregate_phase(c, q, &st, build, build_key, R, &probe));
   } else {
     CUDA_TRY(cudaEventRecord(ev[2], c->stream));
   }
   CUDA_TRY(cudaEventRecord(ev[3], c->stream));
+  phase.end();
   AIQ_TRY(sync_and_check(c));
   float t01 = 0, t12 = 0, t23 = 0, t03 = 0;
   cudaEventElapsedTime(&t01, ev[0], ev[1]);
@@ -1163,10 +1196,13 @@ aiq_status run_transform(aiq_ctx* c, const TableD& t, ModelD* m, const aiq_selec
   c->launches = 0;
   cudaEvent_t ev[4];
   for (auto& e : ev) e = take_event(c);
+  NvtxPhase whole("aiq_run_transform");
+  NvtxPhase phase("relational");
   CUDA_TRY(cudaEventRecord(ev[0], c->stream));
   QueryState st;
   AIQ_TRY(filter_compact(c, t, ps, ProbeSpec{}, "sel", &st.S, &st.ids, nullptr));
   CUDA_TRY(cudaEventRecord(ev[1], c->stream));
+  phase.begin("prefill");
   const int64_t S = st.S;
   const int W = gen->max_new_tokens;
   GenPlan gp;
@@ -1177,6 +1213,7 @@ aiq_status run_transform(aiq_ctx* c, const TableD& t, ModelD* m, const aiq_selec
   AIQ_TRY(ws(c, "g.len", std::max<int64_t>(S, 1), &gp.len));
   AIQ_TRY(prefill_phase(c, t, *m, q, &st, &gp));
   CUDA_TRY(cudaEventRecord(ev[2], c->stream));
+  phase.begin("aggregate");
 
   ResultH R;
   R.gen_max_new = W;
@@ -1290,6 +1327,8 @@ aiq_status run_pair_select(aiq_ctx* c, const TableD& t, int32_t key_col, ModelD*
   c->launches = 0;
   cudaEvent_t ev[4];
   for (auto& e : ev) e = take_event(c);
+  NvtxPhase whole("aiq_run_pair_select");
+  NvtxPhase phase("relational");
   CUDA_TRY(cudaEventRecord(ev[0], c->stream));
   int64_t S = 0;
   int32_t* ids;
@@ -1339,10 +1378,13 @@ aiq_status run_pair_select(aiq_ctx* c, const TableD& t, int32_t key_col, ModelD*
       CUDA_TRY(cudaMemcpyAsync(R.cand_build.data(), st.ids2, n_pairs * 4, cudaMemcpyDeviceToHost, c->stream));
     }
   }
+  phase.begin("prefill");
   AIQ_TRY(prefill_phase(c, t, *m, q, &st));
   CUDA_TRY(cudaEventRecord(ev[2], c->stream));
+  phase.begin("aggregate");
   AIQ_TRY(aggregate_phase(c, q, &st, nullptr, -1, R));
   CUDA_TRY(cudaEventRecord(ev[3], c->stream));
+  phase.end();
   AIQ_TRY(sync_and_check(c));
   float t01 = 0, t12 = 0, t23 = 0, t03 = 0;
   cudaEventElapsedTime(&t01, ev[0], ev[1]);
@@ -1750,6 +1792,11 @@ aiq_status aiq_set_option(aiq_ctx* c, const char* name, int64_t value) {
   }
   if (!std::strcmp(name, "attention_tc")) {
     c->attention_tc = value != 0;
+    return AIQ_OK;
+  }
+  if (!std::strcmp(name, "device_bytes_max")) {
+    // 0 lifts the cap; a cap below what is already allocated only stops growth
+    c->bytes_max = value <= 0 ? SIZE_MAX : static_cast<size_t>(value);
     return AIQ_OK;
   }
   return fail(AIQ_ERR_INVALID_ARG, std::string("unknown option ") + name);
