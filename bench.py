@@ -27,10 +27,11 @@ import time
 
 # The CPU oracle (the reference arm and the cpu_baseline leg) runs numpy BLAS on
 # every host core.  torchrun sets OMP_NUM_THREADS=1 for each rank, which would
-# pin the reference arm's rank 0 to one thread: give BLAS the host's cores
-# before numpy loads it.
-if "reference" in sys.argv and os.environ.get("OMP_NUM_THREADS") == "1" and "OPENBLAS_NUM_THREADS" not in os.environ:
-    os.environ["OPENBLAS_NUM_THREADS"] = str(os.cpu_count() or 1)
+# pin the reference arm's rank 0 to one thread: give every BLAS flavour the
+# host's cores before numpy loads it.
+if "reference" in sys.argv and os.environ.get("OMP_NUM_THREADS") == "1":
+    for _k in ("OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "OMP_NUM_THREADS"):
+        os.environ[_k] = str(os.cpu_count() or 1)
 
 import numpy as np
 
@@ -58,7 +59,10 @@ def parse():
     p.add_argument("--rows", type=int, default=0, help="override the table size (testing)")
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--cpu-sample-rows", type=int, default=64)
+    p.add_argument("--cpu-sample-candidates", type=int, default=16,
+                   help="CPU oracle: LM candidates per step (stratified by prompt length)")
+    p.add_argument("--relational-micro-rows", type=int, default=1 << 28,
+                   help="rows of the predicate + compaction micro-measurement in the default line (0: skip)")
     p.add_argument("--micro", default="", choices=["", "relational"],
                    help="relational: predicate + compaction alone on a 2^28-row table, against HBM bandwidth")
     p.add_argument("--micro-rows", type=int, default=1 << 28)
@@ -92,8 +96,9 @@ def make_step(ctx, w, q, model, aiq):
 
 
 def blas_threads() -> int:
-    """Threads the CPU oracle's BLAS runs on: threadpoolctl's report where it
-    is installed, else the thread count OpenBLAS takes from the environment."""
+    """Threads the CPU oracle's BLAS actually runs on: threadpoolctl's report
+    where it is installed, else OpenBLAS's own answer through the library
+    numpy has loaded, else the environment's setting."""
     try:
         from threadpoolctl import threadpool_info
         n = [int(p["num_threads"]) for p in threadpool_info() if p.get("user_api") == "blas"]
@@ -101,7 +106,27 @@ def blas_threads() -> int:
             return max(n)
     except Exception:
         pass
-    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+    try:
+        import ctypes
+        libs = set()
+        with open("/proc/self/maps") as fh:
+            for line in fh:
+                path = line.split()[-1] if "/" in line else ""
+                if "openblas" in os.path.basename(path).lower():
+                    libs.add(path)
+        for path in sorted(libs):
+            lib = ctypes.CDLL(path)
+            for sym in ("scipy_openblas_get_num_threads64_", "openblas_get_num_threads64_",
+                        "openblas_get_num_threads"):
+                f = getattr(lib, sym, None)
+                if f is not None:
+                    f.restype = ctypes.c_int
+                    n = int(f())
+                    if n > 0:
+                        return n
+    except Exception:
+        pass
+    for k in ("OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "OMP_NUM_THREADS"):
         v = os.environ.get(k, "")
         if v.isdigit() and int(v) > 0:
             return int(v)
@@ -190,19 +215,55 @@ def gemm_source_sha():
 
 # ------------------------------------------------------------ CPU oracle ---
 
-def cpu_oracle_sample(w, q, W, n_rows: int, start: int = 0):
-    """The oracle on input rows [start, start + n_rows): relational terms, then
-    the fp64 transformer on the survivors, then the aggregate.  Returns
-    (seconds, rows, candidates)."""
+def oracle_candidates(w, q):
+    """The oracle's relational phase on the whole table (the join for the
+    reviews-movies workload): candidate rows that reach the LM, ascending."""
     from oracle import query as oq
-    from oracle import transformer as tf
-    sub = synth.Table(n_rows, {k: v[start:start + n_rows] for k, v in q.table.cols.items()},
-                      q.table.offsets[start:start + n_rows + 1] - q.table.offsets[start],
-                      q.table.tokens[q.table.offsets[start]:q.table.offsets[start + n_rows]])
+    from oracle import relational as rel
+    if w.join_build_rows:
+        bp = [(p.column, p.op, p.value) for p in w.join_build_preds]
+        pp = [(p.column, p.op, p.value) for p in w.preds]
+        return oq.join_candidates(q.table, q.build, "movie_id", "movie_id", pp, bp)[0]
     preds = [(p.column, p.op, p.value) for p in w.preds]
+    return rel.compact(rel.predicate_mask(q.table.cols, preds, q.table.n_rows))
+
+
+def stratified_sample(lens: np.ndarray, m: int, seed: int) -> np.ndarray:
+    """m candidate positions, one from each of m equal-count strata of the
+    candidates sorted by prompt length (seeded pick inside each stratum), so
+    that every sample spans the length distribution."""
+    n = len(lens)
+    if n == 0:
+        return np.zeros(0, np.int64)
+    m = min(m, n)
+    order = np.argsort(lens, kind="stable")
+    edges = np.linspace(0, n, m + 1).astype(np.int64)
+    rng = np.random.default_rng(seed)
+    pick = [order[rng.integers(edges[i], edges[i + 1])] for i in range(m) if edges[i + 1] > edges[i]]
+    return np.sort(np.array(pick, dtype=np.int64))
+
+
+def cpu_oracle_step(w, q, model, m: int, seed: int):
+    """One bounded step of the CPU oracle as it stands: its relational phase
+    on the whole table, then its fp64 transformer on m stratified candidates.
+    The query's time is extrapolated from the sample by prompt tokens (the
+    transformer's cost is linear in them up to the small attention term).
+    Returns (step seconds, extrapolated query seconds, candidates, sample size)."""
+    from oracle import query as oq
+    from oracle import relational as rel
+    from oracle import transformer as tf
     t0 = time.perf_counter()
-    o = oq.run_select(sub, q.prefix, preds, w.label_ids, w.agg, tf.Model(w.model, W))
-    return time.perf_counter() - t0, n_rows, len(o.cand_rows)
+    cand = oracle_candidates(w, q)
+    t_rel = time.perf_counter() - t0
+    lens = (np.diff(q.table.offsets)[cand] + len(q.prefix)).astype(np.float64)
+    pos = stratified_sample(lens, m, seed)
+    t1 = time.perf_counter()
+    if len(pos):
+        z = tf.label_logits(model, oq.prompts(q.prefix, q.table.offsets, q.table.tokens, cand[pos]), w.label_ids)
+        rel.decide(z)
+    t_lm = time.perf_counter() - t1
+    scale = float(lens.sum() / lens[pos].sum()) if len(pos) else 0.0
+    return t_rel + t_lm, t_rel + t_lm * scale, len(cand), len(pos)
 
 
 def attention_flops_host(w, q) -> float:
@@ -245,33 +306,40 @@ def kernel_rooflines(stats, steps, pk, attn_flops) -> dict:
 
 
 def reference_arm(args):
-    """The CPU oracle as it stands, timed on this host's cores, on a bounded
-    sample of the workload per step (rank 0 only)."""
+    """The CPU oracle as it stands, timed on this host's cores (rank 0 only):
+    each step runs the relational phase on the whole table and the fp64
+    transformer on a stratified sample of candidates (a different seeded
+    sample per step), and the query's rows/s is extrapolated from it."""
     rank, world, _ = dist_env()
     if rank != 0:
         return
+    from oracle import transformer as tf
     w = workload(args)
     q = synth.make_inputs(w)
-    W = synth.make_weights(w.model, w.weight_seed)
-    n = args.cpu_sample_rows
-    for i in range(args.warmup):
-        cpu_oracle_sample(w, q, W, n, start=(i * n) % (w.n_rows - n))
-    times, cands = [], 0
+    model = tf.Model(w.model, synth.make_weights(w.model, w.weight_seed))
+    m = args.cpu_sample_candidates
+    for i in range(args.warmup):            # warm-up steps: one candidate each
+        cpu_oracle_step(w, q, model, 1, w.data_seed + 100 + i)
+    steps, extrap, n_cand, n_sampled = [], [], 0, 0
     for k in range(args.steps):
-        s, _, c = cpu_oracle_sample(w, q, W, n, start=((args.warmup + k) * n) % (w.n_rows - n))
-        times.append(s)
-        cands += c
-    total = sum(times)
-    value = n * args.steps / total
+        s, e, n_cand, ns = cpu_oracle_step(w, q, model, m, w.data_seed + k)
+        steps.append(s)
+        extrap.append(e)
+        n_sampled += ns
+    value = w.n_rows / statistics.mean(extrap)
+    threads = blas_threads()
+    sample = (f"per step: relational phase on all {w.n_rows} rows, fp64 transformer on {m} of the {n_cand} "
+              f"LM candidates (one per prompt-length stratum, new seed each step; {n_sampled} in all), "
+              f"query time extrapolated by prompt tokens")
     line = {"impl": "reference", "metric": "AI-query input rows/s", "value": value, "unit": "rows/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": 1000 * total / args.steps, "higher_is_better": True, "scaling": "weak",
+            "ms_per_step": 1000 * statistics.mean(steps), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "rows": w.n_rows, "model": model_desc(w.model),
-                       "sample_rows_per_step": n},
-            "cpu_baseline": {"value": value, "unit": "rows/s", "cores": blas_threads(), "kind": "oracle",
-                             "sample": f"{n} consecutive input rows per step ({cands} LM candidates over "
-                                       f"{args.steps} steps), fp64 numpy"},
+                       "sample_candidates_per_step": m},
+            "extrapolated_query_s": statistics.mean(extrap),
+            "cpu_baseline": {"value": value, "unit": "rows/s", "cores": threads, "host_cores": os.cpu_count(),
+                             "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -376,11 +444,20 @@ def ours(args):
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         e2e_per = float(t.item())
 
+    micro = None
+    if rank == 0 and world == 1 and args.relational_micro_rows > 0:
+        micro = relational_micro(ctx, aiq, args.relational_micro_rows, 5, 2)
+
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and not w.join_build_rows:
-        s, n, c = cpu_oracle_sample(w, q, W, args.cpu_sample_rows)
-        cpu = {"value": n / s, "unit": "rows/s", "cores": blas_threads(), "kind": "oracle",
-               "sample": f"first {n} input rows ({c} LM candidates), relational + fp64 transformer, numpy"}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        from oracle import transformer as tf
+        m = args.cpu_sample_candidates
+        s, e, n_cand, ns = cpu_oracle_step(w, q, tf.Model(w.model, W), m, w.data_seed)
+        cpu = {"value": w.n_rows / e, "unit": "rows/s", "cores": blas_threads(), "host_cores": os.cpu_count(),
+               "kind": "oracle", "seconds": round(s, 1),
+               "sample": f"relational phase on all {w.n_rows} rows, fp64 transformer on {ns} of the {n_cand} "
+                         f"LM candidates (one per prompt-length stratum, seed {w.data_seed}); query time "
+                         f"extrapolated by prompt tokens"}
 
     if rank == 0:
         line = {
@@ -407,6 +484,7 @@ def ours(args):
                          "peak_source": f"{src} bf16_tflops_sustained (fp16 dense rate = bf16)",
                          "launches": gemm_launches},
             "cpu_baseline": cpu,
+            "relational_micro": micro,
             "e2e": ({"value": world * w.n_rows / (e2e_per / 1000.0), "unit": "rows/s",
                      "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_per}
                     if e2e_ms else None),
@@ -419,39 +497,35 @@ def ours(args):
         torch.distributed.destroy_process_group()
 
 
-def micro_relational(args):
+def relational_micro(ctx, aiq, n: int, steps: int, warmup: int) -> dict:
     """Predicate (rating >= 4 AND year >= 2000) + order-preserving compaction
-    over a 2^28-row table of two int32 columns, timed per kernel with events."""
-    import torch
-    from paper_2608_10139_gb300 import aiq
-    from paper_2608_10139_gb300 import build as _build
-    _build.build()
-    n = args.micro_rows
+    over an n-row table of two int32 columns (rating uniform 1..5, year
+    uniform 1950..2024), each kernel timed with CUDA events on the library's
+    stream, against the measured HBM copy bandwidth.  The table is far larger
+    than L2, so every step reads it from HBM."""
     rng = np.random.Generator(np.random.PCG64(7))
     cols = {"rating": rng.integers(1, 6, n, dtype=np.int32), "year": rng.integers(1950, 2025, n, dtype=np.int32)}
     preds = [("rating", aiq.GE, 4), ("year", aiq.GE, 2000)]
-    ctx = aiq.Context(0)
     t = ctx.load_table(cols, n_rows=n)
-    for _ in range(args.warmup):
+    del cols
+    for _ in range(warmup):
         ctx.run_select(t, 0, preds, [], [0, 1], flags=aiq.FLAG_RELATIONAL_ONLY)
     ctx.reset_kernel_stats()
     ctx.set_option("profile", 1)
-    clocks = ClockSampler(0)
-    clocks.start()
     totals = []
-    for _ in range(args.steps):
+    for _ in range(steps):
         r = ctx.run_select(t, 0, preds, [], [0, 1], flags=aiq.FLAG_RELATIONAL_ONLY)
         totals.append(r.ms_relational)
-    clk = clocks.stop()
+    ctx.set_option("profile", 0)
     st = ctx.kernel_stats()
+    ctx.free_table(t)
     S = r.n_candidates
     pk, src = peaks()
-    mask_ms = st["predicate_mask"]["total_ms"] / args.steps
-    comp_ms = st["compact"]["total_ms"] / args.steps
+    mask_ms = st["predicate_mask"]["total_ms"] / steps
+    comp_ms = st["compact"]["total_ms"] / steps
     mask_bytes = 8.0 * n + n / 8          # two int32 columns read, 1 bit/row written
     comp_bytes = n / 8 + 4.0 * S          # bitmask read, survivor ids written
-    line = {"metric": "relational predicate + compaction HBM throughput", "rows": n, "survivors": S,
-            "steps": args.steps, "warmup": args.warmup,
+    return {"rows": n, "survivors": S, "steps": steps, "warmup": warmup,
             "predicate_mask": {"ms": mask_ms, "GB/s": mask_bytes / mask_ms / 1e6,
                                "frac": mask_bytes / mask_ms / 1e6 / pk["hbm_gbs"]},
             "compact": {"ms": comp_ms, "GB/s": comp_bytes / comp_ms / 1e6,
@@ -459,8 +533,20 @@ def micro_relational(args):
             "combined": {"ms": mask_ms + comp_ms, "GB/s": (mask_bytes + comp_bytes) / (mask_ms + comp_ms) / 1e6,
                          "frac": (mask_bytes + comp_bytes) / (mask_ms + comp_ms) / 1e6 / pk["hbm_gbs"]},
             "query_relational_ms_p50": statistics.median(totals),
-            "peak": {"hbm_gbs": pk["hbm_gbs"], "source": src}, "clocks": clk}
-    print(json.dumps(line), flush=True)
+            "peak": {"hbm_gbs": pk["hbm_gbs"], "source": f"{src} hbm_gbs"}}
+
+
+def micro_relational(args):
+    """`--micro relational`: the relational micro-measurement alone, one JSON line."""
+    from paper_2608_10139_gb300 import aiq
+    from paper_2608_10139_gb300 import build as _build
+    _build.build()
+    ctx = aiq.Context(0)
+    clocks = ClockSampler(0)
+    clocks.start()
+    d = relational_micro(ctx, aiq, args.micro_rows, args.steps, args.warmup)
+    d = {"metric": "relational predicate + compaction HBM throughput", **d, "clocks": clocks.stop()}
+    print(json.dumps(d), flush=True)
     ctx.close()
 
 

@@ -69,3 +69,36 @@ def test_reference_arm_json_line_on_the_tiny_workload():
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
     assert d["e2e"] == {"value": d["value"], "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_reference_arm_runs_the_join_workload():
+    """The reference arm times the oracle's join (movies year >= 2010, reviews
+    joined on movie id) on a scaled-down reviews-movies workload."""
+    import json
+    import subprocess
+    import sys
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload",
+                        "c3_join_1b", "--rows", "2000", "--steps", "1", "--warmup", "1",
+                        "--cpu-sample-candidates", "1"], capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    d = json.loads([ln for ln in r.stdout.splitlines() if ln.startswith("{")][0])
+    assert d["config"]["workload"] == "c3_join_1b_n2000" and d["value"] > 0
+    assert "of the" in d["cpu_baseline"]["sample"] and d["cpu_baseline"]["cores"] >= 1
+
+
+def test_stratified_sample_spans_the_length_distribution():
+    b = _bench()
+    lens = np.random.default_rng(3).lognormal(np.log(120), 0.5, 5000)
+    pos = b.stratified_sample(lens, 16, 9)
+    assert len(pos) == 16 and len(set(pos.tolist())) == 16 and np.all(np.diff(pos) > 0)
+    # one pick per sixteenth of the sorted lengths
+    ranks = np.argsort(np.argsort(lens, kind="stable"), kind="stable")[pos]
+    assert sorted((ranks * 16) // 5000) == list(range(16))
+    assert np.array_equal(pos, b.stratified_sample(lens, 16, 9))          # seeded
+    assert len(b.stratified_sample(lens[:5], 16, 9)) == 5                  # fewer candidates than strata
+    assert len(b.stratified_sample(lens[:0], 16, 9)) == 0
+
+
+def test_blas_threads_reports_a_positive_count():
+    b = _bench()
+    assert b.blas_threads() >= 1
