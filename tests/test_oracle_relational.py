@@ -39,7 +39,7 @@ def test_compare_ops_match_python(op, pyop):
     assert got.tolist() == [pyop(int(v), 2) for v in vals]
 
 
-@pytest.mark.parametrize("n", [0, 1, 31, 32, 33, 1000])
+@pytest.mark.parametrize("n", [0, 1, 31, 32, 33, 1000, 4096, 4097, 100_003])
 def test_compaction_brute_force(n):
     rng = np.random.default_rng(n)
     cols = {"a": rng.integers(0, 10, n).astype(np.int32), "b": rng.integers(-5, 5, n).astype(np.int64)}
@@ -139,3 +139,36 @@ def test_masked_sum_hand_cases_and_exactness():
     assert abs(exact - float(np.sum(np.sort(r.astype(np.float64))))) < 1e-9
     agg = oq.aggregate(oq.AGG_SUM, dec, cand, 2, sum_values=vals)
     assert agg == {"count": 3, "sum": 110}
+
+
+def test_margins_hand_worked():
+    """K = 2: z_yes - z_no.  K = 5: z_k - z_{k*} for every k, with k* the
+    reference decision when one is given (else the first argmax)."""
+    z2 = np.array([[2.0, 0.5], [-1.0, 3.0], [0.25, 0.25]])
+    assert rel.margins(z2).tolist() == [1.5, -4.0, 0.0]
+    z5 = np.array([[1.0, 3.5, 3.5, -2.0, 0.25],
+                   [0.0, -1.0, -2.0, -3.0, 4.0]])
+    # own argmax: row 0 -> label 1 (first of the tied maxima), row 1 -> label 4
+    assert rel.margins(z5).tolist() == [[-2.5, 0.0, 0.0, -5.5, -3.25],
+                                        [-4.0, -5.0, -6.0, -7.0, 0.0]]
+    # a reference decision that is not this row's own argmax is used as given
+    assert rel.margins(z5, np.array([4, 0])).tolist() == [[0.75, 3.25, 3.25, -2.25, 0.0],
+                                                          [0.0, -1.0, -2.0, -3.0, 4.0]]
+
+
+def test_parity_comparison_rule_on_hand_cases():
+    """The tests' margin comparison (tolerance 2e-2 * max(1, |ref|), decisions
+    equal on clear rows) accepts and rejects the cases it should."""
+    from helpers import compare_logits
+    ref = np.array([[1.0, 3.5, 3.49, -2.0, 0.25],       # runner-up 0.01 below: not clear
+                    [0.0, -1.0, -2.0, -3.0, 4.0]])      # clear
+    ok = ref + np.array([[0.0, 0.0, 0.015, 0.0, 0.0],   # flips the near tie within 0.02: allowed
+                         [0.01, 0.0, 0.0, 0.0, -0.05]])  # within 2e-2 * |margin| (4 -> 0.08)
+    compare_logits(ok, ref)
+    bad = ref + np.array([[0.0, 0.0, 0.0, 0.0, 0.0], [0.0, 0.0, 0.0, 0.0, -0.2]])
+    with pytest.raises(AssertionError):
+        compare_logits(bad, ref)                        # margin error 0.2 > 0.08
+    ref2 = np.array([[0.3, 0.0], [0.01, 0.0]])
+    compare_logits(np.array([[0.29, 0.0], [-0.005, 0.0]]), ref2)  # |0.01| <= 0.1: may flip
+    with pytest.raises(AssertionError):
+        compare_logits(np.array([[0.3, 0.31], [0.01, 0.0]]), ref2)  # clear row flipped
