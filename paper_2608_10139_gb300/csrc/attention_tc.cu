@@ -9,20 +9,30 @@
 //   warp 0    TMA: the Q tile (3-D box hd x heads x tokens) into one of two
 //             slots, then K and V blocks of 64 keys into two separate rings of
 //             NKV slots (128-byte swizzle).  A K slot is free once the S MMA
-//             that read it has completed, a V slot once the softmax warps have
-//             transposed it, so a block's loads are issued NKV blocks before
-//             its scores are needed instead of one.
-//   warp 1    tcgen05.mma: S = Q K^T into one of two TMEM score buffers, and
-//             O += P V^T into the item's TMEM output accumulator.
+//             that read it has completed, a V slot once the PV MMA that read
+//             it has, so a block's loads are issued NKV blocks ahead.
+//   warp 1    tcgen05.mma: S = Q K^T into one of two 64-column TMEM score
+//             buffers, and O += P V into the item's TMEM output accumulator,
+//             with P read from TMEM (it overwrites its own scores) and V read
+//             as an MN-major operand straight from its TMA tile.
 //   warps 2-5 one query row per thread: read its 64 scores with tcgen05.ld,
 //             apply the causal / prefix / length mask, keep the running max
 //             (the output is rescaled only when the max grows by more than
-//             2^8, so P never exceeds 256), write exp2(s - max) as fp16 into
-//             the swizzled P tile, then transpose their quarter of the V block
-//             into the K-major V^T tile with ldmatrix.trans (P and V^T are
-//             rewritten once the previous block's PV has completed); an item's
-//             output is divided by the row sum and stored after the next
-//             item's first block.
+//             2^8, so P never exceeds 256), and write exp2(s - max) as fp16
+//             pairs back over the first 32 columns of the same score buffer
+//             with tcgen05.st; an item's output is divided by the row sum and
+//             stored after the next item's first block.
+//
+// Ordering without extra waits: the MMA warp issues S(g+1) before PV(g), and
+// tcgen05 MMAs of one thread run in issue order, so S(g+2), which reuses the
+// score buffer of block g, only starts after PV(g) has read P(g).  The commit
+// that signals S(g) tracks every earlier MMA of the thread, so a softmax
+// thread that has seen S(g) complete knows PV(g-2) has too: its parity waits
+// on the two PV barriers can never be a full phase behind.  The softmax warps
+// signal P on one barrier per score buffer: S(g+1) is ready before PV(g) is
+// issued, so one warp may finish block g+1 while another still writes P(g),
+// and on a single barrier its second arrival would complete block g's phase
+// early; a warp cannot reach block g+2 before PV(g), so two barriers suffice.
 // Work items are persistent per CTA; every wait is bounded.
 #include <cudaTypedefs.h>
 
@@ -42,15 +52,11 @@ struct ACfg {
   static constexpr int Q_BYTES = 128 * HD * 2;   // 128 rows
   static constexpr int SUB = 64 * 128;           // one [64 x 64] fp16 sub-tile
   static constexpr int K_BYTES = NC * SUB;
-  static constexpr int VT_BYTES = HD * 128;      // HD rows x 64 keys
-  static constexpr int P_BYTES = 128 * 128;      // 128 rows x 64 keys
   static constexpr int OFF_Q = 0;                // two slots
   static constexpr int OFF_K = OFF_Q + 2 * Q_BYTES;
   static constexpr int OFF_V = OFF_K + NKV * K_BYTES;
-  static constexpr int OFF_VT = OFF_V + NKV * K_BYTES;
-  static constexpr int OFF_P = OFF_VT + VT_BYTES;
-  static constexpr int OFF_BAR = OFF_P + P_BYTES;
-  static constexpr int N_BARS = 4 + 4 * NKV + 2 + 1 + 2 + 2 + 1;
+  static constexpr int OFF_BAR = OFF_V + NKV * K_BYTES;
+  static constexpr int N_BARS = 4 + 4 * NKV + 2 + 2 + 2 + 2 + 1;
   static constexpr int SMEM = 1024 + OFF_BAR + N_BARS * 8 + 16;
   // two 64-column score buffers, then two HD-column output accumulators (one
   // per alternating work item), rounded up to a power of two
@@ -111,18 +117,27 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   return bits_f2(r);
 }
 
-__device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t saddr) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(saddr));
+// MN-major operand (N contiguous) in the 128-byte swizzle: rows of 64 N
+// elements, 8-row groups 1024 B apart along K, 64-column atoms 8 KB apart along N.
+__device__ __forceinline__ uint64_t smem_desc_mn_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(lbo >> 4) << 16;
+  d |= static_cast<uint64_t>(sbo >> 4) << 32;
+  d |= static_cast<uint64_t>(1u) << 46;
+  d |= static_cast<uint64_t>(2u) << 61;
+  return d;
 }
 
-__device__ __forceinline__ void st_shared_u32(uint32_t saddr, uint32_t v) {
-  asm volatile("st.shared.u32 [%0], %1;" ::"r"(saddr), "r"(v) : "memory");
-}
-__device__ __forceinline__ void st_shared_v4(uint32_t saddr, uint4 v) {
-  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(saddr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
-               : "memory");
+// D (TMEM) (+)= A (TMEM: lane = row, two fp16 per 32-bit column along K) * B (smem).
+__device__ __forceinline__ void umma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
 }
 
 template <int HD>
@@ -139,10 +154,10 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
   uint64_t* k_full = bars + 4;             // [NKV]
   uint64_t* k_empty = k_full + NKV;        // [NKV]: the S MMA of the block has completed
   uint64_t* v_full = k_empty + NKV;        // [NKV]
-  uint64_t* v_empty = v_full + NKV;        // [NKV]: the softmax warps have transposed the block
+  uint64_t* v_empty = v_full + NKV;        // [NKV]: the PV MMA of the block has completed
   uint64_t* s_full = v_empty + NKV;        // [2]
-  uint64_t* p_full = s_full + 2;           // P and V^T of the block written
-  uint64_t* o_done = p_full + 1;           // [2]: PV of block g commits o_done[g & 1]
+  uint64_t* p_full = s_full + 2;           // [2]: P of block g written over its scores (score buffer g & 1)
+  uint64_t* o_done = p_full + 2;           // [2]: PV of block g commits o_done[g & 1]
   uint64_t* o_free = o_done + 2;           // [2]: output accumulator it & 1 read out
   uint64_t* mma_done = o_free + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
@@ -150,8 +165,6 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
   auto sQ = [&](int b) { return smem + C::OFF_Q + b * C::Q_BYTES; };
   auto sK = [&](int b) { return smem + C::OFF_K + b * C::K_BYTES; };
   auto sV = [&](int b) { return smem + C::OFF_V + b * C::K_BYTES; };
-  uint8_t* sVt = smem + C::OFF_VT;
-  uint8_t* sP = smem + C::OFF_P;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   int* err = a.err;
@@ -160,6 +173,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       mbar_init(&q_full[b], 1);
       mbar_init(&q_empty[b], 1);
       mbar_init(&s_full[b], 1);
+      mbar_init(&p_full[b], 4);
       mbar_init(&o_done[b], 1);
       mbar_init(&o_free[b], 4);
     }
@@ -167,9 +181,8 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       mbar_init(&k_full[b], 1);
       mbar_init(&k_empty[b], 1);
       mbar_init(&v_full[b], 1);
-      mbar_init(&v_empty[b], 4);
+      mbar_init(&v_empty[b], 1);
     }
-    mbar_init(p_full, 4);
     mbar_init(mma_done, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -248,7 +261,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
     if (lane == 0) {
       // ------------------------------------------------------------ MMA
       constexpr uint32_t idesc_s = idesc_f16_f32(128, kKeys);
-      constexpr uint32_t idesc_o = idesc_f16_f32(128, HD);
+      constexpr uint32_t idesc_o = idesc_f16_f32(128, HD) | (1u << 16);  // B (= V) MN-major
       uint32_t g = 0;
       int it = 0;
       bool ok = true;
@@ -307,7 +320,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
                 }
               }
             }
-            if (!mbar_wait_bounded(p_full, g & 1, abort_flag, err)) {
+            if (!mbar_wait_bounded(&p_full[g & 1], (g >> 1) & 1, abort_flag, err)) {
               ok = false;
               break;
             }
@@ -317,11 +330,18 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
               ok = false;
               break;
             }
+            const int vb = g % NKV;
+            if (!mbar_wait_bounded(&v_full[vb], (g / NKV) & 1, abort_flag, err)) {
+              ok = false;
+              break;
+            }
             tc_fence_after();
 #pragma unroll
             for (int k = 0; k < 4; ++k)
-              umma_f16_ss(tmem_base + C::O_COL + qb * HD, smem_desc_k_sw128(smem_u32(sP) + k * 32),
-                          smem_desc_k_sw128(smem_u32(sVt) + k * 32), idesc_o, (j | k) != 0);
+              umma_f16_ts(tmem_base + C::O_COL + qb * HD, tmem_base + (g & 1) * kKeys + k * 8,
+                          smem_desc_mn_sw128(smem_u32(sV(vb)) + k * 2048, HD == 64 ? 1024u : 8192u, 1024u),
+                          idesc_o, (j | k) != 0);
+            umma_commit(&v_empty[vb]);
             umma_commit(&o_done[g & 1]);
           }
           if (!ok || n_next == 0) break;
@@ -428,19 +448,17 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         const float mr = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
                                fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
         const float mx = mr * a.scale_log2;
-        // P and V^T are rewritten, and the output may be rescaled, only once
-        // the previous block's PV has completed
-        if (g > 0 && !wait_pv(g - 1)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
         if (j == 0) {
           m_used = mx == -INFINITY ? 0.f : mx;
         } else {
           const bool grow = mx > m_used + 8.f;
           if (__any_sync(0xffffffffu, grow)) {
-            // rescale this warp's output rows
+            // rescale this warp's output rows once the previous block's PV is done
+            if (!wait_pv(g - 1)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
             const float f = grow ? ex2_approx(m_used - mx) : 1.f;
             if (grow) {
               l *= f;
@@ -459,59 +477,23 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
           }
         }
         float2 ps[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-        const uint32_t prow = smem_u32(sP) + r * 128;
         const float2 sc2 = make_float2(a.scale_log2, a.scale_log2), nm2 = make_float2(-m_used, -m_used);
+        uint32_t pk[32];
 #pragma unroll
-        for (int ch = 0; ch < 8; ++ch) {
-          uint32_t pk[4];
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const float2 x = ffma2(make_float2(v[ch * 8 + 2 * i], v[ch * 8 + 2 * i + 1]), sc2, nm2);
-            const float2 p = make_float2(ex2_approx(x.x), ex2_approx(x.y));
-            ps[i] = fadd2(ps[i], p);
-            __half2 h = __floats2half2_rn(p.x, p.y);
-            pk[i] = *reinterpret_cast<uint32_t*>(&h);
-          }
-          st_shared_v4(prow + ((ch ^ (r & 7)) << 4), make_uint4(pk[0], pk[1], pk[2], pk[3]));
+        for (int i = 0; i < 32; ++i) {
+          const float2 x = ffma2(make_float2(v[2 * i], v[2 * i + 1]), sc2, nm2);
+          const float2 p = make_float2(ex2_approx(x.x), ex2_approx(x.y));
+          ps[i & 3] = fadd2(ps[i & 3], p);
+          __half2 h = __floats2half2_rn(p.x, p.y);
+          pk[i] = *reinterpret_cast<uint32_t*>(&h);
         }
         l += ((ps[0].x + ps[0].y) + (ps[1].x + ps[1].y)) + ((ps[2].x + ps[2].y) + (ps[3].x + ps[3].y));
-        // transpose this warp's 16 keys of the V block into the K-major V^T tile,
-        // then hand the V slot back to the producer
-        const int vb = g % NKV;
-        if (!mbar_wait_bounded(&v_full[vb], (g / NKV) & 1, abort_flag, err)) {
-          ok = false;
-          break;
-        }
-        {
-          const uint32_t vbase = smem_u32(sV(vb));
-          const uint32_t tbase = smem_u32(sVt);
-          const int mi = lane >> 3, rr = lane & 7;
-#pragma unroll
-          for (int i = 0; i < HD / 16; ++i) {
-            const int q = 4 * i + mi;           // 8x8 block: key group (q / (HD/8)), dim group (q % (HD/8))
-            const int kg = q / (HD / 8), dg = q % (HD / 8);
-            const int key = quarter * 16 + kg * 8 + rr;
-            const int d = dg * 8;
-            const uint32_t src = vbase + (d / 64) * C::SUB + key * 128 + ((((d % 64) >> 3) ^ (key & 7)) << 4);
-            uint32_t x[4];
-            ldsm_x4_trans(x, src);
-#pragma unroll
-            for (int m = 0; m < 4; ++m) {
-              const int qm = 4 * i + m;
-              const int kgm = qm / (HD / 8), dgm = qm % (HD / 8);
-              const int dd = dgm * 8 + (lane >> 2);
-              const int kk = quarter * 16 + kgm * 8 + 2 * (lane & 3);
-              st_shared_u32(tbase + dd * 128 + ((((kk >> 3) ^ (dd & 7))) << 4) + (kk & 7) * 2, x[m]);
-            }
-          }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();  // this block's score reads are complete
+        // P (fp16 pairs) over the first 32 columns of this block's score buffer
+        tmem_st_32x32b_x32(trow + b * kKeys, pk);
+        tmem_st_wait();
+        tc_fence_before();  // this block's score reads and P writes are complete
         __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&v_empty[vb]);
-          mbar_arrive(p_full);
-        }
+        if (lane == 0) mbar_arrive(&p_full[b]);
         if (j == 0 && pend.on && !flush()) {
           ok = false;
           break;

@@ -267,3 +267,48 @@ def test_attention_tcgen05_matches_mma_sync_kernel(ctx):
         outs.append(_np64(out))
     ctx.set_option("attention_tc", 1)
     _close(outs[0], outs[1], 4e-3, 4e-3, "tcgen05 vs mma.sync attention")
+
+
+@pytest.mark.parametrize("hd,growing", [(64, False), (64, True), (128, True)])
+def test_attention_tcgen05_many_items_per_cta(ctx, hd, growing):
+    """A batch large enough that every persistent CTA of the tcgen05 kernel runs
+    hundreds of work items back to back (item boundaries, alternating output
+    accumulators, read-outs after the next item's first block), against the
+    mma.sync kernel on every element and the oracle on sampled rows.  With
+    growing keys the scores rise along each row, so the running maximum grows
+    by more than 2^8 inside items and the output is rescaled in place."""
+    rng = np.random.default_rng(hd + 17 * growing)
+    Hq, Hkv, P = 32, 8, 64
+    n_rows = 2500 if hd == 64 else 1200          # about 300 work items per CTA either way
+    lens = np.clip(np.round(np.exp(rng.normal(np.log(120.0), 0.5, n_rows))), 1, 512).astype(np.int64)
+    T = int(lens.sum())
+    W = (Hq + 2 * Hkv) * hd
+    starts = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    rows = rng.standard_normal((T, W), dtype=np.float32)
+    pre = rng.standard_normal((P, W), dtype=np.float32)
+    if growing:
+        # keys scaled by 1 + position / 24 (prefix keys at their positions, row keys after them)
+        pos = np.concatenate([np.arange(n) for n in lens]) + P
+        rows[:, Hq * hd:(Hq + Hkv) * hd] *= (1.0 + pos / 24.0)[:, None] * 0.35
+        pre[:, Hq * hd:(Hq + Hkv) * hd] *= (1.0 + np.arange(P) / 24.0)[:, None] * 0.35
+    rows, pre = rows.astype(np.float16), pre.astype(np.float16)
+    pkv = np.ascontiguousarray(pre[:, Hq * hd:])
+    dq, ds, dp = _h(rows), _h(starts), _h(pkv)
+    outs = []
+    for tc in (1, 0):
+        ctx.set_option("attention_tc", tc)
+        out = torch.zeros((T, Hq * hd), dtype=torch.float16, device="cuda")
+        ctx.op_attention(dq.data_ptr(), T, ds.data_ptr(), len(lens), Hq, Hkv, hd, out.data_ptr(), dp.data_ptr(), P)
+        outs.append(_np64(out))
+    ctx.set_option("attention_tc", 1)
+    assert np.isfinite(outs[0]).all()
+    _close(outs[0], outs[1], 4e-3, 4e-3, f"tcgen05 vs mma.sync attention, {T} tokens, hd {hd}")
+    for i in rng.choice(len(lens), 4, replace=False):
+        s, n = int(starts[i]), int(lens[i])
+        seq = np.concatenate([pre, rows[s:s + n]]).astype(np.float64)
+        m = P + n
+        q = seq[:, :Hq * hd].reshape(m, Hq, hd)
+        k = seq[:, Hq * hd:(Hq + Hkv) * hd].reshape(m, Hkv, hd)
+        v = seq[:, (Hq + Hkv) * hd:].reshape(m, Hkv, hd)
+        ref = tf.causal_attention(q, k, v).reshape(m, Hq * hd)[P:]
+        _close(outs[0][s:s + n], ref, 4e-3, 4e-3, f"tcgen05 attention row {i} len {n}")
