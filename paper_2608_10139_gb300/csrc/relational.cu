@@ -26,18 +26,6 @@ namespace {
 constexpr int kThreads = 256;  // 256 threads x 8 rows = kRowsPerBlock
 constexpr unsigned long long kEmptyKey = 0x8000000000000000ull;
 
-template <typename T>
-__device__ __forceinline__ bool cmp(T v, int op, T c) {
-  switch (op) {
-    case 0: return v < c;
-    case 1: return v <= c;
-    case 2: return v > c;
-    case 3: return v >= c;
-    case 4: return v == c;
-    default: return v != c;
-  }
-}
-
 // Raw 8 rows [r0, r0 + 8) of one term's column, as four 16-byte words for
 // 4-byte columns (two used) or 64-bit words for int64 columns.
 struct TermRows {
@@ -71,25 +59,52 @@ __device__ __forceinline__ void load_term(const PredDev& p, int64_t r0, int64_t 
   }
 }
 
-// The term's 8 result bits for rows loaded by load_term.
-__device__ __forceinline__ uint32_t eval_term(const PredDev& p, const TermRows& t) {
+// The term's 8 result bits for rows loaded by load_term.  The operator is
+// resolved once per term (the switch is outside the loop over the 8 values).
+template <typename T>
+__device__ __forceinline__ uint32_t cmp8(const T* v, int op, T c) {
   uint32_t bits = 0;
-  if (p.type == 1) {
-    const int64_t* v = reinterpret_cast<const int64_t*>(t.w);
+  switch (op) {
+    case 0:
 #pragma unroll
-    for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<int64_t>(v[j], p.op, p.ivalue)) << j;
-  } else if (p.type == 0) {
-    // compare in int64 so that constants outside the int32 range behave as in SQL
-    const int32_t* v = reinterpret_cast<const int32_t*>(t.w);
+      for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(v[j] < c) << j;
+      break;
+    case 1:
 #pragma unroll
-    for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<int64_t>(v[j], p.op, p.ivalue)) << j;
-  } else {
-    const float* v = reinterpret_cast<const float*>(t.w);
-    const float fc = static_cast<float>(p.fvalue);
+      for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(v[j] <= c) << j;
+      break;
+    case 2:
 #pragma unroll
-    for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(cmp<float>(v[j], p.op, fc)) << j;
+      for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(v[j] > c) << j;
+      break;
+    case 3:
+#pragma unroll
+      for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(v[j] >= c) << j;
+      break;
+    case 4:
+#pragma unroll
+      for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(v[j] == c) << j;
+      break;
+    default:
+#pragma unroll
+      for (int j = 0; j < 8; ++j) bits |= static_cast<uint32_t>(v[j] != c) << j;
+      break;
   }
   return bits;
+}
+
+__device__ __forceinline__ uint32_t eval_term(const PredDev& p, const TermRows& t) {
+  if (p.type == 1) return cmp8<int64_t>(reinterpret_cast<const int64_t*>(t.w), p.op, p.ivalue);
+  if (p.type == 2) return cmp8<float>(reinterpret_cast<const float*>(t.w), p.op, static_cast<float>(p.fvalue));
+  // int32: a constant outside the int32 range decides every row alike (as the
+  // SQL comparison in int64 would); inside it, compare in 32 bits
+  const int32_t* v = reinterpret_cast<const int32_t*>(t.w);
+  if (p.ivalue > INT32_MAX || p.ivalue < INT32_MIN) {
+    const bool below = p.ivalue > INT32_MAX;  // every value is below the constant
+    const bool r = p.op == 0 || p.op == 1 ? below : (p.op == 2 || p.op == 3 ? !below : p.op == 5);
+    return r ? 0xFFu : 0u;
+  }
+  return cmp8<int32_t>(v, p.op, static_cast<int32_t>(p.ivalue));
 }
 
 __device__ __forceinline__ int probe_lookup(const ProbeSpec& pr, unsigned long long key) {
@@ -186,6 +201,68 @@ __global__ void __launch_bounds__(kThreads) k_predicate_mask(PredSet ps, ProbeSp
   (void)err;
 }
 
+// The common case, 1..4 terms on 4-byte columns and no join probe: every
+// term's loads are issued before the first compare, in a coalesced layout
+// (lane l of warp w takes rows 4l..4l+3 and 128+4l..128+4l+3 of the warp's
+// 256 rows, so one 16-byte load instruction covers 512 contiguous bytes),
+// and eight lanes' nibbles form one bitmask word.  Same bitmask and tile
+// counts as k_predicate_mask.
+template <int NT>
+__global__ void __launch_bounds__(kThreads) k_predicate_mask4(PredSet ps, int64_t n, uint32_t* bits,
+                                                              int32_t* block_counts) {
+  __shared__ int red[kThreads / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t ra = static_cast<int64_t>(blockIdx.x) * kRowsPerBlock + warp * 256 + lane * 4;
+  const int64_t rb = ra + 128;
+  int4 va[NT], vb[NT];
+  const bool full = rb + 4 <= n;
+#pragma unroll
+  for (int i = 0; i < NT; ++i) {
+    const int32_t* c = static_cast<const int32_t*>(ps.p[i].col);
+    if (full) {
+      va[i] = __ldg(reinterpret_cast<const int4*>(c + ra));
+      vb[i] = __ldg(reinterpret_cast<const int4*>(c + rb));
+    } else {
+      int32_t* x = reinterpret_cast<int32_t*>(&va[i]);
+      int32_t* y = reinterpret_cast<int32_t*>(&vb[i]);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        x[j] = ra + j < n ? c[ra + j] : 0;
+        y[j] = rb + j < n ? c[rb + j] : 0;
+      }
+    }
+  }
+  uint32_t byte = 0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) byte |= (static_cast<uint32_t>(ra + j < n) << j) | (static_cast<uint32_t>(rb + j < n) << (4 + j));
+#pragma unroll
+  for (int i = 0; i < NT; ++i) {
+    TermRows t;
+    t.w[0] = va[i];
+    t.w[1] = vb[i];
+    // eval_term's value j < 4 is row ra + j, value 4 + j is row rb + j
+    byte &= eval_term(ps.p[i], t);
+  }
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    uint32_t w = ((byte >> (4 * h)) & 0xFu) << (4 * (lane & 7));
+    w |= __shfl_xor_sync(0xffffffffu, w, 1);
+    w |= __shfl_xor_sync(0xffffffffu, w, 2);
+    w |= __shfl_xor_sync(0xffffffffu, w, 4);
+    if ((lane & 7) == 0) bits[blockIdx.x * int64_t(kRowsPerBlock / 32) + warp * 8 + h * 4 + (lane >> 3)] = w;
+  }
+  int c = __popc(byte);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if (lane == 0) red[warp] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int total = 0;
+    for (int i = 0; i < kThreads / 32; ++i) total += red[i];
+    block_counts[blockIdx.x] = total;
+  }
+}
+
 // Block-wide exclusive scan of one int per thread (kThreads threads).
 __device__ __forceinline__ int block_excl_scan(int v, int* sh, int* total) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -212,63 +289,52 @@ __device__ __forceinline__ int block_excl_scan(int v, int* sh, int* total) {
   return before + x - v;
 }
 
-constexpr int kCompactWarps = 4;  // warps (= 2048-row tiles) per compaction block
+constexpr int kCompactWarps = 4;  // warps (= 2048-row tiles at a time) per compaction block
 
-// One warp per 2048-row tile: each lane owns 64 rows (two bitmask words), a
-// warp shuffle scan gives every lane its output position, the ids are staged
-// in the warp's own shared-memory slice in order and then written out as one
-// coalesced run.  No block-wide barrier is involved.  A payload (the join's
-// build row per probe row) is gathered straight to its output position.
-// Warps are persistent over the tiles (grid-stride) and load the next tile's
-// bitmask words and output offset before they work on the current one, so
-// two tiles' loads are in flight per warp.
+// One warp per 2048-row tile: lane l owns bitmask words l and 32 + l of the
+// tile (two coalesced loads).  In two passes (words 0..31, then 32..63) a warp
+// shuffle scan gives every lane its output position and the lane writes the
+// row offsets of its word's set bits, in order, into the warp's own 16-bit
+// shared-memory slice; the slice is then written out as one coalesced run of
+// ids.  No block-wide barrier is involved.  A payload (the join's build row
+// per probe row) is gathered straight to its output position (PAYLOAD).
+template <bool PAYLOAD>
 __global__ void __launch_bounds__(kCompactWarps * 32) k_compact(const uint32_t* bits, const int64_t* block_offsets,
                                                                 int64_t n, int32_t* ids, const int32_t* payload,
                                                                 int32_t* payload_out) {
-  __shared__ int32_t s_ids[kCompactWarps][kRowsPerBlock];
+  __shared__ uint16_t s_ids[kCompactWarps][kRowsPerBlock];  // row offsets within the tile
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t n_tiles = (n + kRowsPerBlock - 1) / kRowsPerBlock;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * kCompactWarps;
-  int64_t tile = static_cast<int64_t>(blockIdx.x) * kCompactWarps + warp;
-  if (tile >= n_tiles) return;
-  uint2 w2 = reinterpret_cast<const uint2*>(bits + tile * (kRowsPerBlock / 32))[lane];
-  int64_t out = block_offsets[tile];
-  for (; tile < n_tiles; tile += stride) {
-    const int64_t next = tile + stride;
-    uint2 w2n = make_uint2(0u, 0u);
-    int64_t out_n = 0;
-    if (next < n_tiles) {
-      w2n = reinterpret_cast<const uint2*>(bits + next * (kRowsPerBlock / 32))[lane];
-      out_n = block_offsets[next];
-    }
-    const int c = __popc(w2.x) + __popc(w2.y);
-    int incl = c;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += y;
-    }
-    const int total = __shfl_sync(0xffffffffu, incl, 31);
-    int at = incl - c;
-    const int64_t r0 = tile * kRowsPerBlock + lane * 64;
-    uint32_t wd[2] = {w2.x, w2.y};
+  const int64_t tile = static_cast<int64_t>(blockIdx.x) * kCompactWarps + warp;
+  if (tile < n_tiles) {
+    const uint32_t* wt = bits + tile * (kRowsPerBlock / 32);
+    const uint32_t wa = wt[lane], wb = wt[32 + lane];
+    const int64_t out = block_offsets[tile];
+    const int64_t tile0 = tile * kRowsPerBlock;
+    int at0 = 0;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      uint32_t b = wd[h];
+      uint32_t b = h ? wb : wa;
+      const int c = __popc(b);
+      int incl = c;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      int at = at0 + incl - c;
+      const int base = (h * 32 + lane) * 32;
       while (b) {
         const int j = __ffs(b) - 1;
         b &= b - 1;
-        const int64_t r = r0 + 32 * h + j;
-        s_ids[warp][at] = static_cast<int32_t>(r);
-        if (payload_out) payload_out[out + at] = payload[r];  // joins: a gather, written in place
+        s_ids[warp][at] = static_cast<uint16_t>(base + j);
+        if (PAYLOAD) payload_out[out + at] = payload[tile0 + base + j];  // joins: a gather, written in place
         ++at;
       }
+      at0 += __shfl_sync(0xffffffffu, incl, 31);
     }
     __syncwarp();
-    for (int i = lane; i < total; i += 32) ids[out + i] = s_ids[warp][i];
-    __syncwarp();  // the slice is rewritten by the next tile
-    w2 = w2n;
-    out = out_n;
+    for (int i = lane; i < at0; i += 32) ids[out + i] = static_cast<int32_t>(tile0 + s_ids[warp][i]);
   }
 }
 
@@ -500,7 +566,19 @@ void launch_predicate_mask(const PredSet& ps, const ProbeSpec& probe, int64_t n_
                            int32_t* block_counts, int* err, cudaStream_t s) {
   if (n_rows <= 0) return;
   const unsigned grid = blocks_for(n_rows, kRowsPerBlock);
-  k_predicate_mask<<<grid, kThreads, 0, s>>>(ps, probe, n_rows, bits, block_counts, err);
+  bool four = ps.n >= 1 && ps.n <= 4 && !probe.keys;
+  for (int i = 0; i < ps.n; ++i)
+    four = four && ps.p[i].type != 1 && (reinterpret_cast<uintptr_t>(ps.p[i].col) & 15) == 0;
+  if (four) {
+    switch (ps.n) {
+      case 1: k_predicate_mask4<1><<<grid, kThreads, 0, s>>>(ps, n_rows, bits, block_counts); break;
+      case 2: k_predicate_mask4<2><<<grid, kThreads, 0, s>>>(ps, n_rows, bits, block_counts); break;
+      case 3: k_predicate_mask4<3><<<grid, kThreads, 0, s>>>(ps, n_rows, bits, block_counts); break;
+      default: k_predicate_mask4<4><<<grid, kThreads, 0, s>>>(ps, n_rows, bits, block_counts); break;
+    }
+  } else {
+    k_predicate_mask<<<grid, kThreads, 0, s>>>(ps, probe, n_rows, bits, block_counts, err);
+  }
   const cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     char buf[160];
@@ -516,15 +594,11 @@ void launch_scan_counts(const int32_t* counts, int64_t n, int64_t* offsets, cuda
 void launch_compact(const uint32_t* bits, const int64_t* block_offsets, int64_t n_rows, int32_t* ids_out,
                     const int32_t* payload, int32_t* payload_out, cudaStream_t s) {
   if (n_rows <= 0) return;
-  // persistent warps: as many blocks as fit on the device at once, at most one warp per tile
-  int dev = 0, sms = 0, per_sm = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_compact, kCompactWarps * 32, 0);
-  const int64_t need = blocks_for(n_rows, int64_t(kRowsPerBlock) * kCompactWarps);
-  const int64_t resident = std::max<int64_t>(1, static_cast<int64_t>(sms) * std::max(per_sm, 1));
-  const unsigned grid = static_cast<unsigned>(std::min<int64_t>(need, resident));
-  k_compact<<<grid, kCompactWarps * 32, 0, s>>>(bits, block_offsets, n_rows, ids_out, payload, payload_out);
+  const unsigned grid = blocks_for(n_rows, int64_t(kRowsPerBlock) * kCompactWarps);  // one tile per warp
+  if (payload_out)
+    k_compact<true><<<grid, kCompactWarps * 32, 0, s>>>(bits, block_offsets, n_rows, ids_out, payload, payload_out);
+  else
+    k_compact<false><<<grid, kCompactWarps * 32, 0, s>>>(bits, block_offsets, n_rows, ids_out, payload, payload_out);
 }
 
 void launch_hash_build(const int64_t* keys, const int32_t* rows, int64_t n, unsigned long long* table_keys,

@@ -50,7 +50,7 @@ PRED_SETS = [
 ]
 
 
-@pytest.mark.parametrize("n", [0, 1, 31, 2047, 2048, 2049, 100_003, 1 << 24])
+@pytest.mark.parametrize("n", [0, 1, 31, 2047, 2048, 2049, 100_003, (1 << 22) + 777, 1 << 24])
 def test_filter_compaction_bit_exact(ctx, n):
     t = _random_table(n, n)
     ref_t = ctx.load_table(t.cols, n_rows=n)
