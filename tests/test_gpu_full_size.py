@@ -1,7 +1,17 @@
 """Parity at the workloads' full sizes, in the launch configuration the
 benchmark times (default token budget): relational results and aggregates in
 full, bit-exact; label logits of a seeded sample of candidates against the
-fp64 oracle, each candidate row run alone."""
+fp64 oracle, each candidate row run alone.
+
+The large samples (hundreds of candidates per workload) come from
+tests/golden/oracle_logits_<workload>.json, written by
+tests/golden/make_oracle_samples.py from the oracle alone and keyed by the
+sha256 of the oracle's and the input generator's sources; a few of those rows
+are recomputed by the oracle here, on this machine, as a cross-check of the
+stored values."""
+import importlib.util
+import json
+import os
 from dataclasses import replace
 
 import numpy as np
@@ -24,6 +34,50 @@ def ctx():
     c.close()
 
 
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _samples_module():
+    spec = importlib.util.spec_from_file_location("make_oracle_samples",
+                                                  os.path.join(GOLDEN, "make_oracle_samples.py"))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    return mod
+
+
+def cached_oracle(w):
+    """The stored oracle sample of workload w, after checking that it was made
+    from the current oracle and input-generator sources and the same seeds."""
+    mod = _samples_module()
+    path = os.path.join(GOLDEN, f"oracle_logits_{w.name}.json")
+    assert os.path.exists(path), f"{path} missing: run tests/golden/make_oracle_samples.py --only {w.name}"
+    with open(path) as fh:
+        d = json.load(fh)
+    key = mod.key_of(w, d["sample_k"])
+    stale = [k for k, v in key.items() if d.get(k) != v]
+    assert not stale, f"{path} is stale ({', '.join(stale)}): rerun make_oracle_samples.py --only {w.name}"
+    return d
+
+
+def check_cached(w, r, model, q, n_live=3):
+    """GPU label logits at the stored sample positions against the stored
+    oracle logits (margins within tolerance, decisions on every clear row);
+    the first n_live stored rows are recomputed by the oracle here."""
+    d = cached_oracle(w)
+    pos = np.asarray(d["positions"], np.int64)
+    ref = np.asarray(d["logits"], np.float64)
+    assert r.n_candidates == d["n_candidates"]
+    assert np.array_equal(r.cand_row_ids[pos], np.asarray(d["row_ids"], np.int32))
+    worst = compare_logits(r.label_logits[pos], ref, f"{w.name} ({len(pos)} stored oracle rows)")
+    live = oq.prompts(q.prefix, q.table.offsets, q.table.tokens, np.asarray(d["row_ids"][:n_live]))
+    z = tf.label_logits(model, live, w.label_ids)
+    np.testing.assert_allclose(z, ref[:n_live], rtol=1e-9, atol=1e-9)
+    dec = rel.decide(ref)
+    print(f"{w.name}: {len(pos)} stored rows, worst margin error / tolerance {worst:.3f}, "
+          f"{int((rel.decide(r.label_logits[pos]) == dec).sum())} decisions equal")
+    return worst
+
+
 def _sample(n_cand, k, seed, lens=None):
     """k seeded candidate positions; always include the shortest and longest prompt."""
     rng = np.random.default_rng(seed)
@@ -33,7 +87,9 @@ def _sample(n_cand, k, seed, lens=None):
     return np.array(sorted(pick), dtype=np.int64)
 
 
-def _run_select_full(ctx, w, k_sample):
+def _run_select_full(ctx, w, k_sample, stored=False):
+    """The full query on the GPU; its logits checked on k_sample candidates
+    the oracle computes here, or (stored) on the stored oracle sample."""
     q = synth.make_inputs(w)
     W = synth.make_weights(w.model, w.weight_seed)
     m = ctx.load_model(w.model, weights_list(w.model, W))
@@ -46,15 +102,19 @@ def _run_select_full(ctx, w, k_sample):
     assert np.array_equal(r.cand_row_ids, cand)
     lens = np.diff(q.table.offsets)[cand]
     assert r.n_tokens == int(lens.sum()) + len(q.prefix) * len(cand)
-    sample = _sample(len(cand), k_sample, w.data_seed, lens)
-    o = oq.run_select(q.table, q.prefix, preds, w.label_ids, w.agg, tf.Model(w.model, W), sample=sample)
-    compare_logits(r.label_logits[sample], o.logits, w.name)
+    model = tf.Model(w.model, W)
+    if stored:
+        check_cached(w, r, model, q)
+    else:
+        sample = _sample(len(cand), k_sample, w.data_seed, lens)
+        o = oq.run_select(q.table, q.prefix, preds, w.label_ids, w.agg, model, sample=sample)
+        compare_logits(r.label_logits[sample], o.logits, w.name)
     agg = oq.aggregate(w.agg, r.decisions, cand, len(w.label_ids))
     return r, agg
 
 
 def test_c2_select_1b_full_size(ctx):
-    r, agg = _run_select_full(ctx, synth.C2_SELECT, 10)
+    r, agg = _run_select_full(ctx, synth.C2_SELECT, 0, stored=True)
     assert r.count == agg["count"] == len(r.row_ids)
     assert np.array_equal(r.row_ids, agg["row_ids"])
     # rating uniform 1..5 and year uniform 1950..2024: P = 2/5 * 25/75 = 13.3 %
@@ -77,10 +137,7 @@ def test_c3_join_1b_full_size(ctx):
     cand, cand_b = oq.join_candidates(q.table, q.build, "movie_id", "movie_id", [], bp)
     assert np.array_equal(r.cand_row_ids, cand)
     assert np.array_equal(r.cand_build_rows, cand_b)
-    sample = _sample(len(cand), 8, w.data_seed)
-    o = oq.run_join_select(q.table, q.build, "movie_id", "movie_id", [], bp, q.prefix, w.label_ids, w.agg,
-                           tf.Model(w.model, W), sample=sample)
-    compare_logits(r.label_logits[sample], o.logits, w.name)
+    check_cached(w, r, tf.Model(w.model, W), q)
     agg = oq.aggregate(w.agg, r.decisions, cand, 2, cand_b, q.build.cols["movie_id"])
     assert np.array_equal(r.group_build_rows, agg["group_build_rows"])
     assert np.array_equal(r.group_keys, agg["group_keys"])
