@@ -98,3 +98,58 @@ def test_join_shards_merge_to_the_unsharded_result(ctx):
     ctx.free_model(m)
     assert len(full["group_build_rows"]) > 0
     _check_merge(full, parts)
+
+
+def _plan(ctx, run, q, world):
+    """The ranks' row ranges, from the library's relational-only pass over the
+    whole table (the first thing every rank does in the multi-GPU benchmark)."""
+    cand = run([], aiq.FLAG_RELATIONAL_ONLY).cand_row_ids
+    toks = len(q.prefix) + np.diff(q.table.offsets)[cand]
+    return shard.token_balanced_ranges(q.table.n_rows, cand, toks, world)
+
+
+@pytest.mark.parametrize("name", list(SELECT_CASES))
+@pytest.mark.parametrize("world", [2, 4])
+def test_row_range_terms_on_one_table_merge_to_the_unsharded_result(ctx, name, world):
+    """The benchmark's multi-GPU step, one rank after another: every rank holds
+    the whole table plus its row-id column, plans token-balanced ranges from a
+    relational-only pass, runs the query restricted by the two row-id terms,
+    and the merged results equal the unsharded query's."""
+    w = SELECT_CASES[name]
+    q = synth.make_inputs(w)
+    m = ctx.load_model(w.model, weights_list(w.model, synth.make_weights(w.model, w.weight_seed)))
+    t = ctx.load_table(shard.with_row_ids(q.table.cols, q.table.n_rows), (q.table.offsets, q.table.tokens))
+    preds = oracle_preds(w.preds)
+
+    def run(extra, flags=0):
+        return ctx.run_select(t, m, preds + extra, q.prefix, w.label_ids, agg=w.agg, flags=flags)
+
+    full = shard.local_result(run([]), 0)
+    ranges = _plan(ctx, run, q, world)
+    parts = [shard.local_result(run(shard.range_terms(lo, hi)), 0) for lo, hi in ranges]
+    ctx.free_table(t)
+    ctx.free_model(m)
+    assert sum(int(p["n_candidates"]) for p in parts) == int(full["n_candidates"]) > 0
+    _check_merge(full, parts)
+
+
+def test_row_range_terms_on_the_join_probe_side(ctx):
+    w = replace(synth.C3_JOIN, name="c3_tiny_ranges", n_rows=4000, join_build_rows=500, model=synth.TINY,
+                text=synth.TextRecipe("lognormal", 16, 120, median=40.0), prefix_len=16)
+    q = synth.make_inputs(w)
+    m = ctx.load_model(w.model, weights_list(w.model, synth.make_weights(w.model, w.weight_seed)))
+    tb = ctx.load_table(q.build.cols, n_rows=q.build.n_rows)
+    tp = ctx.load_table(shard.with_row_ids(q.table.cols, q.table.n_rows), (q.table.offsets, q.table.tokens))
+    bp = oracle_preds(w.join_build_preds)
+
+    def run(extra, flags=0):
+        return ctx.run_join_select(tb, "movie_id", bp, tp, "movie_id", 0 if flags else m, extra, q.prefix,
+                                   w.label_ids, agg=synth.AGG_GROUP_BUILD_KEY, flags=flags)
+
+    full = shard.local_result(run([]), 0)
+    parts = [shard.local_result(run(shard.range_terms(lo, hi)), 0) for lo, hi in _plan(ctx, run, q, 3)]
+    for h in (tb, tp):
+        ctx.free_table(h)
+    ctx.free_model(m)
+    assert len(full["group_build_rows"]) > 0
+    _check_merge(full, parts)
