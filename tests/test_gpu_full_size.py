@@ -171,6 +171,23 @@ def test_c5_sweep_1pct_full_query(ctx):
     assert np.array_equal(r.row_ids, agg["row_ids"])
 
 
+@pytest.mark.slow
+def test_c5_sweep_100pct_fixed_text_full_query(ctx):
+    """Every one of the 1M rows reaches the model (64-token texts): the longest
+    chunk loop of the sweep, checked on the stored oracle sample."""
+    w = synth.sweep_workload("100%", "fixed")
+    r, agg = _run_select_full(ctx, w, 0, stored=True)
+    assert r.n_candidates == w.n_rows and r.n_chunks > 1
+    assert np.array_equal(r.row_ids, agg["row_ids"])
+
+
+@pytest.mark.slow
+def test_c5_sweep_25pct_lognormal_full_query(ctx):
+    w = synth.sweep_workload("25%", "lognormal")
+    r, agg = _run_select_full(ctx, w, 0, stored=True)
+    assert np.array_equal(r.row_ids, agg["row_ids"])
+
+
 def test_transform_c2_select_1b_full_size(ctx):
     """AI_TRANSFORM over the select workload's 13,050 candidates (1B shape) in
     the benchmark's launch configuration (decode batches of ~4096 rows): row
