@@ -192,7 +192,9 @@ def test_attention_with_shared_prefix(ctx, hd, Hq, Hkv, P):
 
 @pytest.mark.parametrize("pair", [0, 1])
 @pytest.mark.parametrize("M,N,K,epi", [(512, 256, 128, 0), (1000, 512, 2048, 0), (4099, 1536, 512, 2),
-                                       (4099, 1536, 512, 5), (3000, 2048, 256, 3), (70000, 1024, 256, 0)])
+                                       (4099, 1536, 512, 5), (3000, 2048, 256, 3), (70000, 1024, 256, 0),
+                                       (1024, 512, 8192, 2),   # the down projection's depth
+                                       (600, 256, 192, 0)])    # K % 128 != 0: CTA pairs fall back to one CTA
 def test_gemm_cta_pair_vs_single(ctx, pair, M, N, K, epi):
     """256 x 256 tiles on CTA pairs (tcgen05 cta_group::2) and 128 x 256 tiles on
     single CTAs give the oracle's product, ragged M included."""
