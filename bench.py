@@ -56,6 +56,8 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="c2_select_1b")
     p.add_argument("--rows", type=int, default=0, help="override the table size (testing)")
+    p.add_argument("--token-budget", type=int, default=0,
+                   help="prefill tokens per chunk (0: the library default); small values keep profiler captures small")
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-sample-candidates", type=int, default=16,
@@ -395,6 +397,8 @@ def ours(args):
     tensors = [W[n] for n, _, _ in synth.weight_specs(w.model)]
     preds = [(p.column, p.op, p.value) for p in w.preds]
     ctx = aiq.Context(local)
+    if args.token_budget:
+        ctx.set_option("token_budget", args.token_budget)
     model = ctx.load_model(w.model, tensors)
     step, tables = make_step(ctx, w, q, model, aiq, world, rank)
     stream = torch.cuda.ExternalStream(ctx.stream())

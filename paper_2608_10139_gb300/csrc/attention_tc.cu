@@ -10,7 +10,11 @@
 //             slots, then K and V blocks of 64 keys into two separate rings of
 //             NKV slots (128-byte swizzle).  A K slot is free once the S MMA
 //             that read it has completed, a V slot once the PV MMA that read
-//             it has, so a block's loads are issued NKV blocks ahead.
+//             it has, so a block's loads are issued NKV blocks ahead.  The
+//             same thread publishes each item's bounds (sequence start and
+//             length, first token, key/value head) in a four-slot shared
+//             ring, so the softmax warps never wait on global loads between
+//             items.
 //   warp 1    tcgen05.mma: S = Q K^T into one of two 64-column TMEM score
 //             buffers, and O += P V into the item's TMEM output accumulator,
 //             with P read from TMEM (it overwrites its own scores) and V read
@@ -21,7 +25,9 @@
 //             2^8, so P never exceeds 256), and write exp2(s - max) as fp16
 //             pairs back over the first 32 columns of the same score buffer
 //             with tcgen05.st; an item's output is divided by the row sum and
-//             stored after the next item's first block.
+//             stored after the next item's first block: through a shared
+//             staging tile and one TMA store when all the tile's tokens
+//             belong to its sequence, row by row otherwise.
 //
 // Ordering without extra waits: the MMA warp issues S(g+1) before PV(g), and
 // tcgen05 MMAs of one thread run in issue order, so S(g+2), which reuses the
@@ -55,8 +61,10 @@ struct ACfg {
   static constexpr int OFF_Q = 0;                // two slots
   static constexpr int OFF_K = OFF_Q + 2 * Q_BYTES;
   static constexpr int OFF_V = OFF_K + NKV * K_BYTES;
-  static constexpr int OFF_BAR = OFF_V + NKV * K_BYTES;
-  static constexpr int N_BARS = 4 + 4 * NKV + 2 + 2 + 2 + 2 + 1;
+  static constexpr int OFF_OUT = OFF_V + NKV * K_BYTES;  // output staging tile (TMA store source)
+  static constexpr int OFF_INFO = OFF_OUT + Q_BYTES;     // item bounds ring, 4 x int4
+  static constexpr int OFF_BAR = OFF_INFO + 4 * 16;
+  static constexpr int N_BARS = 4 + 4 * NKV + 2 + 2 + 2 + 2 + 1 + 4 + 4 + 2;
   static constexpr int SMEM = 1024 + OFF_BAR + N_BARS * 8 + 16;
   // two 64-column score buffers, then two HD-column output accumulators (one
   // per alternating work item), rounded up to a power of two
@@ -117,6 +125,14 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   return bits_f2(r);
 }
 
+// Shared -> global tile copy by the TMA unit (3-D box), in a bulk async-group.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* smem_src, int x, int y, int z) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.tile.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z), "r"(smem_u32(smem_src))
+               : "memory");
+}
+
 // MN-major operand (N contiguous) in the 128-byte swizzle: rows of 64 N
 // elements, 8-row groups 1024 B apart along K, 64-column atoms 8 KB apart along N.
 __device__ __forceinline__ uint64_t smem_desc_mn_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
@@ -143,7 +159,7 @@ __device__ __forceinline__ void umma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
 template <int HD>
 __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
     k_attention_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kv,
-                   const __grid_constant__ CUtensorMap tm_pre, AttnArgs a) {
+                   const __grid_constant__ CUtensorMap tm_pre, const __grid_constant__ CUtensorMap tm_out, AttnArgs a) {
   using C = ACfg<HD>;
   constexpr int NKV = C::NKV;
   extern __shared__ uint8_t smem_raw[];
@@ -160,7 +176,13 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
   uint64_t* o_done = p_full + 2;           // [2]: PV of block g commits o_done[g & 1]
   uint64_t* o_free = o_done + 2;           // [2]: output accumulator it & 1 read out
   uint64_t* mma_done = o_free + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  uint64_t* info_full = mma_done + 1;      // [4]: item bounds published by the TMA thread
+  uint64_t* info_empty = info_full + 4;    // [4]: read by the four softmax warps
+  uint64_t* out_full = info_empty + 4;     // the staging tile holds an item's output (4 warps)
+  uint64_t* out_free = out_full + 1;       // the previous TMA store has read the staging tile
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(out_free + 1);
+  int4* info = reinterpret_cast<int4*>(smem + C::OFF_INFO);
+  uint8_t* sOut = smem + C::OFF_OUT;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   auto sQ = [&](int b) { return smem + C::OFF_Q + b * C::Q_BYTES; };
   auto sK = [&](int b) { return smem + C::OFF_K + b * C::K_BYTES; };
@@ -184,11 +206,18 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       mbar_init(&v_empty[b], 1);
     }
     mbar_init(mma_done, 1);
+    for (int b = 0; b < 4; ++b) {
+      mbar_init(&info_full[b], 1);
+      mbar_init(&info_empty[b], 4);
+    }
+    mbar_init(out_full, 4);
+    mbar_init(out_free, 1);
     *abort_flag = 0;
     fence_mbar_init();
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_kv);
     tma_prefetch_desc(&tm_pre);
+    tma_prefetch_desc(&tm_out);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -215,6 +244,12 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         const int st = a.seq_start[s], len = a.seq_start[s + 1] - st;
         const int q_end = min(q0 + a.TQ, len);
         const int n_kv = n_pre + (q_end + kKeys - 1) / kKeys;
+        // the softmax warps take the item's bounds from this ring instead of
+        // reading them from global memory at every item start
+        const int is = it & 3;
+        if (!mbar_wait_bounded(&info_empty[is], ((it >> 2) & 1) ^ 1, abort_flag, err)) break;
+        info[is] = make_int4(st, len, q0, kvh);
+        mbar_arrive(&info_full[is]);
         const int qb = it & 1;
         if (!mbar_wait_bounded(&q_empty[qb], ((it >> 1) & 1) ^ 1, abort_flag, err)) break;
         mbar_arrive_expect_tx(&q_full[qb], C::Q_BYTES);
@@ -372,23 +407,55 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
     // The output of an item is read out after the next item's first block
     // (its last PV may still be running meanwhile): O / l, stored for the
     // tile's real tokens, then the accumulator is handed back to the MMA warp.
+    // A tile whose tokens all belong to its sequence is written by one TMA
+    // store of the CTA's staging tile (rows in TMEM-lane order = the box's
+    // token-major, head-minor order, 128-byte swizzle); a ragged last tile is
+    // written row by row, live rows only, since its box would reach into the
+    // next sequence's tokens.  nf counts the full-tile read-outs: the k-th
+    // waits for out_free phase k - 1 (the store of read-out k - 1 has read
+    // the staging tile) and its four warps complete out_full phase k.
     struct Pending {
-      bool on, live;
-      int buf;
+      bool on, live, full;
+      int buf, kvh, tok;
       uint32_t g_last;
       float inv;
       __half* dst;
-    } pend{false, false, 0, 0, 0.f, nullptr};
+    } pend{false, false, false, 0, 0, 0, 0, 0.f, nullptr};
+    uint32_t nf = 0;
+    const bool issuer = threadIdx.x == 64;
     auto flush = [&]() -> bool {
       if (!wait_pv(pend.g_last)) return false;
       tc_fence_after();
+      if (pend.full) {
+        if (nf > 0) {
+          if (issuer) {
+            bulk_wait_group_read<0>();
+            mbar_arrive(out_free);
+          }
+          if (!mbar_wait_bounded(out_free, (nf - 1) & 1, abort_flag, err)) return false;
+        }
+      }
       const uint32_t ocol = trow + C::O_COL + pend.buf * HD;
 #pragma unroll 1
       for (int c = 0; c < HD; c += 32) {
         uint32_t o[32];
         tmem_ld_32x32b_x32(ocol + c, o);
         tmem_ld_wait();
-        if (pend.live) {
+        if (pend.full) {
+          uint8_t* row = sOut + (c >> 6) * (128 * 128) + r * 128;
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4) {
+            uint32_t pk[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              __half2 h = __floats2half2_rn(__uint_as_float(o[q4 * 8 + 2 * i]) * pend.inv,
+                                            __uint_as_float(o[q4 * 8 + 2 * i + 1]) * pend.inv);
+              pk[i] = *reinterpret_cast<uint32_t*>(&h);
+            }
+            const int chunk = ((c & 63) >> 3) + q4;
+            *reinterpret_cast<uint4*>(row + ((chunk ^ (r & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          }
+        } else if (pend.live) {
           uint4* d4 = reinterpret_cast<uint4*>(pend.dst + c);
 #pragma unroll
           for (int q4 = 0; q4 < 4; ++q4) {
@@ -404,15 +471,34 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         }
       }
       tc_fence_before();
+      if (pend.full) fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&o_free[pend.buf]);
+      if (lane == 0) {
+        mbar_arrive(&o_free[pend.buf]);
+        if (pend.full) mbar_arrive(out_full);
+      }
+      if (pend.full) {
+        if (issuer) {
+          if (!mbar_wait_bounded(out_full, nf & 1, abort_flag, err)) return false;
+#pragma unroll
+          for (int cc = 0; cc < C::NC; ++cc) tma_store_3d(&tm_out, sOut + cc * (128 * 128), cc * 64, pend.kvh * a.G, pend.tok);
+          bulk_commit_group();
+        }
+        ++nf;
+      }
       pend.on = false;
       return true;
     };
     for (int w = blockIdx.x; w < n_work && ok; w += gridDim.x, ++it) {
-      const int tidx = w / a.Hkv, kvh = w % a.Hkv;
-      const int s = a.tile_seq[tidx], q0 = a.tile_q0[tidx];
-      const int st = a.seq_start[s], len = a.seq_start[s + 1] - st;
+      const int is = it & 3;
+      if (!mbar_wait_bounded(&info_full[is], (it >> 2) & 1, abort_flag, err)) {
+        ok = false;
+        break;
+      }
+      const int4 inf = info[is];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&info_empty[is]);
+      const int st = inf.x, len = inf.y, q0 = inf.z, kvh = inf.w;
       const int q_end = min(q0 + a.TQ, len);
       const int n_kv = n_pre + (q_end + kKeys - 1) / kKeys;
       const int qpos = q0 + t;
@@ -502,12 +588,17 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       if (!ok) break;
       pend.on = true;
       pend.live = qpos < len;
+      pend.full = q0 + a.TQ <= len;
+      pend.kvh = kvh;
+      pend.tok = st + q0;
       pend.buf = it & 1;
       pend.g_last = g - 1;
       pend.inv = l > 0.f ? 1.f / l : 0.f;
       pend.dst = a.out + static_cast<int64_t>(st + qpos) * (a.Hq * HD) + (kvh * a.G + gq) * HD;
     }
     if (ok && pend.on) flush();
+    // the CTA's shared memory must outlive the TMA stores that read it
+    if (issuer) bulk_wait_group_all();
   }
 
   __syncthreads();
@@ -555,7 +646,8 @@ bool map3d_q(CUtensorMap* m, const __half* base, int64_t T, int heads, int hd, i
 }
 
 template <int HD>
-int launch_tc(const CUtensorMap& mq, const CUtensorMap& mkv, const CUtensorMap& mpre, const AttnArgs& a,
+int launch_tc(const CUtensorMap& mq, const CUtensorMap& mkv, const CUtensorMap& mpre, const CUtensorMap& mout,
+              const AttnArgs& a,
               int n_work_max, int num_sms, cudaStream_t s) {
   using C = ACfg<HD>;
   cudaError_t e = cudaFuncSetAttribute(k_attention_tc<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
@@ -563,7 +655,7 @@ int launch_tc(const CUtensorMap& mq, const CUtensorMap& mkv, const CUtensorMap& 
   const int per_sm = C::SMEM <= 113 * 1024 ? 2 : 1;
   const int grid = n_work_max < num_sms * per_sm ? n_work_max : num_sms * per_sm;
   if (grid <= 0) return 0;
-  k_attention_tc<HD><<<grid, kThreadsTC, C::SMEM, s>>>(mq, mkv, mpre, a);
+  k_attention_tc<HD><<<grid, kThreadsTC, C::SMEM, s>>>(mq, mkv, mpre, mout, a);
   return cudaGetLastError();
 }
 
@@ -583,8 +675,10 @@ int launch_attention_tc(const __half* qkv, int64_t T, const int32_t* seq_start, 
   if (n_tiles_max <= 0 || T <= 0) return 0;
   const int G = Hq / Hkv, TQ = 128 / G;
   const int heads = Hq + 2 * Hkv;
-  CUtensorMap mq, mkv, mpre;
-  if (!map3d_q(&mq, qkv, T, heads, hd, G, TQ) || !map2d(&mkv, qkv, T, int64_t(heads) * hd)) return cudaErrorInvalidValue;
+  CUtensorMap mq, mkv, mpre, mout;
+  if (!map3d_q(&mq, qkv, T, heads, hd, G, TQ) || !map2d(&mkv, qkv, T, int64_t(heads) * hd) ||
+      !map3d_q(&mout, out, T, Hq, hd, G, TQ))
+    return cudaErrorInvalidValue;
   if (prefix_kv && P > 0) {
     if (!map2d(&mpre, prefix_kv, P, int64_t(2) * Hkv * hd)) return cudaErrorInvalidValue;
   } else {
@@ -594,8 +688,8 @@ int launch_attention_tc(const __half* qkv, int64_t T, const int32_t* seq_start, 
   AttnArgs a{seq_start, tile_seq, tile_q0, n_tiles_dev, Hq, Hkv, G, TQ, P,
              1.4426950408889634f / sqrtf(static_cast<float>(hd)), out, err};
   const int n_work_max = n_tiles_max * Hkv;
-  return hd == 64 ? launch_tc<64>(mq, mkv, mpre, a, n_work_max, num_sms, s)
-                  : launch_tc<128>(mq, mkv, mpre, a, n_work_max, num_sms, s);
+  return hd == 64 ? launch_tc<64>(mq, mkv, mpre, mout, a, n_work_max, num_sms, s)
+                  : launch_tc<128>(mq, mkv, mpre, mout, a, n_work_max, num_sms, s);
 }
 
 }  // namespace aiq
