@@ -64,8 +64,9 @@ def parse():
                    help="CPU oracle: LM candidates per step (stratified by prompt length)")
     p.add_argument("--relational-micro-rows", type=int, default=1 << 28,
                    help="rows of the predicate + compaction micro-measurement in the default line (0: skip)")
-    p.add_argument("--micro", default="", choices=["", "relational"],
-                   help="relational: predicate + compaction alone on a 2^28-row table, against HBM bandwidth")
+    p.add_argument("--micro", default="", choices=["", "relational", "attention"],
+                   help="relational: predicate + compaction alone on a 2^28-row table, against HBM bandwidth; "
+                        "attention: one prefill chunk's varlen GQA attention launch (select-query shape)")
     p.add_argument("--micro-rows", type=int, default=1 << 28)
     p.add_argument("--sweep", default="", help="selectivity sweep: 'fixed', 'lognormal' or 'both'")
     p.add_argument("--transform", type=int, default=0,
@@ -582,6 +583,61 @@ def micro_relational(args):
     ctx.close()
 
 
+def attention_micro(args):
+    """`--micro attention`: one launch of the library's varlen GQA attention
+    (aiq_op_attention) on a chunk of the select workload's shape: 970 rows of
+    lognormal length (median 120, sigma 0.5, clipped 16..512; 125,560 tokens),
+    each behind the same 64-token prefix, 32 query / 8 key-value heads of
+    head_dim 64, fp16 q/k/v of N(0, 0.25).  CUDA events around each launch on
+    the library's stream; median of `steps` launches after `warmup`.  FLOPs:
+    4 * Hq * hd per causal (query, key) pair, prefix keys included."""
+    import torch
+    from paper_2608_10139_gb300 import aiq
+    from paper_2608_10139_gb300 import build as _build
+    _build.build()
+    rng = np.random.default_rng(7)
+    lens = np.clip(np.round(np.exp(rng.normal(np.log(120.0), 0.5, 970))), 16, 512).astype(np.int64)
+    T = int(lens.sum())
+    ss = np.zeros(len(lens) + 1, np.int32)
+    np.cumsum(lens, out=ss[1:])
+    Hq, Hkv, hd, P = 32, 8, 64, 64
+    ctx = aiq.Context(0)
+    qkv = (torch.randn(T, (Hq + 2 * Hkv) * hd, device="cuda") * 0.5).half()
+    pkv = (torch.randn(P, 2 * Hkv * hd, device="cuda") * 0.5).half()
+    out = torch.empty(T, Hq * hd, device="cuda", dtype=torch.half)
+    sst = torch.as_tensor(ss).cuda()
+    torch.cuda.synchronize()
+    stream = torch.cuda.ExternalStream(ctx.stream())
+
+    def run():
+        ctx.op_attention(qkv.data_ptr(), T, sst.data_ptr(), len(lens), Hq, Hkv, hd, out.data_ptr(), pkv.data_ptr(), P)
+
+    for _ in range(max(args.warmup, 1)):
+        run()
+    clocks = ClockSampler(0)
+    clocks.start()
+    ms = []
+    for _ in range(max(args.steps, 1)):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        run()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    clk = clocks.stop()
+    med = statistics.median(ms)
+    pairs = float((lens * P + lens * (lens + 1) // 2).sum())
+    flops = 4.0 * Hq * hd * pairs
+    pk, src = peaks()
+    print(json.dumps({"metric": "attention launch time", "tokens": T, "rows": len(lens), "prefix": P,
+                      "heads": [Hq, Hkv], "head_dim": hd, "us_median": med * 1e3, "us_min": min(ms) * 1e3,
+                      "TFLOP/s": flops / (med * 1e-3) / 1e12,
+                      "frac": flops / (med * 1e-3) / 1e12 / pk["bf16_tflops"],
+                      "peak": {"bf16_tflops": pk["bf16_tflops"], "source": f"{src} bf16_tflops"},
+                      "steps": len(ms), "clocks": clk}), flush=True)
+    ctx.close()
+
+
 def sweep(args):
     """Selectivity sweep on the 1M-row table: rows/s, p50 latency and the
     relational / prefill time split at each point (one JSON line per point)."""
@@ -761,6 +817,8 @@ def main():
         reference_arm(args)
     elif args.micro == "relational":
         micro_relational(args)
+    elif args.micro == "attention":
+        attention_micro(args)
     elif args.sweep:
         sweep(args)
     elif args.transform:
