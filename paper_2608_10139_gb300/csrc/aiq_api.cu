@@ -71,7 +71,7 @@ struct TableD {
 struct LayerD {
   uint16_t* attn_norm = nullptr;
   uint16_t* mlp_norm = nullptr;
-  __half* wqkv = nullptr;  // [(Hq + 2 Hkv) hd, d], columns scaled by attn_norm's gain
+  __half* wqkv = nullptr;  // [(Hq + 2 Hkv) hd, d]
   __half* wo = nullptr;    // [d, Hq hd]
   __half* wgu = nullptr;   // [2 f, d], gate/up interleaved in blocks of bn_gu / 2 rows
   __half* wd = nullptr;    // [d, f]
@@ -496,16 +496,19 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
   const int64_t ldkv = 2 * static_cast<int64_t>(Hkv) * hd;
   const int M = static_cast<int>(T);
   // The attention-side RMSNorm is fused: the embedding and every down
-  // projection leave the residual in b.xn as fp16 with its partial sums of
-  // squares in ss_attn, and the QKV GEMM (attn_norm gain folded into its
-  // weights) scales each row by 1/RMS in its epilogue.  The MLP-side norm is
-  // a standalone kernel: fusing it into the O-projection epilogue cost more
+  // projection leave the residual times the next attention norm's gain in
+  // b.xn as fp16, with the residual's partial sums of squares in ss_attn, and
+  // the QKV GEMM scales each row by 1/RMS in its epilogue.  The gain is put on
+  // the activation, not folded into the QKV weights: a rounded weight
+  // perturbs every token alike, and over 32 layers that was the largest error
+  // of the fp16 path against the fp64 oracle.  The MLP-side norm is a
+  // standalone kernel: fusing it into the O-projection epilogue cost more
   // there than the kernel it removed.
   const int parts = d / 128;
   {
     // bf16 row in; fp32 residual, fp16 copy and the partial sums of squares out
     ProfScope p(c, "embed", 0, double(T) * d * 8.0 + double(T) * parts * 4.0);
-    launch_embed(b.tok, T, m.embed, d, b.resid, b.xn, b.ss_attn, c->d_err, c->stream);
+    launch_embed(b.tok, T, m.embed, d, b.resid, b.xn, b.ss_attn, m.layers[0].attn_norm, c->d_err, c->stream);
     counted(c, T > 0);
   }
   for (int l = 0; l < g.n_layers; ++l) {
@@ -555,6 +558,7 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
       // the down projection's epilogue prepares the next layer's attention norm
       // (b.xn is free again: the gate/up GEMM before it has consumed it)
       e2.xh_out = b.xn;
+      e2.xh_gain = l + 1 < g.n_layers ? m.layers[l + 1].attn_norm : nullptr;
       e2.ss_out = b.ss_attn;
       AIQ_TRY(gemm(c, "gemm_down_resid", b.act, f, L.wd, f, M, d, f, m.bn_d, e2));
     } else {
@@ -663,7 +667,7 @@ aiq_status decode_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const Deco
   const int parts = dm / 128;
   {
     ProfScope p(c, "embed", 0, double(R) * dm * 8.0 + double(R) * parts * 4.0);
-    launch_embed(d.next, R, m.embed, dm, b.resid, b.xn, b.ss_attn, c->d_err, c->stream);
+    launch_embed(d.next, R, m.embed, dm, b.resid, b.xn, b.ss_attn, m.layers[0].attn_norm, c->d_err, c->stream);
     counted(c, 1);
   }
   for (int l = 0; l < g.n_layers; ++l) {
@@ -717,6 +721,7 @@ aiq_status decode_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const Deco
     e3.err = c->d_err;
     AIQ_TRY(gemm(c, "dec_gemm_gateup_swiglu", b.xn, dm, L.wgu, dm, R, 2 * f, dm, m.bn_gu, e3));
     e2.xh_out = b.xn;
+    e2.xh_gain = l + 1 < g.n_layers ? m.layers[l + 1].attn_norm : nullptr;
     e2.ss_out = b.ss_attn;
     AIQ_TRY(gemm(c, "dec_gemm_down_resid", b.act, f, L.wd, f, R, dm, f, m.bn_d, e2));
   }
@@ -1642,13 +1647,13 @@ aiq_status aiq_load_model(aiq_ctx* c, const aiq_model_config* cfg, const void* c
   for (int l = 0; l < g.n_layers; ++l) {
     LayerD& L = m.layers[l];
     M_TRY(up_bf16(tensors[ti++], d, &L.attn_norm));
-    // q, k, v stacked then converted: [(Hq + 2 Hkv) hd, d], attn_norm gain folded in
+    // q, k, v stacked then converted: [(Hq + 2 Hkv) hd, d] (exact: bf16 values in fp16)
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(qd) * d * 2, cudaMemcpyHostToDevice);
     cudaMemcpy(stage + size_t(qd) * d, tensors[ti++], size_t(kd) * d * 2, cudaMemcpyHostToDevice);
     cudaMemcpy(stage + size_t(qd + kd) * d, tensors[ti++], size_t(kd) * d * 2, cudaMemcpyHostToDevice);
     M_TRY(model_alloc(c, m, size_t(qd + 2 * kd) * d, &L.wqkv));
-    launch_bf16_to_f16(stage, L.wqkv, qd + 2 * kd, d, 0, 0, L.attn_norm, c->d_err, c->stream);
+    launch_bf16_to_f16(stage, L.wqkv, qd + 2 * kd, d, 0, 0, nullptr, c->d_err, c->stream);
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(d) * qd * 2, cudaMemcpyHostToDevice);
     M_TRY(model_alloc(c, m, size_t(d) * qd, &L.wo));

@@ -212,10 +212,26 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
         add_store_f32x32(o + c + 32, v1, v1);
         if (ep.xh_out) {
           __half* xh = ep.xh_out + static_cast<int64_t>(row) * ep.ldo + n0 + c;
-          store_f16x32(xh, v0, bad);
-          store_f16x32(xh + 32, v1, bad);
 #pragma unroll
           for (int j = 0; j < 32; ++j) part += v0[j] * v0[j] + v1[j] * v1[j];
+          if (ep.xh_gain) {
+            // the next attention norm's gain goes on the activation (the QKV
+            // weights stay exact): one fp16 rounding of x * g per element
+            const uint4* g4 = reinterpret_cast<const uint4*>(ep.xh_gain + n0 + c);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              const uint4 gv = __ldg(g4 + q);
+              const uint32_t gw[4] = {gv.x, gv.y, gv.z, gv.w};
+              float* v = q < 4 ? v0 + 8 * q : v1 + 8 * (q - 4);
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                v[2 * j] *= __uint_as_float(gw[j] << 16);
+                v[2 * j + 1] *= __uint_as_float(gw[j] & 0xFFFF0000u);
+              }
+            }
+          }
+          store_f16x32(xh, v0, bad);
+          store_f16x32(xh + 32, v1, bad);
           if ((c & 127) == 64) {
             ep.ss_out[static_cast<int64_t>(row) * ep.ss_parts + (n0 + c) / 128] = part;
             part = 0.f;

@@ -29,16 +29,18 @@ struct GemmEpilogue {
   int rope_cols = 0;
   int head_dim = 0;
   int* err = nullptr;
-  // RMSNorm fused across GEMMs (the norm gain is folded into the weights):
+  // RMSNorm fused across GEMMs:
   //  - consumer (ROPE / SWIGLU): scale each accumulator row by
   //    rsqrt(sum(row_ss[row][0..ss_parts)) / d_norm + eps) before the epilogue;
-  //  - producer (RESID): also write the new residual as fp16 (xh_out) and its
-  //    per-128-column sums of squares (ss_out [row][n / 128]).
+  //  - producer (RESID): also write the new residual as fp16 (xh_out), times
+  //    the next norm's gain (xh_gain, bf16 [N]) when given, and the unscaled
+  //    residual's per-128-column sums of squares (ss_out [row][n / 128]).
   const float* row_ss = nullptr;
   int ss_parts = 0;
   float d_norm = 1.f;
   float eps = 0.f;
   __half* xh_out = nullptr;
+  const uint16_t* xh_gain = nullptr;
   float* ss_out = nullptr;
   // EPI_ARGMAX: fp32 bias [N] (-inf marks padding columns) and the per-row packed result
   const float* bias = nullptr;
@@ -124,10 +126,11 @@ void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t tile_to
 void launch_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int interleave_block,
                         int64_t half_rows, const uint16_t* gain, int* err, cudaStream_t s);
 void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, float theta, cudaStream_t s);
-// Embedding rows into the fp32 residual; with xh/ss also its fp16 copy and
-// per-128-column sums of squares (the first layer's fused RMSNorm input).
+// Embedding rows into the fp32 residual; with xh/ss also its fp16 copy (times
+// `gain`, the first layer's attention-norm gain, when given) and the unscaled
+// row's per-128-column sums of squares (the first layer's fused RMSNorm input).
 void launch_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, __half* xh, float* ss,
-                  int* err, cudaStream_t s);
+                  const uint16_t* gain, int* err, cudaStream_t s);
 // g may be null (unit gain).
 void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int* err,
                     cudaStream_t s);

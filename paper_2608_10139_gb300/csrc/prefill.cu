@@ -51,10 +51,12 @@ __global__ void k_rope_table(float* cos_t, float* sin_t, int max_pos, int hd, do
 }
 
 // One warp per token; 8 bf16 (16 bytes) per lane per step.  With xh / ss the
-// row is also written as fp16 and its sums of squares per 128 columns (16
-// lanes x 8 values) are stored, in a fixed order, for the fused RMSNorm.
+// row is also written as fp16, times the first layer's attention-norm gain
+// when `gain` is given (the fused RMSNorm's input), and its sums of squares
+// per 128 columns (16 lanes x 8 values, of the unscaled row) are stored, in a
+// fixed order.
 __global__ void k_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, __half* xh, float* ss,
-                        int* err) {
+                        const uint16_t* gain, int* err) {
   const int64_t t = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (t >= T) return;
@@ -77,10 +79,21 @@ __global__ void k_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int 
       dst[2 * c + 1] = make_float4(f[4], f[5], f[6], f[7]);
       if (xh) {
         uint32_t pk[4];
+        float gf[8] = {1.f, 1.f, 1.f, 1.f, 1.f, 1.f, 1.f, 1.f};
+        if (gain) {
+          const uint4 gv = reinterpret_cast<const uint4*>(gain)[c];
+          const uint32_t gw[4] = {gv.x, gv.y, gv.z, gv.w};
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            gf[2 * j] = __uint_as_float(gw[j] << 16);
+            gf[2 * j + 1] = __uint_as_float(gw[j] & 0xFFFF0000u);
+          }
+        }
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          bad |= !(fabsf(f[2 * j]) <= 65504.f) || !(fabsf(f[2 * j + 1]) <= 65504.f);
-          __half2 h = __floats2half2_rn(f[2 * j], f[2 * j + 1]);
+          const float a = f[2 * j] * gf[2 * j], b = f[2 * j + 1] * gf[2 * j + 1];
+          bad |= !(fabsf(a) <= 65504.f) || !(fabsf(b) <= 65504.f);
+          __half2 h = __floats2half2_rn(a, b);
           pk[j] = *reinterpret_cast<uint32_t*>(&h);
           part += f[2 * j] * f[2 * j] + f[2 * j + 1] * f[2 * j + 1];
         }
@@ -218,9 +231,9 @@ void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, fl
 }
 
 void launch_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, __half* xh, float* ss,
-                  int* err, cudaStream_t s) {
+                  const uint16_t* gain, int* err, cudaStream_t s) {
   if (T <= 0) return;
-  k_embed<<<grid_for(T * 32), 256, 0, s>>>(tok, T, emb, d, resid, xh, ss, err);
+  k_embed<<<grid_for(T * 32), 256, 0, s>>>(tok, T, emb, d, resid, xh, ss, gain, err);
 }
 
 void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int* err,
