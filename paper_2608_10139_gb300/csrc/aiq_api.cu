@@ -623,7 +623,7 @@ aiq_status ensure_lm_f16(aiq_ctx* c, ModelD& m) {
   b = static_cast<float*>(p);
   m.allocs.push_back(DevBuf{p, std::max<size_t>(static_cast<size_t>(vpad) * sizeof(float), 256)});
   CUDA_TRY(cudaMemsetAsync(w, 0, static_cast<size_t>(vpad) * g.d_model * sizeof(__half), c->stream));
-  launch_bf16_to_f16(m.lm_head, w, g.vocab, g.d_model, 0, 0, nullptr, c->d_err, c->stream);
+  launch_bf16_to_f16(m.lm_head, w, g.vocab, g.d_model, 0, 0, c->d_err, c->stream);
   launch_bias_f32(m.lm_bias, g.vocab, vpad, b, c->stream);
   counted(c, 2);
   AIQ_TRY(sync_and_check(c));
@@ -1653,21 +1653,21 @@ aiq_status aiq_load_model(aiq_ctx* c, const aiq_model_config* cfg, const void* c
     cudaMemcpy(stage + size_t(qd) * d, tensors[ti++], size_t(kd) * d * 2, cudaMemcpyHostToDevice);
     cudaMemcpy(stage + size_t(qd + kd) * d, tensors[ti++], size_t(kd) * d * 2, cudaMemcpyHostToDevice);
     M_TRY(model_alloc(c, m, size_t(qd + 2 * kd) * d, &L.wqkv));
-    launch_bf16_to_f16(stage, L.wqkv, qd + 2 * kd, d, 0, 0, nullptr, c->d_err, c->stream);
+    launch_bf16_to_f16(stage, L.wqkv, qd + 2 * kd, d, 0, 0, c->d_err, c->stream);
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(d) * qd * 2, cudaMemcpyHostToDevice);
     M_TRY(model_alloc(c, m, size_t(d) * qd, &L.wo));
-    launch_bf16_to_f16(stage, L.wo, d, qd, 0, 0, nullptr, c->d_err, c->stream);
+    launch_bf16_to_f16(stage, L.wo, d, qd, 0, 0, c->d_err, c->stream);
     M_TRY(up_bf16(tensors[ti++], d, &L.mlp_norm));
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(f) * d * 2, cudaMemcpyHostToDevice);
     cudaMemcpy(stage + size_t(f) * d, tensors[ti++], size_t(f) * d * 2, cudaMemcpyHostToDevice);
     M_TRY(model_alloc(c, m, size_t(2 * f) * d, &L.wgu));
-    launch_bf16_to_f16(stage, L.wgu, 2 * f, d, m.bn_gu / 2, f, nullptr, c->d_err, c->stream);
+    launch_bf16_to_f16(stage, L.wgu, 2 * f, d, m.bn_gu / 2, f, c->d_err, c->stream);
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(d) * f * 2, cudaMemcpyHostToDevice);
     M_TRY(model_alloc(c, m, size_t(d) * f, &L.wd));
-    launch_bf16_to_f16(stage, L.wd, d, f, 0, 0, nullptr, c->d_err, c->stream);
+    launch_bf16_to_f16(stage, L.wd, d, f, 0, 0, c->d_err, c->stream);
   }
   M_TRY(up_bf16(tensors[ti++], d, &m.final_norm));
   M_TRY(up_bf16(tensors[ti++], V * d, &m.lm_head));

@@ -120,11 +120,10 @@ void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t tile_to
                        int32_t* tile_q0, int32_t* n_tiles_dev, cudaStream_t s);
 
 // --------------------------------------------------------------- prefill ---
-// gain (optional, bf16 [cols]): dst[r][c] = fp16(src[r][c] * gain[c]), the product
-// formed exactly in fp32 and rounded once (an RMSNorm gain folded into the
-// following linear layer).
+// dst[r][c] = fp16(src[r][c]) (exact for bf16 values in fp16's range; rows
+// optionally interleaved in blocks, see k_bf16_to_f16).
 void launch_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int interleave_block,
-                        int64_t half_rows, const uint16_t* gain, int* err, cudaStream_t s);
+                        int64_t half_rows, int* err, cudaStream_t s);
 void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, float theta, cudaStream_t s);
 // Embedding rows into the fp32 residual; with xh/ss also its fp16 copy (times
 // `gain`, the first layer's attention-norm gain, when given) and the unscaled

@@ -18,7 +18,7 @@ __device__ __forceinline__ float bf16_bits_to_float(uint16_t b) {
 // matrices (gate then up) and dst rows alternate blocks of ib gate rows and
 // ib up rows, so that one GEMM output tile holds matching gate/up columns.
 __global__ void k_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int ib, int64_t half_rows,
-                              const uint16_t* gain, int* err) {
+                              int* err) {
   const int64_t n = rows * cols;
   bool bad = false;
   for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < n;
@@ -29,8 +29,7 @@ __global__ void k_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, in
       const int64_t b = r / (2 * ib), w = r % (2 * ib);
       sr = w < ib ? b * ib + w : half_rows + b * ib + (w - ib);
     }
-    float v = bf16_bits_to_float(src[sr * cols + c]);
-    if (gain) v *= bf16_bits_to_float(gain[c]);  // exact: two 8-bit significands
+    const float v = bf16_bits_to_float(src[sr * cols + c]);
     bad |= !(fabsf(v) <= 65504.f);
     dst[e] = __float2half_rn(v);
   }
@@ -214,12 +213,12 @@ inline unsigned grid_for(int64_t threads) { return static_cast<unsigned>((thread
 }  // namespace
 
 void launch_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int interleave_block,
-                        int64_t half_rows, const uint16_t* gain, int* err, cudaStream_t s) {
+                        int64_t half_rows, int* err, cudaStream_t s) {
   const int64_t n = rows * cols;
   if (n <= 0) return;
   unsigned g = grid_for(n);
   if (g > 8192) g = 8192;
-  k_bf16_to_f16<<<g, 256, 0, s>>>(src, dst, rows, cols, interleave_block, half_rows, gain, err);
+  k_bf16_to_f16<<<g, 256, 0, s>>>(src, dst, rows, cols, interleave_block, half_rows, err);
 }
 
 void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, float theta, cudaStream_t s) {
