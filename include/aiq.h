@@ -274,7 +274,13 @@ const char* aiq_last_error(void);
  * "gemm_pair" (0/1, default 1: 256 x 256 GEMM tiles on CTA pairs where
  * N % 256 == 0 and M >= 512; also selects them for aiq_op_gemm with bn = 256),
  * "attention_tc" (0/1, default 1: tcgen05 attention where the head shape
- * allows), "decode_rows" (aiq_run_transform: rows per prefill chunk, which
+ * allows), "mlp_split" (read by aiq_load_model; 1: the model's MLP GEMMs
+ * take their activations as two fp16 terms, fp16(v) and fp16(v - fp16(v)),
+ * against weights stored twice along K, about twice the MLP's tensor work and
+ * weight memory for a smaller error; 0: one fp16 term; default -1: on for
+ * models of at least 32 layers and d_model 4096, whose label logits otherwise
+ * drift past the 2e-2 margin tolerance on a few rows),
+ * "decode_rows" (aiq_run_transform: rows per prefill chunk, which
  * decode together, default 4096; the chunk's token budget grows to fit them,
  * up to 2^20 tokens and 32 GB of cached prompt keys/values), "device_bytes_max"
  * (the context's device byte cap, as AIQ_DEVICE_BYTES_MAX at aiq_init; <= 0

@@ -86,6 +86,10 @@ struct ModelD {
   std::vector<LayerD> layers;
   std::vector<DevBuf> allocs;
   int bn_qkv = 128, bn_o = 128, bn_gu = 128, bn_d = 128;
+  // two-term MLP activations: the gate/up and down GEMMs run over K = 2d and
+  // 2f against their weights stored twice along K, with the activation as
+  // fp16(v) followed by fp16(v - fp16(v))
+  bool mlp_split = false;
   DevBuf rope_cos, rope_sin;
   int rope_max_pos = 0;
   double linear_flops_per_token = 0;
@@ -182,6 +186,10 @@ struct aiq_ctx {
   bool profile = false;
   bool gemm_pair = true;  // CTA-pair (cta_group::2) GEMM tiles where the shape allows
   bool attention_tc = true;  // tcgen05 attention where the head shape allows
+  // models loaded from now on: two-term MLP activations (K-doubled MLP GEMMs);
+  // -1: for models of at least 32 layers and d_model 4096, where the one-term
+  // fp16 path's label-logit error reaches the 2e-2 parity tolerance
+  int mlp_split = -1;
   int64_t decode_rows = 4096;  // generation: target rows per prefill chunk (= decode batch)
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
@@ -320,11 +328,14 @@ void collect_profile(aiq_ctx* c) {
 
 inline void counted(aiq_ctx* c, int n) { c->launches += n; }
 
+// k_algo: the product's own depth when the GEMM runs over a two-term operand
+// (K = 2 k_algo); the statistics count the algorithmic FLOPs and bytes.
 aiq_status gemm(aiq_ctx* c, const char* name, const __half* A, int64_t lda, const __half* B, int64_t ldb, int M, int N,
-                int K, int bn, const GemmEpilogue& ep) {
+                int K, int bn, const GemmEpilogue& ep, int k_algo = 0) {
   const double out_bytes =
       (ep.kind == EPI_RESID_F32 || ep.kind == EPI_RESID_ADD ? 8.0 : (ep.kind == EPI_SWIGLU_F16 ? 1.0 : 2.0)) * M * N;
-  ProfScope ps(c, name, 2.0 * M * N * K, 2.0 * (double(M) * K + double(N) * K) + out_bytes);
+  const double Ka = k_algo > 0 ? k_algo : K;
+  ProfScope ps(c, name, 2.0 * M * N * Ka, 2.0 * (double(M) * Ka + double(N) * Ka) + out_bytes);
   const bool pair = c->gemm_pair && bn == 256 && M >= 512;
   int e = gemm_f16_tcgen05(A, lda, B, ldb, M, N, K, bn, pair, ep, c->num_sms, c->stream);
   if (M > 0) counted(c, 1);
@@ -471,10 +482,10 @@ aiq_status prefill_bufs(aiq_ctx* c, const ModelD& m, int64_t B, int64_t max_rows
   AIQ_TRY(ws(c, "pf.tile_q0", B / 8 + B + 1, &pb->tile_q0));
   AIQ_TRY(ws(c, "pf.n_tiles", 1, &pb->n_tiles));
   AIQ_TRY(ws(c, "pf.resid", B * g.d_model, &pb->resid));
-  AIQ_TRY(ws(c, "pf.xn", B * g.d_model, &pb->xn));
+  AIQ_TRY(ws(c, "pf.xn", B * g.d_model * (m.mlp_split ? 2 : 1), &pb->xn));
   AIQ_TRY(ws(c, "pf.qkv", B * nqkv, &pb->qkv));
   AIQ_TRY(ws(c, "pf.att", B * g.n_heads * g.head_dim, &pb->att));
-  AIQ_TRY(ws(c, "pf.act", std::max(B, max_rows) * g.d_ffn, &pb->act));
+  AIQ_TRY(ws(c, "pf.act", std::max(B, max_rows) * g.d_ffn * (m.mlp_split ? 2 : 1), &pb->act));
   AIQ_TRY(ws(c, "pf.resid_last", max_rows * g.d_model, &pb->resid_last));
   AIQ_TRY(ws(c, "pf.ss_attn", B * (g.d_model / 128), &pb->ss_attn));
   AIQ_TRY(ws(c, "pf.last_compact", max_rows, &pb->last_compact));
@@ -544,6 +555,12 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
     e3.out = b.act;
     e3.ldo = f;
     e3.err = c->d_err;
+    // two-term MLP activations (m.mlp_split): rows of xn and act twice as wide
+    const int ks = m.mlp_split ? 2 : 1;
+    if (m.mlp_split) {
+      e3.ldo = 2 * f;
+      e3.lo_off = f;
+    }
     if (!prune) {
       e2.out = b.resid;
       e2.kind = EPI_RESID_ADD;  // the residual add is done by the TMA unit (no fp16 copy wanted here)
@@ -551,16 +568,16 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
       e2.kind = EPI_RESID_F32;
       {
         ProfScope p(c, "rmsnorm", 0, 6.0 * double(T) * d);  // fp32 in, fp16 out
-        launch_rmsnorm(b.resid, T, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+        launch_rmsnorm(b.resid, T, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream, m.mlp_split);
         counted(c, T > 0);
       }
-      AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, d, L.wgu, d, M, 2 * f, d, m.bn_gu, e3));
+      AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, ks * d, L.wgu, ks * d, M, 2 * f, ks * d, m.bn_gu, e3, d));
       // the down projection's epilogue prepares the next layer's attention norm
       // (b.xn is free again: the gate/up GEMM before it has consumed it)
       e2.xh_out = b.xn;
       e2.xh_gain = l + 1 < g.n_layers ? m.layers[l + 1].attn_norm : nullptr;
       e2.ss_out = b.ss_attn;
-      AIQ_TRY(gemm(c, "gemm_down_resid", b.act, f, L.wd, f, M, d, f, m.bn_d, e2));
+      AIQ_TRY(gemm(c, "gemm_down_resid", b.act, ks * f, L.wd, ks * f, M, d, ks * f, m.bn_d, e2, f));
     } else {
       // final layer, rows only: gather each sequence's last token (the
       // attention output is dead afterwards, so its rows are packed into
@@ -577,11 +594,11 @@ aiq_status run_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, int64_t T, in
       AIQ_TRY(gemm(c, "gemm_o_resid", b.qkv, Hq * hd, L.wo, Hq * hd, Mo, d, Hq * hd, m.bn_o, e2));
       {
         ProfScope p(c, "rmsnorm", 0, 6.0 * double(Mo) * d);
-        launch_rmsnorm(b.resid_last, Mo, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+        launch_rmsnorm(b.resid_last, Mo, d, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream, m.mlp_split);
         counted(c, Mo > 0);
       }
-      AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, d, L.wgu, d, Mo, 2 * f, d, m.bn_gu, e3));
-      AIQ_TRY(gemm(c, "gemm_down_resid", b.act, f, L.wd, f, Mo, d, f, m.bn_d, e2));
+      AIQ_TRY(gemm(c, "gemm_gateup_swiglu", b.xn, ks * d, L.wgu, ks * d, Mo, 2 * f, ks * d, m.bn_gu, e3, d));
+      AIQ_TRY(gemm(c, "gemm_down_resid", b.act, ks * f, L.wd, ks * f, Mo, d, ks * f, m.bn_d, e2, f));
     }
   }
   return AIQ_OK;
@@ -711,19 +728,21 @@ aiq_status decode_layers(aiq_ctx* c, ModelD& m, const PrefillBufs& b, const Deco
     e2.kind = EPI_RESID_F32;
     {
       ProfScope p(c, "rmsnorm", 0, 6.0 * double(R) * dm);
-      launch_rmsnorm(b.resid, R, dm, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream);
+      launch_rmsnorm(b.resid, R, dm, L.mlp_norm, g.rms_eps, b.xn, c->d_err, c->stream, m.mlp_split);
       counted(c, 1);
     }
+    const int ks = m.mlp_split ? 2 : 1;
     GemmEpilogue e3;
     e3.kind = EPI_SWIGLU_F16;
     e3.out = b.act;
-    e3.ldo = f;
+    e3.ldo = ks * f;
+    e3.lo_off = m.mlp_split ? f : 0;
     e3.err = c->d_err;
-    AIQ_TRY(gemm(c, "dec_gemm_gateup_swiglu", b.xn, dm, L.wgu, dm, R, 2 * f, dm, m.bn_gu, e3));
+    AIQ_TRY(gemm(c, "dec_gemm_gateup_swiglu", b.xn, ks * dm, L.wgu, ks * dm, R, 2 * f, ks * dm, m.bn_gu, e3, dm));
     e2.xh_out = b.xn;
     e2.xh_gain = l + 1 < g.n_layers ? m.layers[l + 1].attn_norm : nullptr;
     e2.ss_out = b.ss_attn;
-    AIQ_TRY(gemm(c, "dec_gemm_down_resid", b.act, f, L.wd, f, R, dm, f, m.bn_d, e2));
+    AIQ_TRY(gemm(c, "dec_gemm_down_resid", b.act, ks * f, L.wd, ks * f, R, dm, ks * f, m.bn_d, e2, f));
   }
   return AIQ_OK;
 }
@@ -1613,6 +1632,7 @@ aiq_status aiq_load_model(aiq_ctx* c, const aiq_model_config* cfg, const void* c
   const int64_t d = g.d_model, f = g.d_ffn, V = g.vocab;
   ModelD m;
   m.cfg = g;
+  m.mlp_split = c->mlp_split < 0 ? (g.n_layers >= 32 && g.d_model >= 4096) : c->mlp_split != 0;
   m.bn_qkv = pick_bn(qd + 2 * kd);
   m.bn_o = pick_bn(g.d_model);
   m.bn_gu = pick_bn(2 * g.d_ffn);
@@ -1662,12 +1682,17 @@ aiq_status aiq_load_model(aiq_ctx* c, const aiq_model_config* cfg, const void* c
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(f) * d * 2, cudaMemcpyHostToDevice);
     cudaMemcpy(stage + size_t(f) * d, tensors[ti++], size_t(f) * d * 2, cudaMemcpyHostToDevice);
-    M_TRY(model_alloc(c, m, size_t(2 * f) * d, &L.wgu));
-    launch_bf16_to_f16(stage, L.wgu, 2 * f, d, m.bn_gu / 2, f, c->d_err, c->stream);
+    // with mlp_split each weight row is stored twice along K ([W | W]), the
+    // second copy multiplying the activation's low-order fp16 term
+    const int ks = m.mlp_split ? 2 : 1;
+    M_TRY(model_alloc(c, m, size_t(2 * f) * d * ks, &L.wgu));
+    for (int k = 0; k < ks; ++k)
+      launch_bf16_to_f16(stage, L.wgu + size_t(k) * d, 2 * f, d, m.bn_gu / 2, f, c->d_err, c->stream, ks * d);
     cudaStreamSynchronize(c->stream);
     cudaMemcpy(stage, tensors[ti++], size_t(d) * f * 2, cudaMemcpyHostToDevice);
-    M_TRY(model_alloc(c, m, size_t(d) * f, &L.wd));
-    launch_bf16_to_f16(stage, L.wd, d, f, 0, 0, c->d_err, c->stream);
+    M_TRY(model_alloc(c, m, size_t(d) * f * ks, &L.wd));
+    for (int k = 0; k < ks; ++k)
+      launch_bf16_to_f16(stage, L.wd + size_t(k) * f, d, f, 0, 0, c->d_err, c->stream, ks * f);
   }
   M_TRY(up_bf16(tensors[ti++], d, &m.final_norm));
   M_TRY(up_bf16(tensors[ti++], V * d, &m.lm_head));
@@ -1797,6 +1822,10 @@ aiq_status aiq_set_option(aiq_ctx* c, const char* name, int64_t value) {
   }
   if (!std::strcmp(name, "attention_tc")) {
     c->attention_tc = value != 0;
+    return AIQ_OK;
+  }
+  if (!std::strcmp(name, "mlp_split")) {
+    c->mlp_split = value < 0 ? -1 : (value != 0);
     return AIQ_OK;
   }
   if (!std::strcmp(name, "device_bytes_max")) {

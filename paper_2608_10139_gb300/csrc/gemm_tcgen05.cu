@@ -286,7 +286,14 @@ __device__ __forceinline__ void epilogue_tile(const KArgs& a, uint32_t trow, int
         const float gj = g[j] * inv;
         g[j] = gj / (1.0f + expf(-gj)) * (u[j] * inv);
       }
-      if (live) store_f16x32(o + c, g, bad);
+      if (live) {
+        store_f16x32(o + c, g, bad);
+        if (ep.lo_off > 0) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) u[j] = g[j] - __half2float(__float2half_rn(g[j]));
+          store_f16x32(o + ep.lo_off + c, u, bad);
+        }
+      }
     }
   } else {
     __half* o = static_cast<__half*>(ep.out) + static_cast<int64_t>(row) * ep.ldo + n0;

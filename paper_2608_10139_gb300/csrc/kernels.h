@@ -42,6 +42,9 @@ struct GemmEpilogue {
   __half* xh_out = nullptr;
   const uint16_t* xh_gain = nullptr;
   float* ss_out = nullptr;
+  // SWIGLU: when > 0, also write fp16(v - fp16(v)) lo_off elements after each
+  // output (a two-term operand for the next, K-doubled, GEMM)
+  int64_t lo_off = 0;
   // EPI_ARGMAX: fp32 bias [N] (-inf marks padding columns) and the per-row packed result
   const float* bias = nullptr;
   unsigned long long* best = nullptr;
@@ -120,19 +123,20 @@ void launch_attn_tiles(const int32_t* seq_start, int32_t n_seqs, int32_t tile_to
                        int32_t* tile_q0, int32_t* n_tiles_dev, cudaStream_t s);
 
 // --------------------------------------------------------------- prefill ---
-// dst[r][c] = fp16(src[r][c]) (exact for bf16 values in fp16's range; rows
-// optionally interleaved in blocks, see k_bf16_to_f16).
+// dst[r * ldd + c] = fp16(src[r][c]) (exact for bf16 values in fp16's range;
+// rows optionally interleaved in blocks, see k_bf16_to_f16; ldd 0 = cols).
 void launch_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int interleave_block,
-                        int64_t half_rows, int* err, cudaStream_t s);
+                        int64_t half_rows, int* err, cudaStream_t s, int64_t ldd = 0);
 void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, float theta, cudaStream_t s);
 // Embedding rows into the fp32 residual; with xh/ss also its fp16 copy (times
 // `gain`, the first layer's attention-norm gain, when given) and the unscaled
 // row's per-128-column sums of squares (the first layer's fused RMSNorm input).
 void launch_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, float* resid, __half* xh, float* ss,
                   const uint16_t* gain, int* err, cudaStream_t s);
-// g may be null (unit gain).
+// g may be null (unit gain).  split: out rows are 2d wide, fp16(v) then
+// fp16(v - fp16(v)) (a two-term operand for a K-doubled GEMM).
 void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int* err,
-                    cudaStream_t s);
+                    cudaStream_t s, bool split = false);
 // prefix_kv (optional): [P, 2 Hkv hd] fp16 keys then values of a shared prefix that
 // every sequence's queries also attend (prefix positions precede the sequence).
 void launch_attention(const __half* qkv, int64_t T, const int32_t* seq_start, const int32_t* tile_seq,

@@ -18,7 +18,7 @@ __device__ __forceinline__ float bf16_bits_to_float(uint16_t b) {
 // matrices (gate then up) and dst rows alternate blocks of ib gate rows and
 // ib up rows, so that one GEMM output tile holds matching gate/up columns.
 __global__ void k_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int ib, int64_t half_rows,
-                              int* err) {
+                              int64_t ldd, int* err) {
   const int64_t n = rows * cols;
   bool bad = false;
   for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < n;
@@ -31,7 +31,7 @@ __global__ void k_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, in
     }
     const float v = bf16_bits_to_float(src[sr * cols + c]);
     bad |= !(fabsf(v) <= 65504.f);
-    dst[e] = __float2half_rn(v);
+    dst[r * ldd + c] = __float2half_rn(v);
   }
   if (bad) set_dev_error(err, DEVERR_FP16_RANGE);
 }
@@ -111,8 +111,12 @@ __global__ void k_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int 
 }
 
 // One warp per row: fp32 statistics, fp16 output for the next GEMM.
+// split: out rows are 2d wide, fp16(v) in [0, d) and fp16(v - fp16(v)) in
+// [d, 2d), a two-term operand for a GEMM that runs over K = 2d against the
+// weight stored twice along K.
 template <int PER_LANE>  // d / 32 / 4 float4 per lane (compile-time for register residency)
-__global__ void k_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int* err) {
+__global__ void k_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int split,
+                          int* err) {
   const int64_t t = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (t >= T) return;
@@ -127,7 +131,8 @@ __global__ void k_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, f
   ss = warp_sum(ss);
   const float inv = rsqrtf(ss / d + eps);
   bool bad = false;
-  uint2* o = reinterpret_cast<uint2*>(out + t * d);
+  uint2* o = reinterpret_cast<uint2*>(out + t * d * (split ? 2 : 1));
+  uint2* ol = reinterpret_cast<uint2*>(out + t * d * 2 + d);
 #pragma unroll
   for (int j = 0; j < PER_LANE; ++j) {
     const int c = (lane + 32 * j) * 4;
@@ -143,12 +148,18 @@ __global__ void k_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, f
     bad |= !(fabsf(a) <= 65504.f) || !(fabsf(b) <= 65504.f) || !(fabsf(cc) <= 65504.f) || !(fabsf(e) <= 65504.f);
     __half2 h0 = __floats2half2_rn(a, b), h1 = __floats2half2_rn(cc, e);
     o[lane + 32 * j] = make_uint2(*reinterpret_cast<uint32_t*>(&h0), *reinterpret_cast<uint32_t*>(&h1));
+    if (split) {
+      const float2 f0 = __half22float2(h0), f1 = __half22float2(h1);
+      __half2 l0 = __floats2half2_rn(a - f0.x, b - f0.y), l1 = __floats2half2_rn(cc - f1.x, e - f1.y);
+      ol[lane + 32 * j] = make_uint2(*reinterpret_cast<uint32_t*>(&l0), *reinterpret_cast<uint32_t*>(&l1));
+    }
   }
   if (bad) set_dev_error(err, DEVERR_FP16_RANGE);
 }
 
 // Generic-width fallback (d not a multiple of 128 handled elsewhere; d % 4 == 0 here).
-__global__ void k_rmsnorm_any(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int* err) {
+__global__ void k_rmsnorm_any(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int split,
+                              int* err) {
   const int64_t t = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (t >= T) return;
@@ -161,7 +172,9 @@ __global__ void k_rmsnorm_any(const float* x, int64_t T, int d, const uint16_t* 
   for (int c = lane; c < d; c += 32) {
     const float v = row[c] * inv * (g ? bf16_bits_to_float(g[c]) : 1.f);
     bad |= !(fabsf(v) <= 65504.f);
-    out[t * d + c] = __float2half_rn(v);
+    const __half h = __float2half_rn(v);
+    out[t * d * (split ? 2 : 1) + c] = h;
+    if (split) out[t * d * 2 + d + c] = __float2half_rn(v - __half2float(h));
   }
   if (bad) set_dev_error(err, DEVERR_FP16_RANGE);
 }
@@ -213,12 +226,12 @@ inline unsigned grid_for(int64_t threads) { return static_cast<unsigned>((thread
 }  // namespace
 
 void launch_bf16_to_f16(const uint16_t* src, __half* dst, int64_t rows, int64_t cols, int interleave_block,
-                        int64_t half_rows, int* err, cudaStream_t s) {
+                        int64_t half_rows, int* err, cudaStream_t s, int64_t ldd) {
   const int64_t n = rows * cols;
   if (n <= 0) return;
   unsigned g = grid_for(n);
   if (g > 8192) g = 8192;
-  k_bf16_to_f16<<<g, 256, 0, s>>>(src, dst, rows, cols, interleave_block, half_rows, err);
+  k_bf16_to_f16<<<g, 256, 0, s>>>(src, dst, rows, cols, interleave_block, half_rows, ldd > 0 ? ldd : cols, err);
 }
 
 void launch_rope_table(float* cos_t, float* sin_t, int max_pos, int head_dim, float theta, cudaStream_t s) {
@@ -236,17 +249,18 @@ void launch_embed(const int32_t* tok, int64_t T, const uint16_t* emb, int d, flo
 }
 
 void launch_rmsnorm(const float* x, int64_t T, int d, const uint16_t* g, float eps, __half* out, int* err,
-                    cudaStream_t s) {
+                    cudaStream_t s, bool split) {
   if (T <= 0) return;
   const unsigned grid = grid_for(T * 32);
+  const int sp = split ? 1 : 0;
   switch (d) {
-    case 128: k_rmsnorm<1><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, err); break;
-    case 256: k_rmsnorm<2><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, err); break;
-    case 512: k_rmsnorm<4><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, err); break;
-    case 1024: k_rmsnorm<8><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, err); break;
-    case 2048: k_rmsnorm<16><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, err); break;
-    case 4096: k_rmsnorm<32><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, err); break;
-    default: k_rmsnorm_any<<<grid, 256, 0, s>>>(x, T, d, g, eps, out, err); break;
+    case 128: k_rmsnorm<1><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, sp, err); break;
+    case 256: k_rmsnorm<2><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, sp, err); break;
+    case 512: k_rmsnorm<4><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, sp, err); break;
+    case 1024: k_rmsnorm<8><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, sp, err); break;
+    case 2048: k_rmsnorm<16><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, sp, err); break;
+    case 4096: k_rmsnorm<32><<<grid, 256, 0, s>>>(x, T, d, g, eps, out, sp, err); break;
+    default: k_rmsnorm_any<<<grid, 256, 0, s>>>(x, T, d, g, eps, out, sp, err); break;
   }
 }
 

@@ -178,27 +178,15 @@ def c4_run(ctx):
 
 @pytest.mark.slow
 def test_c4_multilabel_8b_full_size(c4_run):
-    """Everything the 8B workload meets: exact candidates, token count and
-    label counts (in the fixture), decisions equal on every clear stored row,
-    and margin errors inside twice the parity tolerance on every stored row
-    (an envelope against gross numerical errors, not the parity bar; the bar
-    itself is the next test)."""
+    """The parity bar on every stored row of the 8B workload, as loaded by
+    default (two-term MLP activations for a model of 32 layers and d 4096):
+    exact candidates, token count and label counts (in the fixture), margins
+    within the tolerance and decisions equal on every clear stored row."""
     gpu, ref = c4_run
     ratio, decisions_ok = margin_ratios(gpu, ref)
     print(f"c4_multilabel_8b: {len(ratio)} stored rows, worst margin error / tolerance {ratio.max():.3f}, "
           f"{int((ratio > 1).sum())} rows above the tolerance, median {np.median(ratio):.3f}")
     assert decisions_ok, "decision mismatch on clear rows"
-    assert ratio.max() <= 2.0
-
-
-@pytest.mark.slow
-@pytest.mark.xfail(strict=True, reason="16-bit tensor-core operands over 32 layers of d 4096: a few of the 129 "
-                                       "stored rows exceed the margin tolerance (worst about 1.2x); see the "
-                                       "precision section of the design notes")
-def test_c4_multilabel_8b_margins_at_the_parity_tolerance(c4_run):
-    """The parity bar on every stored row of the 8B workload."""
-    gpu, ref = c4_run
-    ratio, _ = margin_ratios(gpu, ref)
     assert ratio.max() <= 1.0, f"{int((ratio > 1).sum())} rows above the tolerance (worst {ratio.max():.3f})"
 
 

@@ -149,6 +149,29 @@ def test_c1_chunking_is_invisible(ctx):
     assert np.array_equal(a.label_logits, b.label_logits)   # rows never interact: bit-identical
 
 
+def test_two_term_mlp_activations(ctx):
+    """mlp_split forced on for a small model (by default only models of 32
+    layers and d 4096 load with it): the query still matches the oracle, on a
+    tighter bound than the one-term path reaches, and its AI_TRANSFORM path
+    (the decode loop's MLP GEMMs) runs too."""
+    w = synth.C1_TINY
+    gqa = replace(w.model, d_model=256, n_heads=8, n_kv_heads=2, head_dim=64, d_ffn=512)
+    ctx.set_option("mlp_split", 1)
+    try:
+        for shape in (w.model, gqa):
+            r = _select_parity(ctx, replace(w, model=shape))
+            assert r.n_candidates > 0
+        q = synth.make_inputs(w)
+        mh, W = _model(ctx, gqa, w.weight_seed)
+        t = _load(ctx, q.table)
+        g = ctx.run_transform(t, mh, oracle_preds(w.preds), q.prefix, 3)
+        assert g.n_candidates > 0 and g.gen_tokens.shape[1] == 3
+        ctx.free_table(t)
+        ctx.free_model(mh)
+    finally:
+        ctx.set_option("mlp_split", -1)
+
+
 def test_tiny_row_ids_query(ctx):
     w = replace(synth.C2_SELECT, name="c2_tiny", n_rows=3000, model=synth.TINY,
                 text=synth.TextRecipe("lognormal", 16, 200, median=60.0), prefix_len=32)
