@@ -401,9 +401,13 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
     // PV of block gg done (o_done completes once per block on slot gg & 1;
     // this thread has already seen PV of block gg - 2 complete, and PV of
     // block gg + 2 needs a P that it has not yet written, so parity is exact)
-    auto wait_pv = [&](uint32_t gg) -> bool {
-      return mbar_wait_bounded(&o_done[gg & 1], (gg >> 1) & 1, abort_flag, err);
+    // Every wait of these warps is taken warp-uniformly: a lane that gives up
+    // (timeout or abort) makes the whole warp give up, so no lane is left
+    // alone in the warp-synchronous tcgen05 loads and stores that follow.
+    auto wait_all = [&](uint64_t* bar, uint32_t parity) -> bool {
+      return __all_sync(0xffffffffu, mbar_wait_bounded(bar, parity, abort_flag, err));
     };
+    auto wait_pv = [&](uint32_t gg) -> bool { return wait_all(&o_done[gg & 1], (gg >> 1) & 1); };
     // The output of an item is read out after the next item's first block
     // (its last PV may still be running meanwhile): O / l, stored for the
     // tile's real tokens, then the accumulator is handed back to the MMA warp.
@@ -432,7 +436,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
             bulk_wait_group_read<0>();
             mbar_arrive(out_free);
           }
-          if (!mbar_wait_bounded(out_free, (nf - 1) & 1, abort_flag, err)) return false;
+          if (!wait_all(out_free, (nf - 1) & 1)) return false;
         }
       }
       const uint32_t ocol = trow + C::O_COL + pend.buf * HD;
@@ -478,12 +482,18 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
         if (pend.full) mbar_arrive(out_full);
       }
       if (pend.full) {
+        // the storing thread's wait decides for its whole warp
+        bool stored = true;
         if (issuer) {
-          if (!mbar_wait_bounded(out_full, nf & 1, abort_flag, err)) return false;
+          stored = mbar_wait_bounded(out_full, nf & 1, abort_flag, err);
+          if (stored) {
 #pragma unroll
-          for (int cc = 0; cc < C::NC; ++cc) tma_store_3d(&tm_out, sOut + cc * (128 * 128), cc * 64, pend.kvh * a.G, pend.tok);
-          bulk_commit_group();
+            for (int cc = 0; cc < C::NC; ++cc)
+              tma_store_3d(&tm_out, sOut + cc * (128 * 128), cc * 64, pend.kvh * a.G, pend.tok);
+            bulk_commit_group();
+          }
         }
+        if (!__shfl_sync(0xffffffffu, stored, 0)) return false;
         ++nf;
       }
       pend.on = false;
@@ -491,7 +501,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
     };
     for (int w = blockIdx.x; w < n_work && ok; w += gridDim.x, ++it) {
       const int is = it & 3;
-      if (!mbar_wait_bounded(&info_full[is], (it >> 2) & 1, abort_flag, err)) {
+      if (!wait_all(&info_full[is], (it >> 2) & 1)) {
         ok = false;
         break;
       }
@@ -506,7 +516,7 @@ __global__ void __launch_bounds__(kThreadsTC, HD == 64 ? 2 : 1)
       float m_used = 0.f, l = 0.f;
       for (int j = 0; j < n_kv; ++j, ++g) {
         const int b = g & 1;
-        if (!mbar_wait_bounded(&s_full[b], (g >> 1) & 1, abort_flag, err)) {
+        if (!wait_all(&s_full[b], (g >> 1) & 1)) {
           ok = false;
           break;
         }
