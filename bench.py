@@ -45,7 +45,7 @@ L2_BYTES = 129 * 1024 * 1024
 # DRAM traffic of one tcgen05 GEMM launch from an ncu capture, valid only for the
 # GEMM source it was measured on (sha256 prefix of csrc/gemm_tcgen05.cu followed
 # by csrc/common.cuh, the device helpers it includes).
-GEMM_TRAFFIC = {"source_sha": "3134f6fc281edb64", "bytes_per_launch": 3.897e9}
+GEMM_TRAFFIC = {"source_sha": "e6d25c1d18b681c0", "bytes_per_launch": 3.708e9}
 
 
 def parse():

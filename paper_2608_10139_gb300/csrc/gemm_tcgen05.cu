@@ -557,7 +557,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float inv = (EPI == EPI_ROPE_F16 || EPI == EPI_SWIGLU_F16)
                             ? row_inv_rms(args.ep, m0 + quarter * 32 + lane, m0 + quarter * 32 + lane < args.M)
                             : 1.f;
-      if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
+      // warp-uniform: a lane that gives up makes the whole warp give up, so no
+      // lane is left alone in the warp-synchronous TMEM loads of the epilogue
+      if (!__all_sync(0xffffffffu, mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err))) break;
       tc_fence_after();
       const uint32_t trow = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
       if constexpr (EPI == EPI_RESID_ADD)
@@ -756,7 +758,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float inv = (EPI == EPI_ROPE_F16 || EPI == EPI_SWIGLU_F16)
                             ? row_inv_rms(args.ep, m0 + quarter * 32 + lane, m0 + quarter * 32 + lane < args.M)
                             : 1.f;
-      if (!mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err)) break;
+      // warp-uniform: a lane that gives up makes the whole warp give up, so no
+      // lane is left alone in the warp-synchronous TMEM loads of the epilogue
+      if (!__all_sync(0xffffffffu, mbar_wait_bounded(&tfull[acc], acc_ph, abort_flag, err))) break;
       tc_fence_after();
       const uint32_t trow = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + acc * BN;
       if constexpr (EPI == EPI_RESID_ADD)
