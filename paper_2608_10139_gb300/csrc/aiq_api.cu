@@ -1448,6 +1448,7 @@ void free_model(aiq_ctx* c, ModelD& m) {
 }
 
 void free_table(aiq_ctx* c, TableD& t) {
+  cudaStreamSynchronize(c->stream);  // uploads into these buffers may still be in flight
   for (auto& col : t.cols) {
     dfree(c, col.data, col.bytes);
     if (col.offsets) dfree(c, col.offsets, (t.n_rows + 1) * sizeof(int64_t));
@@ -1578,21 +1579,40 @@ aiq_status aiq_load_table(aiq_ctx* c, const aiq_column* cols, int32_t n_cols, in
         free_table(c, t);
         return st;
       }
-      cudaMemcpy(col.offsets, a.offsets, (n_rows + 1) * sizeof(int64_t), cudaMemcpyHostToDevice);
+      const cudaError_t ce =
+          cudaMemcpyAsync(col.offsets, a.offsets, (n_rows + 1) * sizeof(int64_t), cudaMemcpyHostToDevice, c->stream);
+      if (ce != cudaSuccess) {
+        cudaGetLastError();
+        cudaStreamSynchronize(c->stream);
+        dfree(c, col.offsets, (n_rows + 1) * sizeof(int64_t));
+        free_table(c, t);
+        return fail(AIQ_ERR_CUDA, std::string("table upload: ") + cudaGetErrorString(ce));
+      }
     } else {
       bytes = static_cast<size_t>(n_rows) * (a.type == AIQ_INT64 ? 8 : 4);
     }
     col.bytes = bytes;
     aiq_status st = dalloc(c, &col.data, bytes);
     if (st != AIQ_OK) {
+      cudaStreamSynchronize(c->stream);
       if (col.offsets) dfree(c, col.offsets, (n_rows + 1) * sizeof(int64_t));
       free_table(c, t);
       return st;
     }
-    if (bytes) cudaMemcpy(col.data, a.data, bytes, cudaMemcpyHostToDevice);
+    // on the context's stream: the query kernels that read the column run
+    // there, and a copy on the legacy stream from pageable memory may still
+    // be in flight when it returns
+    const cudaError_t ce = bytes ? cudaMemcpyAsync(col.data, a.data, bytes, cudaMemcpyHostToDevice, c->stream)
+                                 : cudaSuccess;
     t.cols.push_back(col);
+    if (ce != cudaSuccess) {
+      cudaGetLastError();
+      free_table(c, t);
+      return fail(AIQ_ERR_CUDA, std::string("table upload: ") + cudaGetErrorString(ce));
+    }
   }
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
     free_table(c, t);
     return fail(AIQ_ERR_CUDA, std::string("table upload: ") + cudaGetErrorString(e));
@@ -1644,6 +1664,12 @@ aiq_status aiq_load_model(aiq_ctx* c, const aiq_model_config* cfg, const void* c
     CUDA_TRY(cudaMemcpyAsync(*dst, src, count * 2, cudaMemcpyHostToDevice, c->stream));
     return AIQ_OK;
   };
+  // bf16 weights into the staging buffer, ordered on the context's stream
+  // before the conversion kernels that read them
+  auto to_stage = [&](uint16_t* dst, const void* src, size_t count) -> aiq_status {
+    CUDA_TRY(cudaMemcpyAsync(dst, src, count * 2, cudaMemcpyHostToDevice, c->stream));
+    return AIQ_OK;
+  };
   uint16_t* stage = nullptr;
   const size_t stage_elems = std::max<size_t>(2 * f * d, (size_t)(qd + 2 * kd) * d);
   void* sp = nullptr;
@@ -1669,19 +1695,19 @@ aiq_status aiq_load_model(aiq_ctx* c, const aiq_model_config* cfg, const void* c
     M_TRY(up_bf16(tensors[ti++], d, &L.attn_norm));
     // q, k, v stacked then converted: [(Hq + 2 Hkv) hd, d] (exact: bf16 values in fp16)
     cudaStreamSynchronize(c->stream);
-    cudaMemcpy(stage, tensors[ti++], size_t(qd) * d * 2, cudaMemcpyHostToDevice);
-    cudaMemcpy(stage + size_t(qd) * d, tensors[ti++], size_t(kd) * d * 2, cudaMemcpyHostToDevice);
-    cudaMemcpy(stage + size_t(qd + kd) * d, tensors[ti++], size_t(kd) * d * 2, cudaMemcpyHostToDevice);
+    M_TRY(to_stage(stage, tensors[ti++], size_t(qd) * d));
+    M_TRY(to_stage(stage + size_t(qd) * d, tensors[ti++], size_t(kd) * d));
+    M_TRY(to_stage(stage + size_t(qd + kd) * d, tensors[ti++], size_t(kd) * d));
     M_TRY(model_alloc(c, m, size_t(qd + 2 * kd) * d, &L.wqkv));
     launch_bf16_to_f16(stage, L.wqkv, qd + 2 * kd, d, 0, 0, c->d_err, c->stream);
     cudaStreamSynchronize(c->stream);
-    cudaMemcpy(stage, tensors[ti++], size_t(d) * qd * 2, cudaMemcpyHostToDevice);
+    M_TRY(to_stage(stage, tensors[ti++], size_t(d) * qd));
     M_TRY(model_alloc(c, m, size_t(d) * qd, &L.wo));
     launch_bf16_to_f16(stage, L.wo, d, qd, 0, 0, c->d_err, c->stream);
     M_TRY(up_bf16(tensors[ti++], d, &L.mlp_norm));
     cudaStreamSynchronize(c->stream);
-    cudaMemcpy(stage, tensors[ti++], size_t(f) * d * 2, cudaMemcpyHostToDevice);
-    cudaMemcpy(stage + size_t(f) * d, tensors[ti++], size_t(f) * d * 2, cudaMemcpyHostToDevice);
+    M_TRY(to_stage(stage, tensors[ti++], size_t(f) * d));
+    M_TRY(to_stage(stage + size_t(f) * d, tensors[ti++], size_t(f) * d));
     // with mlp_split each weight row is stored twice along K ([W | W]), the
     // second copy multiplying the activation's low-order fp16 term
     const int ks = m.mlp_split ? 2 : 1;
@@ -1689,7 +1715,7 @@ aiq_status aiq_load_model(aiq_ctx* c, const aiq_model_config* cfg, const void* c
     for (int k = 0; k < ks; ++k)
       launch_bf16_to_f16(stage, L.wgu + size_t(k) * d, 2 * f, d, m.bn_gu / 2, f, c->d_err, c->stream, ks * d);
     cudaStreamSynchronize(c->stream);
-    cudaMemcpy(stage, tensors[ti++], size_t(d) * f * 2, cudaMemcpyHostToDevice);
+    M_TRY(to_stage(stage, tensors[ti++], size_t(d) * f));
     M_TRY(model_alloc(c, m, size_t(d) * f * ks, &L.wd));
     for (int k = 0; k < ks; ++k)
       launch_bf16_to_f16(stage, L.wd + size_t(k) * f, d, f, 0, 0, c->d_err, c->stream, ks * f);
