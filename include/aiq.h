@@ -171,8 +171,12 @@ void aiq_shutdown(aiq_ctx* ctx);
 
 /* Table 1, FROM row: copy n_cols columns of n_rows rows to the device.
  * n_rows must be < 2^31 (row ids are int32).  Token offsets are checked
- * (monotone, in range); token ids are checked against nothing here (the model
- * check happens per query). */
+ * (start at 0, non-decreasing, fewer than 2^31 tokens); token ids must be
+ * non-negative here, and are checked against the model's vocabulary per query.
+ * The copy has completed when the call returns: the caller may free or reuse
+ * its buffers.  Errors: AIQ_ERR_INVALID_ARG (a check above, NULL data, an
+ * unknown type), AIQ_ERR_UNSUPPORTED (2^31 tokens or more), AIQ_ERR_OOM,
+ * AIQ_ERR_CUDA; on error nothing stays allocated. */
 aiq_status aiq_load_table(aiq_ctx* ctx, const aiq_column* cols, int32_t n_cols, int64_t n_rows, aiq_table* out);
 aiq_status aiq_free_table(aiq_ctx* ctx, aiq_table table);
 
