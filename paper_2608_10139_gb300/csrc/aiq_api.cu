@@ -257,7 +257,8 @@ aiq_status sync_and_check(aiq_ctx* c) {
   int err = 0;
   CUDA_TRY(cudaMemcpy(&err, c->d_err, sizeof(int), cudaMemcpyDeviceToHost));
   if (err) {
-    CUDA_TRY(cudaMemset(c->d_err, 0, sizeof(int)));
+    // cleared on the context's stream, ordered before the next call's kernels
+    CUDA_TRY(cudaMemsetAsync(c->d_err, 0, sizeof(int), c->stream));
     if (err & (DEVERR_DUP_BUILD_KEY | DEVERR_SENTINEL_KEY))
       return fail(AIQ_ERR_INVALID_ARG, "join build keys must be unique and differ from INT64_MIN");
     if (err & DEVERR_HASH_FULL) return fail(AIQ_ERR_CAPACITY, "hash table probe sequence exhausted");
@@ -1490,10 +1491,14 @@ aiq_status aiq_init(int device, aiq_ctx** out) {
   if (const char* cap = std::getenv("AIQ_DEVICE_BYTES_MAX")) c->bytes_max = std::strtoull(cap, nullptr, 10);
   cudaError_t e = cudaStreamCreateWithFlags(&c->stream, cudaStreamNonBlocking);
   if (e == cudaSuccess) e = cudaMalloc(&c->d_err, sizeof(int));
-  if (e == cudaSuccess) e = cudaMemset(c->d_err, 0, sizeof(int));
+  if (e == cudaSuccess) e = cudaMemsetAsync(c->d_err, 0, sizeof(int), c->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
   if (e == cudaSuccess) e = cudaMallocHost(&c->h_pin, 64 * sizeof(int64_t));
   if (e != cudaSuccess) {
     cudaGetLastError();
+    if (c->h_pin) cudaFreeHost(c->h_pin);
+    if (c->d_err) cudaFree(c->d_err);
+    if (c->stream) cudaStreamDestroy(c->stream);
     delete c;
     return fail(AIQ_ERR_CUDA, std::string("context setup: ") + cudaGetErrorString(e));
   }
@@ -1729,7 +1734,7 @@ aiq_status aiq_load_model(aiq_ctx* c, const aiq_model_config* cfg, const void* c
   int err = 0;
   cudaMemcpy(&err, c->d_err, sizeof(int), cudaMemcpyDeviceToHost);
   if (err) {
-    cudaMemset(c->d_err, 0, sizeof(int));
+    cudaMemsetAsync(c->d_err, 0, sizeof(int), c->stream);
     return fail_model(fail(AIQ_ERR_UNSUPPORTED, "a linear weight is outside the fp16 range"));
   }
 #undef M_TRY
