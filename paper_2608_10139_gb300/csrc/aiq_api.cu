@@ -73,8 +73,8 @@ struct LayerD {
   uint16_t* mlp_norm = nullptr;
   __half* wqkv = nullptr;  // [(Hq + 2 Hkv) hd, d]
   __half* wo = nullptr;    // [d, Hq hd]
-  __half* wgu = nullptr;   // [2 f, d], gate/up interleaved in blocks of bn_gu / 2 rows
-  __half* wd = nullptr;    // [d, f]
+  __half* wgu = nullptr;   // [2 f, d] ([2 f, 2 d] with mlp_split), gate/up interleaved in blocks of bn_gu / 2 rows
+  __half* wd = nullptr;    // [d, f] ([d, 2 f] with mlp_split)
 };
 
 struct ModelD {
